@@ -1,0 +1,421 @@
+"""Decode-step benchmark of the MLKV decode-attention library.
+
+One step = for every layer n in order: store the new token (owner layers only) then attend --
+mlkv_append_decode_attention(n) for owner layers (one launch for both), mlkv_decode_attention(n)
+for the others.  Default workload: Pythia-160M-shaped
+MLKV-2 (12 layers, 12 query heads, head_dim 64, owner layers 0 and 6 with one KV head each),
+batch 64, context 2048, bf16 Q/K/V ~ N(0,1) from a seeded generator.
+
+value   decode tokens/s of the whole job = batch * world / step time; device time of a CUDA-graph
+        replay of the step, CUDA events on the launching stream, L2 flushed (a 512 MiB write)
+        before every step outside the timed events.
+e2e     the same metric through the C ABI called from Python per layer, with the step's inputs
+        copied from pinned host memory and its outputs copied back inside the timed region.
+roofline  the decode kernel: logical K/V bytes per launch / mean launch duration (CUDA events
+        around each launch) against the measured HBM copy bandwidth.
+cpu_baseline  the fp64 oracle (test infrastructure) on the host cores, on a bounded sample.
+
+--impl reference times the oracle alone (the reference arm for this workload).
+Multi-GPU (torchrun): every rank runs an independent replica; no collective touches the data.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "decode-attn tokens/s per step (all layers); HBM GB/s vs GB300 peak"
+UNIT = "tokens/s"
+DEFAULT_WORKLOAD = "pythia160m-mlkv2-b64-L2048"
+FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class Clocks:
+    """Samples the SM clock and the clock-event (throttle) reasons through NVML while the timed
+    region runs: a background thread polls every few milliseconds, plus one sample at entry and
+    one at exit.  Read-only queries; no setting of the GPU is changed."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, index, period_s=0.005):
+        import ctypes
+        import threading
+        self.period = period_s
+        self.samples = []
+        self.max_mhz = None
+        self.stop = threading.Event()
+        self.thread = None
+        self.nvml = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            if nv.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(index), ctypes.byref(h)) != 0:
+                return
+            self.nvml, self.h = nv, h
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = float(mx.value)
+            fn = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None)
+            self.reason_fn = fn or nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        except Exception:
+            self.nvml = None
+
+    def _sample(self):
+        import ctypes
+        c = ctypes.c_uint()
+        r = ctypes.c_ulonglong()
+        if self.nvml.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(c)) != 0:
+            return
+        self.reason_fn(self.h, ctypes.byref(r))
+        self.samples.append((float(c.value), int(r.value)))
+
+    def _loop(self):
+        while not self.stop.wait(self.period):
+            self._sample()
+
+    def __enter__(self):
+        import threading
+        if self.nvml is not None:
+            self._sample()
+            self.thread = threading.Thread(target=self._loop, daemon=True)
+            self.thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        if self.nvml is not None:
+            self.stop.set()
+            self.thread.join()
+            self._sample()
+        return False
+
+    def summary(self):
+        if not self.samples:
+            return None
+        reasons = set()
+        for _, r in self.samples:
+            for bit, name in self.REASONS.items():
+                if r & bit:
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(c for c, _ in self.samples),
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(reasons),
+                "samples": len(self.samples), "source": "nvml"}
+
+
+def oracle_sample(w, rows, nthreads):
+    """Runs the oracle over every layer of the workload for the first `rows` sequences.
+
+    Returns (seconds of oracle work, sequences).  Inputs are the generator's values, built before
+    the clock starts."""
+    import oracle
+    from mlkv_synth import gen
+
+    seq_lens = w.seq_lens()[:rows]
+    L = int(seq_lens.max())
+    betas = list(range(rows))
+    caches = {}
+    for n in w.owners():
+        k = gen.bf16_bits_to_f64(gen.gen_kv(w.seed, n, 0, w.b, w.g, L, w.d, w.sigma_k, betas))
+        v = gen.bf16_bits_to_f64(gen.gen_kv(w.seed, n, 1, w.b, w.g, L, w.d, w.sigma_v, betas))
+        caches[n] = (k, v)
+    qs = [gen.bf16_bits_to_f64(gen.gen_q(w.seed, n, w.b, w.h, w.d, w.sigma_q, betas))
+          for n in range(w.l)]
+    t0 = time.perf_counter()
+    for n in range(w.l):
+        k, v = caches[w.owner[n]]
+        oracle.decode_layer(n, w.owner, w.h, w.g, w.d, seq_lens, qs[n], k, v, nthreads)
+    return time.perf_counter() - t0, rows
+
+
+def cpu_baseline(w, budget_s=12.0):
+    """Times the oracle as it stands on this host's cores over a bounded sample of sequences."""
+    nthreads = os.cpu_count() or 1
+    rows = max(1, min(w.b, nthreads))
+    t, r = oracle_sample(w, rows, nthreads)
+    # grow the sample toward the budget (the oracle's cost is linear in sequences)
+    if t < budget_s / 4 and r < w.b:
+        rows = int(min(w.b, max(r + 1, r * budget_s / 2 / max(t, 1e-3))))
+        t, r = oracle_sample(w, rows, nthreads)
+    return {"value": r / t, "unit": UNIT, "cores": nthreads, "kind": "oracle",
+            "sample": f"first {r} of {w.b} sequences, all {w.l} layers, one decode step "
+                      f"({t:.2f} s); tokens/s = sequences / oracle seconds"}
+
+
+def run_reference(args, w):
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    nthreads = os.cpu_count() or 1
+    rows = max(1, min(w.b, nthreads))
+    for _ in range(args.warmup):
+        oracle_sample(w, rows, nthreads)
+    times = []
+    for _ in range(args.steps):
+        t, r = oracle_sample(w, rows, nthreads)
+        times.append(t)
+    t = sum(times) / len(times)
+    value = rows / t
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": _config_dict(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": nthreads, "kind": "oracle",
+                         "sample": f"first {rows} of {w.b} sequences, all {w.l} layers per step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def _config_dict(w):
+    return {"workload": w.name, "layers": w.l, "q_heads": w.h, "head_dim": w.d,
+            "layer_owner": w.owner, "kv_heads_per_owner": w.g, "batch": w.b,
+            "context": "uniform[1,%d]" % w.L if w.uniform_len else w.L,
+            "l2": "flushed before every timed step (512 MiB write)", "parallelism": "replicas"}
+
+
+def kv_bytes_per_layer(w, seq_lens):
+    return int(np.sum(seq_lens, dtype=np.int64)) * w.g * w.d * 2 * 2
+
+
+def run(args, w):
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device, gen
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    seq_lens = w.seq_lens()
+    cache = mlkv.MLKVCache(w.l, w.h, w.d, w.owner, w.g, w.b, w.max_seq)
+    if args.tile:
+        cache.set_option("tile_tokens", args.tile)
+    if args.grid:
+        cache.set_option("grid", args.grid)
+    if args.l2_persist:
+        cache.set_option("l2_persist", 1)
+    owners = w.owners()
+    # owner caches: generator values at every position [0, max_seq)
+    for n in owners:
+        slot = cache.owner_slot(n)[1]
+        kp, vp, strides = cache.kv_ptr(slot)
+        device.fill_slot(kp, vp, strides, w.seed, n, w.b, w.g, w.d, w.max_seq, w.sigma_k,
+                         w.sigma_v)
+    Q = [device.q_tensor(w.seed, n, w.b, w.h, w.d, w.sigma_q) for n in range(w.l)]
+    # the new token of every owner: the generator's value at L-1 (re-appending it is idempotent)
+    Kn = {n: device.kv_token(w.seed, n, 0, w.b, w.g, w.d, seq_lens, w.sigma_k) for n in owners}
+    Vn = {n: device.kv_token(w.seed, n, 1, w.b, w.g, w.d, seq_lens, w.sigma_v) for n in owners}
+    out = [torch.empty((w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda") for _ in range(w.l)]
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+
+    def step():
+        # owner layers store their new token and attend in one launch; the others only attend
+        for n in range(w.l):
+            if n in Kn:
+                cache.append_decode_attention(n, Kn[n], Vn[n], Q[n], out[n], seq_lens)
+            else:
+                cache.decode_attention(n, Q[n], out[n], seq_lens)
+
+    launches_per_step = w.l
+    step()
+    cache.sync_status()
+
+    # ---- device-timed step: CUDA graph of the whole step --------------------------------------
+    graph = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        step()
+    torch.cuda.current_stream().wait_stream(s)
+    with torch.cuda.graph(graph):
+        step()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        graph.replay()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    with Clocks(local) as clocks:
+        for k in range(args.steps):
+            flush.zero_()
+            ev[k][0].record()
+            graph.replay()
+            ev[k][1].record()
+        barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = sum(step_ms) / len(step_ms)
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = w.b * world / (ms / 1e3)
+
+    # ---- decode kernel durations (events around every launch, step launched eagerly) ---------
+    big_flush = torch.empty(4 * FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    kev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(w.l)] for _ in range(args.steps)]
+    torch.cuda.synchronize()
+    for k in range(args.steps):
+        big_flush.zero_()      # long enough for the host to queue the whole step behind it
+        for n in range(w.l):
+            kev[k][n][0].record()
+            if n in Kn:
+                cache.append_decode_attention(n, Kn[n], Vn[n], Q[n], out[n], seq_lens)
+            else:
+                cache.decode_attention(n, Q[n], out[n], seq_lens)
+            kev[k][n][1].record()
+    torch.cuda.synchronize()
+    kms = [[a.elapsed_time(b) for a, b in row] for row in kev]
+    layer_ms = [statistics.median(kms[k][n] for k in range(args.steps)) for n in range(w.l)]
+    mean_kernel_ms = sum(layer_ms) / w.l
+    kv_layer = kv_bytes_per_layer(w, seq_lens)
+    qo_layer = 2 * w.b * w.h * w.d * 2
+    alg_bytes = kv_layer + qo_layer
+    peak, peak_kind = _peaks()
+    achieved = alg_bytes / (mean_kernel_ms / 1e3) / 1e9
+    # launches that first touch an owner's slot read it from HBM; the others may hit L2
+    cold = [layer_ms[n] for n in range(w.l) if w.owner[n] == n]
+    cold_gbs = alg_bytes / (statistics.mean(cold) / 1e3) / 1e9
+    del big_flush
+
+    # ---- end to end through the C ABI with host buffers --------------------------------------
+    host_q = torch.stack(Q).cpu().pin_memory()
+    host_k = {n: Kn[n].cpu().pin_memory() for n in owners}
+    host_v = {n: Vn[n].cpu().pin_memory() for n in owners}
+    host_out = torch.empty((w.l, w.b, w.h, w.d), dtype=torch.bfloat16).pin_memory()
+    dq = torch.empty_like(host_q, device="cuda")
+    dk = {n: torch.empty_like(host_k[n], device="cuda") for n in owners}
+    dv = {n: torch.empty_like(host_v[n], device="cuda") for n in owners}
+    dout = torch.empty_like(host_out, device="cuda")
+    h2d = host_q.numel() * 2 + sum(host_k[n].numel() * 2 * 2 for n in owners)
+    d2h = host_out.numel() * 2
+
+    def e2e_step():
+        dq.copy_(host_q, non_blocking=True)
+        for n in owners:
+            dk[n].copy_(host_k[n], non_blocking=True)
+            dv[n].copy_(host_v[n], non_blocking=True)
+        for n in range(w.l):
+            if n in dk:
+                mlkv.mlkv_append_decode_attention(cache.handle, n, dk[n], dv[n], dq[n], dout[n],
+                                                  seq_lens)
+            else:
+                mlkv.mlkv_decode_attention(cache.handle, n, dq[n], dout[n], seq_lens)
+        host_out.copy_(dout, non_blocking=True)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        e2e_step()
+    torch.cuda.synchronize()
+    e_times = []
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        e2e_step()
+        e1.record()
+        e1.synchronize()
+        e_times.append(e0.elapsed_time(e1))
+    e_ms = sum(e_times) / len(e_times)
+    if dist is not None:
+        t = torch.tensor([e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e_ms = float(t.item())
+    e2e_val = w.b * world / (e_ms / 1e3)
+    cache.sync_status()
+
+    result = None
+    if rank == 0:
+        result = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": _config_dict(w),
+            "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                    "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms},
+            "gpu_launches": launches_per_step * args.steps,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "peak_source": peak_kind,
+                         "kernel": "decode_kernel", "alg_bytes_per_launch": alg_bytes,
+                         "mean_launch_ms": mean_kernel_ms,
+                         "owner_launch_gbs": cold_gbs, "owner_launch_frac": cold_gbs / peak},
+            "step_kv_gbs": kv_layer * w.l / (ms / 1e3) / 1e9,
+            "layer_ms": layer_ms,
+            "clocks": clocks.summary(),
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            result["cpu_baseline"] = cpu_baseline(w)
+    cache.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    return result
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--config", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--tile", type=int, default=0)
+    ap.add_argument("--grid", type=int, default=0)
+    ap.add_argument("--l2-persist", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    from mlkv_synth import workloads
+    w = workloads.by_name(args.config)
+    if args.impl == "reference":
+        run_reference(args, w)
+        return
+    res = run(args, w)
+    if res is not None:
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,184 @@
+/*
+ * mlkv.h - C ABI of the GB300 (sm_103a) MLKV decode-attention library, libmlkv.so.
+ *
+ * MLKV (Zuhri et al., "MLKV: Multi-Layer Key-Value Heads for Memory Efficient Transformer
+ * Decoding", arXiv 2406.09297) shares KV heads inside a layer (query groups, Sec. 2.3 Eq. 12)
+ * and across layers (Sec. 3, Eqs. 13-18): only the m layers that own KV heads store keys and
+ * values, and every other layer reads the cache of an earlier owner layer.  This library holds
+ * that cache on one GPU and runs the per-layer single-token decode attention over it.
+ *
+ * Conventions shared by every call
+ *  - Indices are 0-based (the paper counts from 1).
+ *  - Return value: MLKV_OK (0) or a negative MLKV_ERR_* code; mlkv_last_error() then holds a
+ *    one-line description for the calling thread.  Arguments are validated on the host before any
+ *    work is queued: a call that returns an error has queued nothing.
+ *  - "device" pointers are CUDA device (or managed) memory of the cache's device; "host" pointers
+ *    are ordinary CPU memory read before the call returns.  The caller owns every buffer it
+ *    passes; device buffers must stay valid until the stream reaches the queued work.
+ *  - Tensors are bf16 (IEEE bfloat16 bit patterns), row-major, densely packed, 16-byte aligned.
+ *  - cuda_stream is a cudaStream_t (NULL = legacy default stream).  Calls are asynchronous with
+ *    respect to the host and ordered on that stream.  Calls on one cache must be ordered with
+ *    respect to each other (one stream, or explicit events): they share the cache's merge scratch.
+ *  - seq_lens (host int32[batch]) counts the token being decoded: sequence beta attends positions
+ *    [0, seq_lens[beta]), 1 <= seq_lens[beta] <= max_seq.
+ *  - No call allocates device memory except mlkv_cache_create; no call synchronises the device
+ *    except mlkv_sync_status and mlkv_cache_destroy.
+ */
+#ifndef MLKV_H_
+#define MLKV_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MLKV_OK 0
+#define MLKV_ERR_INVALID_ARG (-1) /* null handle/pointer, misaligned buffer, bad index */
+#define MLKV_ERR_MAP (-2)         /* invalid layer->owner map or head counts */
+#define MLKV_ERR_RANGE (-3)       /* a sequence length outside [1, max_seq] */
+#define MLKV_ERR_OOM (-4)         /* device allocation failed */
+#define MLKV_ERR_CUDA (-5)        /* a CUDA runtime / driver call failed */
+#define MLKV_ERR_UNSUPPORTED (-6) /* valid request outside what this build supports */
+#define MLKV_ERR_DEVICE (-7)      /* a kernel reported an error (bounded wait expired) */
+
+#define MLKV_MAX_BATCH 1024       /* largest batch a cache may hold */
+#define MLKV_MAX_GROUP 16         /* largest query group h/g per KV head */
+
+typedef struct mlkv_cache *mlkv_cache_t;
+
+/*
+ * mlkv_cache_create - validates an MLKV layout and allocates its KV cache on the current device.
+ *
+ * Paper: Sec. 3 (m owner layers, g KV heads each, cache of 2*b*s*m*g*d_k elements), Eq. 18
+ * (layer -> KV block), Eq. 12 (query head -> KV head within a layer).
+ *
+ *   out                 receives the handle (host pointer, written on success only)
+ *   n_layers            l >= 1
+ *   n_q_heads           h >= 1, query heads per layer
+ *   head_dim            d_k; 64 or 128 in this build (else MLKV_ERR_UNSUPPORTED)
+ *   layer_owner         host int32[n_layers]: layer_owner[n] is the layer whose KV heads layer n
+ *                       reads.  Must satisfy 0 <= owner[n] <= n and owner[owner[n]] == owner[n]
+ *                       (owners own themselves); Eq. 18's contiguous blocks are one such map
+ *                       (see mlkv_block_owner_map), non-uniform maps are accepted too.
+ *   kv_heads_per_owner  g, must divide h; h/g <= MLKV_MAX_GROUP
+ *   batch, max_seq      b in [1, MLKV_MAX_BATCH], s >= 1: the cache holds positions [0, max_seq)
+ *
+ * Device layout (bf16): [m][2 (K,V)][b][g][max_seq][d], slot = rank of the owner among owners.
+ * The cache starts zeroed.  Errors: MLKV_ERR_INVALID_ARG, _MAP, _UNSUPPORTED, _OOM, _CUDA.
+ */
+int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_dim,
+                      const int *layer_owner, int kv_heads_per_owner, int batch, int max_seq);
+
+/* Frees the cache and its scratch after synchronising the device.  NULL is accepted. */
+int mlkv_cache_destroy(mlkv_cache_t c);
+
+/*
+ * mlkv_append - stores the new token's keys and values of an owner layer.
+ *
+ * Paper: Sec. 2.4 (KV caching keeps the keys/values of earlier tokens) and Sec. 3 Eq. 13 (only
+ * the m owner layers have K/V projections; the other layers store nothing).
+ *
+ *   layer      0 <= layer < l.  For a layer that does not own KV heads the call returns MLKV_OK
+ *              and queues nothing.
+ *   K, V       device bf16 [batch][g][d]: the new token's key / value per sequence and KV head
+ *   seq_lens   host int32[batch]; the token is written at position seq_lens[beta] - 1
+ * Writing the same token twice at the same position is idempotent.
+ */
+int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const int *seq_lens,
+                void *cuda_stream);
+
+/*
+ * mlkv_decode_attention - single-token attention of every query head of one layer.
+ *
+ * Paper: Eqs. 2-3 (alpha = softmax(q k^T / sqrt(d_k)), o = alpha v) with the MLKV maps of
+ * Eqs. 15 and 18: query head i of layer n attends over KV head floor(i / (h/g)) of the cache
+ * slot of layer_owner[n], positions [0, seq_lens[beta]).
+ *
+ *   Q        device bf16 [batch][h][d], this layer's queries (post-projection; any positional
+ *            encoding already applied)
+ *   out      device bf16 [batch][h][d], may not alias Q; written with round-to-nearest-even
+ *   seq_lens host int32[batch], 1 <= seq_lens[beta] <= max_seq
+ * Arithmetic: bf16 inputs, fp32 accumulation and softmax, fp32 merge of split-KV partials.
+ */
+int mlkv_decode_attention(mlkv_cache_t c, int layer, const void *Q, void *out,
+                          const int *seq_lens, void *cuda_stream);
+
+/*
+ * mlkv_append_decode_attention - mlkv_append followed by mlkv_decode_attention for one layer,
+ * in one kernel launch.
+ *
+ * Paper: Sec. 3 -- an owner layer stores its new token (Eq. 13) and its query heads then attend
+ * over positions [0, L) including that token (Eqs. 2-3, 15, 18).  For a layer that owns KV heads
+ * the new token's K/V are stored at position seq_lens[beta] - 1 exactly as mlkv_append stores
+ * them; for any other layer K and V are ignored (may be NULL) and the call is
+ * mlkv_decode_attention.  Arguments as for those two calls.
+ */
+int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const void *V,
+                                 const void *Q, void *out, const int *seq_lens,
+                                 void *cuda_stream);
+
+/*
+ * mlkv_load_prefix - bulk-stores positions [0, len) of an owner layer's keys and values
+ * (prefill).  K, V: device bf16 [batch][g][len][d].  No-op (MLKV_OK) for a non-owner layer.
+ * Paper: Sec. 4.5 starts decoding from a pre-filled ("dummy") cache.
+ */
+int mlkv_load_prefix(mlkv_cache_t c, int layer, const void *K, const void *V, int len,
+                     void *cuda_stream);
+
+/* Bytes of the KV cache: 2*b*max_seq*m*g*d*2 (Sec. 3's element count times 2 bytes), or a
+ * negative error code. */
+int64_t mlkv_cache_bytes(mlkv_cache_t c);
+
+/* Number m of owner layers (Sec. 3), or a negative error code. */
+int mlkv_num_slots(mlkv_cache_t c);
+
+/* owner (host int*) receives layer_owner[layer]; slot (host int*) the cache slot of that owner. */
+int mlkv_owner_slot(mlkv_cache_t c, int layer, int *owner, int *slot);
+
+/*
+ * mlkv_kv_ptr - device addresses of one slot's K and V blocks, for bulk initialisation and
+ * inspection.  strides (host int64[4]) receives the element strides of (beta, j, t, e).
+ */
+int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t strides[4]);
+
+/*
+ * mlkv_set_option / mlkv_get_option - tuning knobs (host only, take effect on the next call):
+ *   "tile_tokens"  positions per pipeline stage: 64, 128 or 256 (d=64) / 64 or 128 (d=128);
+ *                  0 (default) picks per call: the longer tile when the mean length is >= 512
+ *   "grid"         persistent CTA count; 0 = one wave of resident CTAs (default)
+ *   "l2_persist"   1 = give each decode launch an L2 access-policy window over its owner's slot
+ *                  (default 0)
+ *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
+ *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
+ *                  run the pieces of a segment as one thread-block cluster and merge them through
+ *                  distributed shared memory; 0 = always the global-memory merge
+ * Read-only (mlkv_get_option): "sm_count", "l2_bytes", "max_grid", "ctas_per_sm", and for the most
+ * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge).
+ * Unknown keys or values return MLKV_ERR_INVALID_ARG.
+ */
+int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);
+int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value);
+
+/* Synchronises the device, then returns MLKV_ERR_DEVICE if a kernel of this cache reported an
+ * error since the last call (and clears it), MLKV_ERR_CUDA on a CUDA error, else MLKV_OK. */
+int mlkv_sync_status(mlkv_cache_t c);
+
+/* One-line description of the calling thread's most recent error ("" if none). */
+const char *mlkv_last_error(void);
+
+/*
+ * mlkv_block_owner_map - the contiguous map of Eq. 18: layer n (0-based) reads the KV heads of
+ * the bottom layer of its block, (n / (l/m)) * (l/m).  Host only.  n_owners must divide
+ * n_layers (else MLKV_ERR_MAP).  layer_owner: host int32[n_layers], written on success.
+ */
+int mlkv_block_owner_map(int n_layers, int n_owners, int *layer_owner);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int mlkv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MLKV_H_ */

@@ -1,0 +1,733 @@
+// Host side of libmlkv: argument validation, the MLKV cache manager and the C ABI of mlkv.h.
+//
+// The cache of an MLKV model (arXiv 2406.09297, Sec. 3) holds K and V only for the m owner
+// layers.  It is one device allocation laid out [m][2][b][g][max_seq][d] (bf16), so that the
+// keys (or values) of one (slot, sequence, KV head) are max_seq*d contiguous elements: a decode
+// tile of T positions is one contiguous T*d*2-byte block, fetched by a 3-D TMA tensor map over
+// (d, max_seq, m*2*b*g).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "mlkv.h"
+#include "mlkv_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return code;
+}
+
+int fail_cuda(cudaError_t e, const char *what)
+{
+    return fail(MLKV_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+using CtxGetDeviceFn = CUresult (*)(CUdevice *);
+
+template <typename Fn>
+Fn driver_entry(const char *name)
+{
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion(name, &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+        return nullptr;
+    return reinterpret_cast<Fn>(fn);
+}
+
+// The device of the CUDA context current on this thread (e.g. the one PyTorch made current);
+// falls back to this runtime's current device.
+int current_device()
+{
+    static CtxGetCurrentFn get_ctx = driver_entry<CtxGetCurrentFn>("cuCtxGetCurrent");
+    static CtxGetDeviceFn get_dev = driver_entry<CtxGetDeviceFn>("cuCtxGetDevice");
+    CUcontext ctx = nullptr;
+    if (get_ctx != nullptr && get_dev != nullptr && get_ctx(&ctx) == CUDA_SUCCESS && ctx) {
+        CUdevice dev;
+        if (get_dev(&dev) == CUDA_SUCCESS)
+            return static_cast<int>(dev);
+    }
+    int d = 0;
+    cudaGetDevice(&d);
+    return d;
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess)
+            prev = -1;
+        if (prev != dev)
+            ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard()
+    {
+        int now = -1;
+        if (prev >= 0 && cudaGetDevice(&now) == cudaSuccess && now != prev)
+            cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct mlkv_cache {
+    int l = 0, h = 0, d = 0, g = 0, G = 0, b = 0, max_seq = 0, m = 0;
+    std::vector<int> owner, slot;
+    int device = 0;
+    int sm_count = 0;
+    int l2_bytes = 0;
+    int window_max = 0;
+    size_t max_smem = 0;        // opt-in dynamic shared memory per block
+    void *cache = nullptr;      // [m][2][b][g][max_seq][d] bf16
+    size_t cache_bytes = 0;
+    float *part_o = nullptr;    // [pieces][G][d]
+    float *part_lse = nullptr;  // [pieces][G]
+    unsigned *counters = nullptr;
+    int *err = nullptr;
+    int max_ctas = 0;           // capacity of the partial buffers beyond b*g pieces
+    // options
+    int tile_tokens = 0;
+    int grid = 0;
+    int l2_persist = 0;
+    int cluster = 1;            // allow the DSMEM cluster merge
+    // the most recent decode launch (read-only options, for tests and tuning)
+    int last_grid = 0, last_tile = 0, last_cluster_k = 0;
+    // per-variant launch state
+    struct Variant {
+        const mlkv::DecodeVariant *v = nullptr;
+        CUtensorMap tmap;
+        int ctas_per_sm = 0;
+        int clusters[5] = {0, 0, 0, 0, 0};   // resident k-CTA clusters, k = 2, 4
+    };
+    std::vector<Variant> variants;
+    std::vector<int> tile_start_scratch;
+};
+
+namespace {
+
+int check_seq_lens(const mlkv_cache *c, const int *seq_lens)
+{
+    if (seq_lens == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "seq_lens is NULL");
+    for (int beta = 0; beta < c->b; ++beta) {
+        if (seq_lens[beta] < 1 || seq_lens[beta] > c->max_seq)
+            return fail(MLKV_ERR_RANGE, "seq_lens[%d] = %d outside [1, %d]", beta, seq_lens[beta],
+                        c->max_seq);
+    }
+    return MLKV_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Longer tiles move more bytes per TMA request and per barrier round trip; shorter ones waste less
+// on short sequences.  mean_len < 0 means "unknown" (reports the long-sequence choice).
+int default_tile_tokens(int d, double mean_len)
+{
+    if (d == 64)
+        return (mean_len < 0 || mean_len >= 512) ? 256 : 128;
+    return (mean_len < 0 || mean_len >= 512) ? 128 : 64;
+}
+
+mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0)
+{
+    const int T = c->tile_tokens > 0 ? c->tile_tokens : default_tile_tokens(c->d, mean_len);
+    for (auto &v : c->variants)
+        if (v.v->tile_tokens == T)
+            return &v;
+    return nullptr;
+}
+
+int encode_tmap(mlkv_cache *c, const mlkv::DecodeVariant *v, CUtensorMap *out)
+{
+    static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
+    if (encode == nullptr)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->max_seq),
+                                static_cast<cuuint64_t>(c->m) * 2 * c->b * c->g};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(c->d) * 2,
+                                   static_cast<cuuint64_t>(c->max_seq) * c->d * 2};
+    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(v->tile_tokens), 1u};
+    const cuuint32_t estr[3] = {1u, 1u, 1u};
+    CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, c->cache, dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", static_cast<int>(r));
+    return MLKV_OK;
+}
+
+void free_all(mlkv_cache *c)
+{
+    if (c->cache) cudaFree(c->cache);
+    if (c->part_o) cudaFree(c->part_o);
+    if (c->part_lse) cudaFree(c->part_lse);
+    if (c->counters) cudaFree(c->counters);
+    if (c->err) cudaFree(c->err);
+    c->cache = nullptr;
+    c->part_o = nullptr;
+    c->part_lse = nullptr;
+    c->counters = nullptr;
+    c->err = nullptr;
+}
+
+int validate_map(int l, int h, int d, const int *owner, int g, int b, int max_seq)
+{
+    if (l < 1 || h < 1 || g < 1 || b < 1 || max_seq < 1 || d < 1)
+        return fail(MLKV_ERR_INVALID_ARG,
+                    "sizes must be positive (l=%d h=%d d=%d g=%d b=%d max_seq=%d)", l, h, d, g, b,
+                    max_seq);
+    if (owner == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "layer_owner is NULL");
+    if (g > h || h % g != 0)
+        return fail(MLKV_ERR_MAP, "kv_heads_per_owner %d must divide n_q_heads %d", g, h);
+    for (int n = 0; n < l; ++n) {
+        const int o = owner[n];
+        if (o < 0 || o > n)
+            return fail(MLKV_ERR_MAP, "layer_owner[%d] = %d: an owner must be a layer <= %d", n,
+                        o, n);
+        if (owner[o] != o)
+            return fail(MLKV_ERR_MAP, "layer_owner[%d] = %d, but layer %d is not its own owner",
+                        n, o, o);
+    }
+    if (d != 64 && d != 128)
+        return fail(MLKV_ERR_UNSUPPORTED, "head_dim %d: this build supports 64 and 128", d);
+    if (h / g > MLKV_MAX_GROUP)
+        return fail(MLKV_ERR_UNSUPPORTED, "query group h/g = %d exceeds %d", h / g,
+                    MLKV_MAX_GROUP);
+    if (b > MLKV_MAX_BATCH)
+        return fail(MLKV_ERR_UNSUPPORTED, "batch %d exceeds %d", b, MLKV_MAX_BATCH);
+    return MLKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int mlkv_version(void) { return 100; }
+
+const char *mlkv_last_error(void) { return g_last_error.c_str(); }
+
+int mlkv_block_owner_map(int n_layers, int n_owners, int *layer_owner)
+{
+    if (layer_owner == nullptr || n_layers < 1 || n_owners < 1)
+        return fail(MLKV_ERR_INVALID_ARG, "bad arguments to mlkv_block_owner_map");
+    if (n_owners > n_layers || n_layers % n_owners != 0)
+        return fail(MLKV_ERR_MAP, "n_owners %d must divide n_layers %d", n_owners, n_layers);
+    const int per = n_layers / n_owners;   // layers per KV block (Eq. 18's l/m)
+    for (int n = 0; n < n_layers; ++n)
+        layer_owner[n] = (n / per) * per;
+    return MLKV_OK;
+}
+
+int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_dim,
+                      const int *layer_owner, int kv_heads_per_owner, int batch, int max_seq)
+{
+    if (out == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "out is NULL");
+    int rc = validate_map(n_layers, n_q_heads, head_dim, layer_owner, kv_heads_per_owner, batch,
+                          max_seq);
+    if (rc != MLKV_OK)
+        return rc;
+
+    mlkv_cache *c = new mlkv_cache();
+    c->l = n_layers;
+    c->h = n_q_heads;
+    c->d = head_dim;
+    c->g = kv_heads_per_owner;
+    c->G = n_q_heads / kv_heads_per_owner;
+    c->b = batch;
+    c->max_seq = max_seq;
+    c->owner.assign(layer_owner, layer_owner + n_layers);
+    c->slot.assign(n_layers, -1);
+    for (int n = 0; n < n_layers; ++n) {
+        if (c->owner[n] == n) {
+            for (int q = 0; q < n_layers; ++q)
+                if (c->owner[q] == n)
+                    c->slot[q] = c->m;
+            ++c->m;
+        }
+    }
+    const long long rows = static_cast<long long>(c->m) * 2 * c->b * c->g;
+    if (rows > 0x7fffffffLL) {
+        delete c;
+        return fail(MLKV_ERR_UNSUPPORTED, "m*2*b*g = %lld rows exceed the TMA coordinate range",
+                    rows);
+    }
+
+    c->device = current_device();
+    DeviceGuard guard(c->device);
+    cudaDeviceProp prop;
+    cudaError_t e = cudaGetDeviceProperties(&prop, c->device);
+    if (e != cudaSuccess) {
+        delete c;
+        return fail_cuda(e, "cudaGetDeviceProperties");
+    }
+    c->sm_count = prop.multiProcessorCount;
+    c->l2_bytes = prop.l2CacheSize;
+    c->window_max = prop.accessPolicyMaxWindowSize;
+    c->max_smem = prop.sharedMemPerBlockOptin;
+
+    for (int T : {64, 128, 256}) {
+        const mlkv::DecodeVariant *v = mlkv::find_decode_variant(c->d, T);
+        if (v == nullptr)
+            continue;
+        e = mlkv::prepare_decode_variant(*v, c->max_smem);
+        if (e != cudaSuccess) {
+            delete c;
+            return fail_cuda(e, "cudaFuncSetAttribute(decode)");
+        }
+        mlkv_cache::Variant var;
+        var.v = v;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&var.ctas_per_sm, v->fn, v->threads,
+                                                          v->smem_bytes);
+        if (e != cudaSuccess || var.ctas_per_sm < 1) {
+            delete c;
+            return fail(MLKV_ERR_CUDA, "decode variant d=%d T=%d cannot be resident", c->d, T);
+        }
+        c->max_ctas = std::max(c->max_ctas, var.ctas_per_sm * c->sm_count);
+        for (int k : {2, 4}) {
+            if (v->smem_bytes + (k - 1) * v->res_bytes > c->max_smem ||
+                mlkv::max_active_clusters(*v, k, &var.clusters[k]) != cudaSuccess) {
+                cudaGetLastError();
+                var.clusters[k] = 0;
+            }
+        }
+        c->variants.push_back(var);
+    }
+    c->max_ctas = std::max(c->max_ctas, 4 * c->sm_count);
+
+    c->cache_bytes = static_cast<size_t>(rows) * c->max_seq * c->d * 2;
+    const size_t pieces = static_cast<size_t>(c->b) * c->g + c->max_ctas;
+    if ((e = cudaMalloc(&c->cache, c->cache_bytes)) != cudaSuccess ||
+        (e = cudaMalloc(reinterpret_cast<void **>(&c->part_o),
+                        pieces * c->G * c->d * sizeof(float))) != cudaSuccess ||
+        (e = cudaMalloc(reinterpret_cast<void **>(&c->part_lse), pieces * c->G * sizeof(float))) !=
+            cudaSuccess ||
+        (e = cudaMalloc(reinterpret_cast<void **>(&c->counters),
+                        static_cast<size_t>(c->b) * c->g * sizeof(unsigned))) != cudaSuccess ||
+        (e = cudaMalloc(reinterpret_cast<void **>(&c->err), sizeof(int))) != cudaSuccess) {
+        cudaGetLastError();
+        free_all(c);
+        const size_t need = c->cache_bytes;
+        delete c;
+        return fail(e == cudaErrorMemoryAllocation ? MLKV_ERR_OOM : MLKV_ERR_CUDA,
+                    "cudaMalloc for a %zu-byte cache: %s", need, cudaGetErrorString(e));
+    }
+    if ((e = cudaMemset(c->cache, 0, c->cache_bytes)) != cudaSuccess ||
+        (e = cudaMemset(c->counters, 0, static_cast<size_t>(c->b) * c->g * sizeof(unsigned))) !=
+            cudaSuccess ||
+        (e = cudaMemset(c->err, 0, sizeof(int))) != cudaSuccess ||
+        (e = cudaDeviceSynchronize()) != cudaSuccess) {
+        free_all(c);
+        delete c;
+        return fail_cuda(e, "initialising the cache");
+    }
+    for (auto &var : c->variants) {
+        rc = encode_tmap(c, var.v, &var.tmap);
+        if (rc != MLKV_OK) {
+            free_all(c);
+            delete c;
+            return rc;
+        }
+    }
+    c->tile_start_scratch.resize(static_cast<size_t>(c->b) + 1);
+    *out = c;
+    return MLKV_OK;
+}
+
+int mlkv_cache_destroy(mlkv_cache_t c)
+{
+    if (c == nullptr)
+        return MLKV_OK;
+    DeviceGuard guard(c->device);
+    cudaDeviceSynchronize();
+    free_all(c);
+    delete c;
+    return MLKV_OK;
+}
+
+int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const int *seq_lens,
+                void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (layer < 0 || layer >= c->l)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->l);
+    if (c->owner[layer] != layer)
+        return MLKV_OK;   // Sec. 3: a layer without KV heads of its own stores nothing
+    if (K == nullptr || V == nullptr || !aligned16(K) || !aligned16(V))
+        return fail(MLKV_ERR_INVALID_ARG, "K and V must be non-NULL and 16-byte aligned");
+    int rc = check_seq_lens(c, seq_lens);
+    if (rc != MLKV_OK)
+        return rc;
+    mlkv::AppendParams p;
+    p.K = static_cast<const __nv_bfloat16 *>(K);
+    p.V = static_cast<const __nv_bfloat16 *>(V);
+    p.cache = static_cast<__nv_bfloat16 *>(c->cache);
+    p.b = c->b;
+    p.g = c->g;
+    p.d = c->d;
+    p.max_seq = c->max_seq;
+    p.slot = c->slot[layer];
+    std::memcpy(p.seq_len, seq_lens, sizeof(int) * c->b);
+    DeviceGuard guard(c->device);
+    cudaError_t e = mlkv::launch_append(p, static_cast<cudaStream_t>(cuda_stream));
+    if (e != cudaSuccess)
+        return fail_cuda(e, "append launch");
+    return MLKV_OK;
+}
+
+static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
+                       const void *Q, void *out, const int *seq_lens, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (layer < 0 || layer >= c->l)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->l);
+    if (Q == nullptr || out == nullptr || !aligned16(Q) || !aligned16(out))
+        return fail(MLKV_ERR_INVALID_ARG, "Q and out must be non-NULL and 16-byte aligned");
+    const size_t qbytes = static_cast<size_t>(c->b) * c->h * c->d * 2;
+    const char *qs = static_cast<const char *>(Q);
+    const char *os = static_cast<const char *>(out);
+    if (qs < os + qbytes && os < qs + qbytes)
+        return fail(MLKV_ERR_INVALID_ARG, "out overlaps Q");
+    if (K_new != nullptr && (V_new == nullptr || !aligned16(K_new) || !aligned16(V_new)))
+        return fail(MLKV_ERR_INVALID_ARG, "K and V must be non-NULL and 16-byte aligned");
+    int rc = check_seq_lens(c, seq_lens);
+    if (rc != MLKV_OK)
+        return rc;
+    double mean_len = 0.0;
+    for (int beta = 0; beta < c->b; ++beta)
+        mean_len += seq_lens[beta];
+    mean_len /= c->b;
+    mlkv_cache::Variant *var = pick_variant(c, mean_len);
+    if (var == nullptr)
+        return fail(MLKV_ERR_UNSUPPORTED, "no decode variant for d=%d tile_tokens=%d", c->d,
+                    c->tile_tokens);
+    bool uniform = true;
+    for (int beta = 1; beta < c->b; ++beta)
+        uniform = uniform && seq_lens[beta] == seq_lens[0];
+    if (!uniform && var->v->smem_bytes + mlkv::table_bytes(c->b) > c->max_smem) {
+        // The per-sequence tables do not fit beside this variant's ring: take the 64-position
+        // tile variant, whose ring is small.
+        var = nullptr;
+        for (auto &v : c->variants)
+            if (v.v->tile_tokens == 64 && v.v->smem_bytes + mlkv::table_bytes(c->b) <= c->max_smem)
+                var = &v;
+        if (var == nullptr)
+            return fail(MLKV_ERR_UNSUPPORTED, "batch %d too large for varied lengths", c->b);
+    }
+    const int T = var->v->tile_tokens;
+
+    // Stream-K style split: tiles of all (beta, j) segments end to end, equal runs per CTA.
+    static thread_local mlkv::DecodeParams p;
+    long long tiles = 0;
+    for (int beta = 0; beta < c->b; ++beta) {
+        p.tile_start[beta] = static_cast<int>(tiles);
+        p.seq_len[beta] = seq_lens[beta];
+        tiles += static_cast<long long>(c->g) * ((seq_lens[beta] + T - 1) / T);
+    }
+    p.uniform_len = uniform ? seq_lens[0] : 0;
+    if (tiles > 0x7fffffffLL)
+        return fail(MLKV_ERR_UNSUPPORTED, "%lld tiles exceed the int32 tile index", tiles);
+    p.tile_start[c->b] = static_cast<int>(tiles);
+    // Cluster mode: every segment splits into k equal pieces held by one k-CTA cluster, merged over
+    // DSMEM; taken when it keeps the one-wave makespan and every cluster is resident at once.
+    int cluster_k = 0;
+    if (uniform && c->grid == 0 && c->cluster) {
+        const long long nt = (seq_lens[0] + T - 1) / T;
+        const long long S = static_cast<long long>(c->b) * c->g;
+        const long long wave = std::min<long long>(
+            std::min(var->ctas_per_sm * c->sm_count, c->max_ctas), tiles);
+        const long long makespan = (tiles + wave - 1) / wave;
+        for (int k : {2, 4}) {
+            if (nt % k == 0 && S * k <= wave && nt / k <= makespan && var->clusters[k] >= S) {
+                cluster_k = k;
+                break;
+            }
+        }
+    }
+    int grid;
+    if (cluster_k > 1) {
+        grid = static_cast<int>(static_cast<long long>(c->b) * c->g * cluster_k);
+    } else if (c->grid > 0) {
+        grid = static_cast<int>(std::min<long long>(std::min(c->grid, c->max_ctas), tiles));
+    } else {
+        // One wave of resident CTAs sets the makespan ceil(tiles / wave); the fewest CTAs with
+        // that makespan split fewer segments (e.g. 512 tiles over 152 SMs: 128 CTAs of 4).
+        const long long wave = std::min<long long>(
+            std::min(var->ctas_per_sm * c->sm_count, c->max_ctas), tiles);
+        const long long per = (tiles + wave - 1) / wave;
+        grid = static_cast<int>((tiles + per - 1) / per);
+    }
+    grid = std::max(grid, 1);
+
+    p.Q = static_cast<const __nv_bfloat16 *>(Q);
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.K_new = static_cast<const __nv_bfloat16 *>(K_new);
+    p.V_new = static_cast<const __nv_bfloat16 *>(V_new);
+    p.cache = static_cast<__nv_bfloat16 *>(c->cache);
+    p.max_seq = c->max_seq;
+    p.part_o = c->part_o;
+    p.part_lse = c->part_lse;
+    p.counters = c->counters;
+    p.err = c->err;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
+    p.b = c->b;
+    p.h = c->h;
+    p.g = c->g;
+    p.G = c->G;
+    p.slot = c->slot[layer];
+    p.num_tiles = static_cast<int>(tiles);
+    p.cluster_k = cluster_k;
+
+    cudaAccessPolicyWindow win = {};
+    const cudaAccessPolicyWindow *winp = nullptr;
+    if (c->l2_persist && c->window_max > 0) {
+        const size_t slot_bytes = c->cache_bytes / c->m;
+        win.base_ptr = static_cast<char *>(c->cache) + slot_bytes * p.slot;
+        win.num_bytes = std::min<size_t>(slot_bytes, static_cast<size_t>(c->window_max));
+        win.hitRatio = 1.0f;
+        win.hitProp = cudaAccessPropertyPersisting;
+        win.missProp = cudaAccessPropertyStreaming;
+        winp = &win;
+    }
+    DeviceGuard guard(c->device);
+    const size_t smem = var->v->smem_bytes +
+                        (cluster_k > 1 ? (cluster_k - 1) * var->v->res_bytes
+                                       : (uniform ? 0 : mlkv::table_bytes(c->b)));
+    cudaError_t e = mlkv::launch_decode(*var->v, grid, smem, static_cast<cudaStream_t>(cuda_stream),
+                                        &var->tmap, p, winp);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "decode launch");
+    c->last_grid = grid;
+    c->last_tile = T;
+    c->last_cluster_k = cluster_k;
+    return MLKV_OK;
+}
+
+int mlkv_decode_attention(mlkv_cache_t c, int layer, const void *Q, void *out,
+                          const int *seq_lens, void *cuda_stream)
+{
+    return decode_impl(c, layer, nullptr, nullptr, Q, out, seq_lens, cuda_stream);
+}
+
+int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const void *V,
+                                 const void *Q, void *out, const int *seq_lens,
+                                 void *cuda_stream)
+{
+    if (c != nullptr && layer >= 0 && layer < c->l && c->owner[layer] == layer) {
+        if (K == nullptr || V == nullptr)
+            return fail(MLKV_ERR_INVALID_ARG, "K and V must be non-NULL for an owner layer");
+        return decode_impl(c, layer, K, V, Q, out, seq_lens, cuda_stream);
+    }
+    return decode_impl(c, layer, nullptr, nullptr, Q, out, seq_lens, cuda_stream);
+}
+
+int mlkv_load_prefix(mlkv_cache_t c, int layer, const void *K, const void *V, int len,
+                     void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (layer < 0 || layer >= c->l)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->l);
+    if (c->owner[layer] != layer)
+        return MLKV_OK;
+    if (len < 0 || len > c->max_seq)
+        return fail(MLKV_ERR_RANGE, "prefix length %d outside [0, %d]", len, c->max_seq);
+    if (len == 0)
+        return MLKV_OK;
+    if (K == nullptr || V == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "K and V must be non-NULL");
+    DeviceGuard guard(c->device);
+    const size_t row = static_cast<size_t>(len) * c->d * 2;
+    const size_t pitch = static_cast<size_t>(c->max_seq) * c->d * 2;
+    const size_t slot_bytes = c->cache_bytes / c->m;
+    char *base = static_cast<char *>(c->cache) + slot_bytes * c->slot[layer];
+    const size_t rows = static_cast<size_t>(c->b) * c->g;
+    cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    cudaError_t e = cudaMemcpy2DAsync(base, pitch, K, row, row, rows, cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpy2DAsync(base + slot_bytes / 2, pitch, V, row, row, rows,
+                              cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "prefix copy");
+    return MLKV_OK;
+}
+
+int64_t mlkv_cache_bytes(mlkv_cache_t c)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    return static_cast<int64_t>(c->cache_bytes);
+}
+
+int mlkv_num_slots(mlkv_cache_t c)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    return c->m;
+}
+
+int mlkv_owner_slot(mlkv_cache_t c, int layer, int *owner, int *slot)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (layer < 0 || layer >= c->l)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->l);
+    if (owner) *owner = c->owner[layer];
+    if (slot) *slot = c->slot[layer];
+    return MLKV_OK;
+}
+
+int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t strides[4])
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (slot < 0 || slot >= c->m)
+        return fail(MLKV_ERR_INVALID_ARG, "slot %d outside [0, %d)", slot, c->m);
+    const size_t slot_bytes = c->cache_bytes / c->m;
+    char *base = static_cast<char *>(c->cache) + slot_bytes * slot;
+    if (k_base) *k_base = base;
+    if (v_base) *v_base = base + slot_bytes / 2;
+    if (strides) {
+        strides[3] = 1;
+        strides[2] = c->d;
+        strides[1] = static_cast<int64_t>(c->max_seq) * c->d;
+        strides[0] = static_cast<int64_t>(c->g) * c->max_seq * c->d;
+    }
+    return MLKV_OK;
+}
+
+int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
+{
+    if (c == nullptr || key == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null argument");
+    if (std::strcmp(key, "tile_tokens") == 0) {
+        if (value != 0 && mlkv::find_decode_variant(c->d, static_cast<int>(value)) == nullptr)
+            return fail(MLKV_ERR_INVALID_ARG, "tile_tokens %lld not built for d=%d",
+                        static_cast<long long>(value), c->d);
+        c->tile_tokens = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "grid") == 0) {
+        if (value < 0 || value > c->max_ctas)
+            return fail(MLKV_ERR_INVALID_ARG, "grid %lld outside [0, %d]",
+                        static_cast<long long>(value), c->max_ctas);
+        c->grid = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_persist") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "l2_persist must be 0 or 1");
+        c->l2_persist = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "cluster") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "cluster must be 0 or 1");
+        c->cluster = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    return fail(MLKV_ERR_INVALID_ARG, "unknown option '%s'", key);
+}
+
+int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
+{
+    if (c == nullptr || key == nullptr || value == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null argument");
+    if (std::strcmp(key, "tile_tokens") == 0) {
+        *value = c->tile_tokens;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "grid") == 0) {
+        *value = c->grid;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_persist") == 0) {
+        *value = c->l2_persist;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "cluster") == 0) {
+        *value = c->cluster;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_grid") == 0) {
+        *value = c->last_grid;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_tile_tokens") == 0) {
+        *value = c->last_tile;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_cluster_k") == 0) {
+        *value = c->last_cluster_k;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "max_grid") == 0) {
+        *value = c->max_ctas;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "sm_count") == 0) {
+        *value = c->sm_count;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_bytes") == 0) {
+        *value = c->l2_bytes;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "ctas_per_sm") == 0) {
+        mlkv_cache::Variant *var = pick_variant(c);
+        *value = var ? var->ctas_per_sm : 0;
+        return MLKV_OK;
+    }
+    return fail(MLKV_ERR_INVALID_ARG, "unknown option '%s'", key);
+}
+
+int mlkv_sync_status(mlkv_cache_t c)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    DeviceGuard guard(c->device);
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess)
+        return fail_cuda(e, "cudaDeviceSynchronize");
+    int word = 0;
+    e = cudaMemcpy(&word, c->err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "reading the device error word");
+    if (word != 0) {
+        // A kernel stopped early: clear the word and the merge counters it may have left behind.
+        cudaMemset(c->err, 0, sizeof(int));
+        cudaMemset(c->counters, 0, static_cast<size_t>(c->b) * c->g * sizeof(unsigned));
+        cudaDeviceSynchronize();
+        return fail(MLKV_ERR_DEVICE, "a kernel reported device error bits 0x%x", word);
+    }
+    return MLKV_OK;
+}
+
+}  // extern "C"

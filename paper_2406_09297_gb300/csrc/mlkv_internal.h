@@ -1,0 +1,81 @@
+// Internal interface between the host side of libmlkv (mlkv_host.cpp) and its kernels
+// (mlkv_kernels.cu).  Not part of the public ABI (include/mlkv.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mlkv.h"
+
+namespace mlkv {
+
+// Error bits a kernel ORs into the cache's device error word.
+enum : int {
+    kErrWaitFull = 1,   // a consumer gave up waiting for a K/V tile
+    kErrWaitEmpty = 2,  // the producer gave up waiting for a free stage
+    kErrDrain = 4,      // the producer gave up waiting for its last copies at exit
+};
+
+// Split-KV decode of one layer.  Passed by value (__grid_constant__), so a launch needs no
+// device-side metadata and is stream-ordered and graph-capturable by construction.
+struct DecodeParams {
+    const __nv_bfloat16 *Q;   // [b][h][D]
+    __nv_bfloat16 *out;       // [b][h][D]
+    const __nv_bfloat16 *K_new;   // fused append: new token [b][g][D], or nullptr
+    const __nv_bfloat16 *V_new;
+    __nv_bfloat16 *cache;     // [m][2][b][g][max_seq][D] (written only by the fused append)
+    int max_seq;
+    float *part_o;            // [pieces][G][D]  normalised partial outputs
+    float *part_lse;          // [pieces][G]     log2-domain log-sum-exp of each partial
+    unsigned *counters;       // [b*g]           pieces finished per segment; zero between launches
+    int *err;                 // device error word
+    float scale_log2;         // log2(e) / sqrt(D)
+    int b, h, g, G, slot;
+    int num_tiles;            // total tiles over all (beta, j) segments
+    int uniform_len;          // the common length when every sequence has the same, else 0
+    int cluster_k;            // > 1: clusters of k CTAs, one segment each, merged over DSMEM
+    int seq_len[MLKV_MAX_BATCH];
+    int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
+};
+
+struct AppendParams {
+    const __nv_bfloat16 *K;   // [b][g][D]
+    const __nv_bfloat16 *V;
+    __nv_bfloat16 *cache;     // [m][2][b][g][max_seq][D]
+    int b, g, d, max_seq, slot;
+    int seq_len[MLKV_MAX_BATCH];
+};
+
+// Static description of one compiled decode variant.
+struct DecodeVariant {
+    int head_dim;
+    int tile_tokens;
+    int stages;
+    int threads;
+    size_t smem_bytes;        // without the per-sequence tables (see table_bytes)
+    size_t res_bytes;         // one piece result slot (cluster mode adds k-1 of them)
+    const void *fn;
+};
+
+// Shared memory a launch adds for the per-sequence tables (only when lengths differ).
+inline size_t table_bytes(int batch) { return ((8 * static_cast<size_t>(batch) + 4) + 15) & ~15ull; }
+
+// Returns the compiled variant for (head_dim, tile_tokens), or nullptr.
+const DecodeVariant *find_decode_variant(int head_dim, int tile_tokens);
+
+// Raises the variant's dynamic shared-memory limit (capped at max_smem, the device's opt-in
+// per-block maximum); call once per device before the first launch.
+cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem);
+
+cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
+                          const CUtensorMap *tmap, const DecodeParams &p,
+                          const cudaAccessPolicyWindow *window);
+
+// How many k-CTA clusters of this variant can be resident at once.
+cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out);
+
+cudaError_t launch_append(const AppendParams &p, cudaStream_t stream);
+
+}  // namespace mlkv

@@ -1,0 +1,1186 @@
+// MLKV decode-attention kernels for GB300 (sm_103a).
+//
+// decode_kernel: single-token attention of one layer over the cache slot of the layer's owner
+// (MLKV, arXiv 2406.09297, Sec. 3 Eqs. 13-18, attention of Eqs. 2-3).
+//
+//   Work split.  A "segment" is one (sequence beta, KV head j) pair: positions [0, L_beta) of one
+//   K/V head, read by the G = h/g query heads of its group (Eq. 15).  Segments are cut into tiles
+//   of T positions and all tiles of the layer are laid end to end (beta-major, j inside).  A
+//   persistent grid of P CTAs takes equal contiguous runs of that tile list, so every CTA streams
+//   the same number of bytes whatever the length mix.  The part of a segment inside one CTA's run
+//   is a "piece"; a CTA that holds a whole segment writes its output directly, otherwise it
+//   writes a normalised partial (o, log-sum-exp) and the last CTA to finish the segment (an atomic
+//   counter, no spinning) merges the partials.
+//
+//   Data movement.  One producer warp issues TMA tensor copies (cp.async.bulk.tensor, 128-byte
+//   swizzle) of each K and V tile into a STAGES-deep shared-memory ring, completion tracked by
+//   mbarrier transaction counts.  Each tile is fetched from HBM exactly once and used by all G
+//   query heads of the group.
+//
+//   Math.  NCW consumer warps (4 or 8) split every tile by positions.  Scores S = Q K^T and the
+//   update
+//   O += P V run on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate) with the
+//   query group padded to M = 16 rows; the softmax is online, in fp32, base 2 with the 1/sqrt(d)
+//   scale folded into the exponent, with quad shuffles for row maxima.  The warps' states are
+//   merged through shared memory at the end of each piece.
+//
+//   Launch.  Programmatic dependent launch: barrier set-up overlaps the previous kernel of the
+//   stream, and no global memory is touched before griddepcontrol.wait.
+//
+// append_kernel: stores the new token's K/V of an owner layer at position L_beta - 1.
+//
+// Every wait on an mbarrier is bounded (about 2 s); on expiry the kernel sets a bit in the
+// device error word, stops issuing copies, keeps its barrier sequence intact, drains the copies
+// it already issued and exits.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mlkv_internal.h"
+
+namespace mlkv {
+namespace {
+
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// ------------------------------------------------------------------------------------------------
+// PTX wrappers
+// ------------------------------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+// Waits for the phase of the given parity to complete; false after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+{
+    if (mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try_wait(bar, parity))
+                return true;
+        if (global_timer_ns() - t0 > kWaitLimitNs)
+            return false;
+    }
+}
+
+__device__ __forceinline__ void fence_barrier_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Orders this thread's generic-proxy shared-memory writes before later async-proxy (TMA) ones.
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
+                                            int x, int y, int z)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map)
+{
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                        uint32_t &r3)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t &r0, uint32_t &r1,
+                                              uint32_t &r2, uint32_t &r3)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+// D = A(16x16, row) * B(16x8, col) + D, bf16 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1)
+{
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// 2^x with the SFU instruction (2^-inf = 0).
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float fast_rcp(float x)
+{
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float fast_log2(float x)
+{
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+template <int NCW>
+__device__ __forceinline__ void consumer_bar_sync()
+{
+    asm volatile("bar.sync 1, %0;" ::"n"(NCW * 32) : "memory");
+}
+
+// Programmatic dependent launch: wait until the previous kernel of the stream has completed and
+// its memory is visible; allow the next kernel of the stream to start its prologue.
+__device__ __forceinline__ void grid_dependency_wait()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+__device__ __forceinline__ void grid_dependents_launch()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// ------------------------------------------------------------------------------------------------
+// tile walk: flattened tile index -> (beta, j, tile within segment)
+// ------------------------------------------------------------------------------------------------
+
+// With one length for every sequence (uniform_len > 0) the walk is arithmetic; otherwise it reads
+// the per-sequence tables, which the kernel copies from its parameters into shared memory.
+template <int T>
+struct TileWalk {
+    int beta, j, tt, nt, L, seg_first;
+
+    __device__ __forceinline__ void init(const DecodeParams &p, const int *s_len,
+                                         const int *s_start, int tile)
+    {
+        if (p.uniform_len > 0) {
+            L = p.uniform_len;
+            nt = (L + T - 1) / T;
+            const int seg = tile / nt;
+            tt = tile - seg * nt;
+            beta = seg / p.g;
+            j = seg - beta * p.g;
+            seg_first = seg * nt;
+            return;
+        }
+        int lo = 0, hi = p.b - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_start[mid] <= tile)
+                lo = mid;
+            else
+                hi = mid - 1;
+        }
+        beta = lo;
+        L = s_len[beta];
+        nt = (L + T - 1) / T;
+        const int rel = tile - s_start[beta];
+        j = rel / nt;
+        tt = rel - j * nt;
+        seg_first = s_start[beta] + j * nt;
+    }
+
+    __device__ __forceinline__ void next(const DecodeParams &p, const int *s_len,
+                                         const int *s_start)
+    {
+        if (++tt < nt)
+            return;
+        tt = 0;
+        if (p.uniform_len > 0) {
+            seg_first += nt;
+            if (++j == p.g) {
+                j = 0;
+                ++beta;
+            }
+            return;
+        }
+        if (++j == p.g) {
+            j = 0;
+            if (++beta < p.b) {
+                L = s_len[beta];
+                nt = (L + T - 1) / T;
+            }
+        }
+        seg_first = (beta < p.b) ? s_start[beta] + j * nt : p.num_tiles;
+    }
+};
+
+// CTA whose contiguous tile run [floor(c*N/P), floor((c+1)*N/P)) contains `tile`.
+__device__ __forceinline__ int cta_of_tile(int tile, int N, int P)
+{
+    return static_cast<int>((static_cast<long long>(tile + 1) * P - 1) / N);
+}
+
+// ------------------------------------------------------------------------------------------------
+// shared-memory plan
+// ------------------------------------------------------------------------------------------------
+
+template <int D, int T, int STAGES, int NCW>
+struct Plan {
+    static constexpr int kThreads = (NCW + 2) * 32;   // consumers, one producer, one epilogue warp
+    static constexpr int kProducer = NCW;             // warp indices
+    static constexpr int kEpilogue = NCW + 1;
+    static constexpr int kSub = D / 64;               // 128-byte-wide column blocks per row
+    static constexpr int kTW = T / NCW;               // positions per warp per tile
+    static constexpr int kTileBytes = T * D * 2;      // one K (or V) tile
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kWarpFrag = D * 64;          // one warp's O fragments: D/8*4 f32 x 32
+    static constexpr int kResO = 16 * D * 4;          // a piece's result: o[16][D] f32
+    static constexpr int kResBytes = kResO + 16 * 4 + 32;   // + lse[16] + 8 ints of metadata
+    static constexpr int kMerge = STAGES * kStageBytes;                 // [NCW/2][kWarpFrag]
+    static constexpr int kRes = kMerge + (NCW / 2) * kWarpFrag;        // [2][kResBytes]
+    static constexpr int kEpiW = kRes + 2 * kResBytes;                 // f32 [kEpiCap] weights
+    static constexpr int kEpiCap = 512;
+    static constexpr int kRedM = kEpiW + kEpiCap * 4;                  // f32 [NCW][16]
+    static constexpr int kRedL = kRedM + NCW * 16 * 4;                 // f32 [NCW][16]
+    static constexpr int kFlags = kRedL + NCW * 16 * 4;                // int [4]
+    // u64 full[S], empty[S], res_full[2], res_empty[2], cluster
+    static constexpr int kBars = kFlags + 16;
+    // Dynamic tail: per-sequence tables (lengths differ) or, in cluster mode, the leader's
+    // slots for the other ranks' results ([k-1][kResBytes]).
+    static constexpr int kTables = kBars + (2 * STAGES + 5) * 8 + 8;
+    static constexpr int kBytes = kTables;
+    static constexpr int kAlloc = kBytes + 1024;      // base aligned up to 1024 in the kernel
+    static_assert(kTW % 16 == 0, "each warp takes whole 16-position mma steps");
+    static_assert(NCW == 4 || NCW == 8, "tree merge over 4 or 8 warps");
+    static_assert(D == 64 || D == 128, "head_dim 64 or 128");
+    static_assert(T <= 256, "TMA box height");
+    static_assert(kResBytes % 16 == 0, "result slots stay 16-byte aligned");
+};
+
+// Byte offset of 16-byte chunk `chunk` (0 .. D/8-1) of row `row` inside a K or V tile laid out by
+// the TMA 128-byte swizzle: the chunk index within a 128-byte row is XORed with (row mod 8).
+template <int T>
+__device__ __forceinline__ uint32_t swz(int row, int chunk)
+{
+    const int sub = chunk >> 3;
+    const int c = chunk & 7;
+    return static_cast<uint32_t>(sub * T * 128 + row * 128 + ((c ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+                 ::: "memory");
+}
+
+// Address, in the cluster's shared window, of this CTA's shared address `a` in CTA `rank`.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t a, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void st_cluster_v4(uint32_t a, float4 v)
+{
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(v.x), "f"(v.y),
+                 "f"(v.z), "f"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ void st_cluster_f32(uint32_t a, float v)
+{
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
+}
+
+__device__ __forceinline__ void fence_acq_rel_cluster()
+{
+    asm volatile("fence.acq_rel.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity)
+{
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity)
+{
+    if (mbar_try_wait_cluster(bar, parity))
+        return true;
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try_wait_cluster(bar, parity))
+                return true;
+        if (global_timer_ns() - t0 > kWaitLimitNs)
+            return false;
+    }
+}
+
+__device__ __forceinline__ unsigned atomic_add_acq_rel_gpu(unsigned *addr, unsigned v)
+{
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "l"(addr), "r"(v)
+                 : "memory");
+    return old;
+}
+
+enum : int { kMetaBeta = 0, kMetaJ, kMetaSeg, kMetaWhole, kMetaFirst, kMetaLast, kMetaStop };
+
+// ------------------------------------------------------------------------------------------------
+// epilogue warp: output, partials and the cross-CTA merge of finished pieces
+// ------------------------------------------------------------------------------------------------
+
+// One piece's result (normalised o, lse, metadata) sits in a shared-memory slot.  A whole segment
+// goes straight to `out`.  Otherwise the slot becomes partial record seg + cta; the counter of the
+// segment (acquire-release) tells the CTA that finished it last, which merges all its records:
+//   o = sum_c 2^(lse_c - M) o_c / sum_c 2^(lse_c - M),  M = max_c lse_c.
+template <int D>
+__device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const float *ro,
+                                               const float *rlse, const int *meta, float *s_w,
+                                               int cap, int lane, int cta)
+{
+    const int G = p.G;
+    const int beta = meta[kMetaBeta], j = meta[kMetaJ], seg = meta[kMetaSeg];
+    __nv_bfloat16 *ob = p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+    if (meta[kMetaWhole]) {
+        for (int i = lane * 4; i < G * D; i += 128) {
+            const float4 v = *reinterpret_cast<const float4 *>(ro + i);
+            uint2 w;
+            w.x = pack_bf16x2(v.x, v.y);
+            w.y = pack_bf16x2(v.z, v.w);
+            *reinterpret_cast<uint2 *>(ob + i) = w;
+        }
+        return;
+    }
+    const size_t piece = static_cast<size_t>(seg + cta);
+    float *po = p.part_o + piece * G * D;
+    for (int i = lane * 4; i < G * D; i += 128)
+        *reinterpret_cast<float4 *>(po + i) = *reinterpret_cast<const float4 *>(ro + i);
+    if (lane < G)
+        p.part_lse[piece * G + lane] = rlse[lane];
+    __syncwarp();
+    const int c_first = meta[kMetaFirst], c_last = meta[kMetaLast];
+    unsigned prev = 0;
+    if (lane == 0)
+        prev = atomic_add_acq_rel_gpu(&p.counters[seg], 1u);
+    prev = __shfl_sync(0xffffffffu, prev, 0);
+    __syncwarp();
+    if (prev != static_cast<unsigned>(c_last - c_first))
+        return;
+    // This CTA finished the segment last.  Records seg + c_first .. seg + c_last are contiguous.
+    const int np = c_last - c_first + 1;
+    const size_t rec0 = static_cast<size_t>(seg + c_first);
+    const float NEG_INF = -__int_as_float(0x7f800000);
+    if (np * G <= cap) {
+        for (int i = lane; i < np * G; i += 32)
+            s_w[i] = __ldcg(&p.part_lse[rec0 * G + i]);
+        __syncwarp();
+        for (int r = lane; r < G; r += 32) {
+            float mx = NEG_INF;
+            for (int k = 0; k < np; ++k)
+                mx = fmaxf(mx, s_w[k * G + r]);
+            float tot = 0.f;
+            for (int k = 0; k < np; ++k) {
+                const float w = fast_exp2(s_w[k * G + r] - mx);
+                s_w[k * G + r] = w;
+                tot += w;
+            }
+            const float inv = 1.f / tot;
+            for (int k = 0; k < np; ++k)
+                s_w[k * G + r] *= inv;
+        }
+        __syncwarp();
+        // Each lane owns CH float4 columns of a 128*CH-element chunk; the loads of all its
+        // columns for two pieces are in flight together.
+        constexpr int CH = 8;
+        const float *base = p.part_o + rec0 * G * D;
+        for (int c0 = 0; c0 < G * D; c0 += 128 * CH) {
+            float4 acc[CH];
+#pragma unroll
+            for (int u = 0; u < CH; ++u)
+                acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int k = 0; k < np; k += 2) {
+                float4 v0[CH], v1[CH];
+#pragma unroll
+                for (int u = 0; u < CH; ++u) {
+                    const int i = c0 + u * 128 + lane * 4;
+                    const bool in = i < G * D;
+                    v0[u] = in ? __ldcg(reinterpret_cast<const float4 *>(
+                                     base + static_cast<size_t>(k) * G * D + i))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+                    v1[u] = (in && k + 1 < np)
+                                ? __ldcg(reinterpret_cast<const float4 *>(
+                                      base + static_cast<size_t>(k + 1) * G * D + i))
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int u = 0; u < CH; ++u) {
+                    const int i = c0 + u * 128 + lane * 4;
+                    if (i < G * D) {
+                        const int row = i / D;
+                        const float w0 = s_w[k * G + row];
+                        const float w1 = (k + 1 < np) ? s_w[(k + 1) * G + row] : 0.f;
+                        acc[u].x += w0 * v0[u].x + w1 * v1[u].x;
+                        acc[u].y += w0 * v0[u].y + w1 * v1[u].y;
+                        acc[u].z += w0 * v0[u].z + w1 * v1[u].z;
+                        acc[u].w += w0 * v0[u].w + w1 * v1[u].w;
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < CH; ++u) {
+                const int i = c0 + u * 128 + lane * 4;
+                if (i < G * D) {
+                    uint2 w2;
+                    w2.x = pack_bf16x2(acc[u].x, acc[u].y);
+                    w2.y = pack_bf16x2(acc[u].z, acc[u].w);
+                    *reinterpret_cast<uint2 *>(ob + i) = w2;
+                }
+            }
+        }
+        __syncwarp();
+    } else {
+        // Very many pieces: the same merge, weights recomputed per element.
+        for (int i = lane; i < G * D; i += 32) {
+            const int row = i / D;
+            float mx = NEG_INF;
+            for (int k = 0; k < np; ++k)
+                mx = fmaxf(mx, __ldcg(&p.part_lse[(rec0 + k) * G + row]));
+            float acc = 0.f, wsum = 0.f;
+            for (int k = 0; k < np; ++k) {
+                const float w = fast_exp2(__ldcg(&p.part_lse[(rec0 + k) * G + row]) - mx);
+                wsum += w;
+                acc += w * __ldcg(&p.part_o[(rec0 + k) * G * D + i]);
+            }
+            ob[i] = __float2bfloat16_rn(acc / wsum);
+        }
+    }
+    if (lane == 0)
+        p.counters[seg] = 0u;
+}
+
+// Cluster mode: the k CTAs of a cluster hold the k equal pieces of one segment.  Ranks 1..k-1
+// write their (o, lse) into slot rank-1 of the leader's shared memory over DSMEM and arrive on the
+// leader's cluster barrier; the leader merges the k results from its own shared memory.
+template <int D, int RES_BYTES, int RES_O>
+__device__ __forceinline__ void epilogue_cluster(const DecodeParams &p, const float *ro,
+                                                 const float *rlse, const int *meta,
+                                                 uint8_t *cslots, uint32_t cslots_addr,
+                                                 uint32_t bar_cluster, int lane,
+                                                 volatile int *flags)
+{
+    const int G = p.G;
+    const int k = p.cluster_k;
+    const uint32_t rank = cluster_ctarank();
+    if (rank != 0) {
+        const uint32_t dst = map_to_rank(cslots_addr + (rank - 1) * RES_BYTES, 0);
+        for (int i = lane * 4; i < G * D; i += 128)
+            st_cluster_v4(dst + i * 4, *reinterpret_cast<const float4 *>(ro + i));
+        if (lane < G)
+            st_cluster_f32(dst + RES_O + lane * 4, rlse[lane]);
+        fence_acq_rel_cluster();
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive_remote(map_to_rank(bar_cluster, 0));
+        return;
+    }
+    if (!mbar_wait_cluster(bar_cluster, 0)) {
+        flags[0] = 1;
+        atomicOr(p.err, kErrWaitFull);
+        return;
+    }
+    const int beta = meta[kMetaBeta], j = meta[kMetaJ];
+    __nv_bfloat16 *ob = p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+    for (int i = lane * 4; i < G * D; i += 128) {
+        const int row = i / D;
+        float mx = rlse[row];
+        for (int r = 1; r < k; ++r)
+            mx = fmaxf(mx, reinterpret_cast<const float *>(cslots + (r - 1) * RES_BYTES + RES_O)[row]);
+        float w = fast_exp2(rlse[row] - mx);
+        float tot = w;
+        float4 v = *reinterpret_cast<const float4 *>(ro + i);
+        float4 acc = make_float4(w * v.x, w * v.y, w * v.z, w * v.w);
+        for (int r = 1; r < k; ++r) {
+            const float *slot = reinterpret_cast<const float *>(cslots + (r - 1) * RES_BYTES);
+            w = fast_exp2(slot[RES_O / 4 + row] - mx);
+            tot += w;
+            v = *reinterpret_cast<const float4 *>(slot + i);
+            acc.x += w * v.x;
+            acc.y += w * v.y;
+            acc.z += w * v.z;
+            acc.w += w * v.w;
+        }
+        const float inv = fast_rcp(tot);
+        uint2 w2;
+        w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+        w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2 *>(ob + i) = w2;
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
+// decode kernel
+// ------------------------------------------------------------------------------------------------
+
+template <int D, int T, int STAGES, int NCW>
+__global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads, 1)
+    decode_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ DecodeParams p)
+{
+    using PL = Plan<D, T, STAGES, NCW>;
+    constexpr int TW = PL::kTW;
+    constexpr int NT = TW / 8;     // 8-position score tiles per warp
+    constexpr int KS = D / 16;     // 16-wide reduction steps over the head dimension
+    constexpr int NO = D / 8;      // 8-wide output column tiles
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const uint32_t sbase = smem_addr(smem);
+    const uint32_t bar_full = sbase + PL::kBars;
+    const uint32_t bar_empty = bar_full + 8 * STAGES;
+    const uint32_t bar_res_full = bar_empty + 8 * STAGES;    // [2]
+    const uint32_t bar_res_empty = bar_res_full + 16;        // [2]
+    const uint32_t bar_cluster = bar_res_empty + 16;         // leader: k-1 remote arrivals
+    volatile int *flags = reinterpret_cast<volatile int *>(smem + PL::kFlags);
+    int *s_len = reinterpret_cast<int *>(smem + PL::kTables);
+    int *s_start = s_len + p.b;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int P = gridDim.x;
+    const int cta = blockIdx.x;
+    const int N = p.num_tiles;
+    const int tile_lo = static_cast<int>(static_cast<long long>(cta) * N / P);
+    const int tile_hi = static_cast<int>(static_cast<long long>(cta + 1) * N / P);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(bar_full + 8 * s, 1);
+            mbar_init(bar_empty + 8 * s, NCW);
+        }
+        for (int r = 0; r < 2; ++r) {
+            mbar_init(bar_res_full + 8 * r, 1);
+            mbar_init(bar_res_empty + 8 * r, 1);
+        }
+        mbar_init(bar_cluster, p.cluster_k > 1 ? p.cluster_k - 1 : 1);
+        flags[0] = 0;   // abort
+        fence_barrier_init();
+    }
+    if (threadIdx.x == PL::kProducer * 32)
+        prefetch_tensormap(&tmap);   // a kernel parameter: safe before the dependency wait
+    if (p.uniform_len <= 0) {
+        for (int i = threadIdx.x; i < p.b; i += blockDim.x) {
+            s_len[i] = p.seq_len[i];
+            s_start[i] = p.tile_start[i];
+        }
+        if (threadIdx.x == 0)
+            s_start[p.b] = p.tile_start[p.b];
+    }
+    __syncthreads();
+    if (p.cluster_k > 1)
+        cluster_sync_all();   // every rank's barriers exist before any remote arrival
+    // Everything above overlaps the previous kernel's tail; global memory is touched only below.
+    grid_dependency_wait();
+    grid_dependents_launch();
+
+    // -------------------------------- producer warp --------------------------------------------
+    if (warp == PL::kProducer) {
+        if (lane != 0)
+            return;
+        int issued = 0;
+        TileWalk<T> wk;
+        if (tile_lo < tile_hi)
+            wk.init(p, s_len, s_start, tile_lo);
+        for (int tile = tile_lo; tile < tile_hi; ++tile) {
+            const int s = issued % STAGES;
+            if (issued >= STAGES && !flags[0] &&
+                !mbar_wait(bar_empty + 8 * s, ((issued / STAGES) & 1) ^ 1)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitEmpty);
+            }
+            if (flags[0])
+                break;
+            const uint32_t fb = bar_full + 8 * s;
+            mbar_arrive_expect_tx(fb, PL::kStageBytes);
+            const int zk = ((p.slot * 2 + 0) * p.b + wk.beta) * p.g + wk.j;
+            const int zv = zk + p.b * p.g;
+            const int y = wk.tt * T;
+            const uint32_t kdst = sbase + s * PL::kStageBytes;
+            const uint32_t vdst = kdst + PL::kTileBytes;
+#pragma unroll
+            for (int sub = 0; sub < PL::kSub; ++sub) {
+                tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
+                tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
+            }
+            ++issued;
+            wk.next(p, s_len, s_start);
+        }
+        // No copy may still be in flight when the CTA exits.
+        const int first = issued > STAGES ? issued - STAGES : 0;
+        for (int k = first; k < issued; ++k)
+            if (!mbar_wait(bar_full + 8 * (k % STAGES), (k / STAGES) & 1))
+                atomicOr(p.err, kErrDrain);
+        return;
+    }
+
+    // -------------------------------- epilogue warp --------------------------------------------
+    if (warp == PL::kEpilogue) {
+        float *s_w = reinterpret_cast<float *>(smem + PL::kEpiW);
+        for (int k = 0;; ++k) {
+            const int rb = k & 1;
+            if (!mbar_wait(bar_res_full + 8 * rb, (k >> 1) & 1)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitFull);
+                return;
+            }
+            const uint8_t *slot = smem + PL::kRes + rb * PL::kResBytes;
+            const int *meta = reinterpret_cast<const int *>(slot + PL::kResO + 64);
+            if (meta[kMetaStop])
+                return;
+            if (!flags[0]) {
+                if (p.cluster_k > 1)
+                    epilogue_cluster<D, PL::kResBytes, PL::kResO>(
+                        p, reinterpret_cast<const float *>(slot),
+                        reinterpret_cast<const float *>(slot + PL::kResO), meta,
+                        smem + PL::kTables, sbase + PL::kTables, bar_cluster, lane, flags);
+                else
+                    epilogue_piece<D>(p, reinterpret_cast<const float *>(slot),
+                                      reinterpret_cast<const float *>(slot + PL::kResO), meta,
+                                      s_w, PL::kEpiCap, lane, cta);
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(bar_res_empty + 8 * rb);
+        }
+    }
+
+    // -------------------------------- consumer warps -------------------------------------------
+    float *merge = reinterpret_cast<float *>(smem + PL::kMerge);
+    float *red_m = reinterpret_cast<float *>(smem + PL::kRedM);
+    float *red_l = reinterpret_cast<float *>(smem + PL::kRedL);
+    const int qr = lane >> 2;              // fragment row (query head within the group)
+    const int qc = (lane & 3) * 2;         // fragment column pair
+    const int G = p.G;
+    const float scale = p.scale_log2;
+    const float NEG_INF = -__int_as_float(0x7f800000);
+
+    int it = 0;
+    int npiece = 0;
+    int tile = tile_lo;
+    TileWalk<T> wk;
+    if (tile < tile_hi)
+        wk.init(p, s_len, s_start, tile);
+
+    while (tile < tile_hi) {
+        const int beta = wk.beta;
+        const int j = wk.j;
+        const int L = wk.L;
+        const int seg = beta * p.g + j;
+        const int seg_first = wk.seg_first;
+        const int seg_end = seg_first + wk.nt;
+        const int piece_first = tile;
+        const int piece_end = seg_end < tile_hi ? seg_end : tile_hi;
+
+        // Query fragments of the group's heads (rows >= G are zero): A operand of S = Q K^T.
+        uint32_t qa[KS][4];
+        {
+            const __nv_bfloat16 *qb =
+                p.Q + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+            const bool r0 = qr < G, r1 = qr + 8 < G;
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                const int c = ks * 16 + qc;
+                qa[ks][0] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c) : 0u;
+                qa[ks][1] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c) : 0u;
+                qa[ks][2] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c + 8) : 0u;
+                qa[ks][3] =
+                    r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c + 8) : 0u;
+            }
+        }
+
+        float o[NO][4];
+#pragma unroll
+        for (int n = 0; n < NO; ++n)
+            o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+        float m_run[2] = {NEG_INF, NEG_INF};
+        float l_run[2] = {0.f, 0.f};
+
+        for (; tile < piece_end; ++tile, ++it) {
+            const int s = it % STAGES;
+            if (!flags[0] && !mbar_wait(bar_full + 8 * s, (it / STAGES) & 1)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitFull);
+            }
+            const int row0 = warp * TW;                 // this warp's first row in the tile
+            const int valid = L - (wk.tt * T + row0);   // visible rows in this warp's slice
+            if (!flags[0] && valid > 0) {
+                const uint32_t kt = sbase + s * PL::kStageBytes;
+                const uint32_t vt = kt + PL::kTileBytes;
+                if (p.K_new != nullptr && valid <= TW) {
+                    // Fused append: this warp's slice holds position L-1, the new token.  Its K/V
+                    // replace the tile rows (the copy read the cache before the token was stored)
+                    // and are stored in the cache for the layers that read this slot later.
+                    const int r_new = row0 + valid - 1;
+                    if (lane < 8 * PL::kSub) {
+                        const size_t src = (static_cast<size_t>(beta) * p.g + j) * D + lane * 8;
+                        const uint4 kn = *reinterpret_cast<const uint4 *>(p.K_new + src);
+                        const uint4 vn = *reinterpret_cast<const uint4 *>(p.V_new + src);
+                        uint8_t *st = smem + s * PL::kStageBytes;
+                        *reinterpret_cast<uint4 *>(st + swz<T>(r_new, lane)) = kn;
+                        *reinterpret_cast<uint4 *>(st + PL::kTileBytes + swz<T>(r_new, lane)) = vn;
+                        const size_t dst =
+                            ((((static_cast<size_t>(p.slot) * 2) * p.b + beta) * p.g + j) *
+                                 static_cast<size_t>(p.max_seq) + (L - 1)) * D + lane * 8;
+                        *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
+                        *reinterpret_cast<uint4 *>(
+                            p.cache + dst + static_cast<size_t>(p.b) * p.g * p.max_seq * D) = vn;
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                }
+                if (valid < TW) {
+                    // Rows past the sequence end hold whatever the cache holds there; zero the V
+                    // rows so that 0-weight * V stays 0 even for non-finite contents.
+                    uint8_t *vrow = smem + s * PL::kStageBytes + PL::kTileBytes;
+                    const int nrows = TW - valid;
+                    for (int idx = lane; idx < nrows * 8 * PL::kSub; idx += 32) {
+                        const int rr = row0 + valid + idx / (8 * PL::kSub);
+                        const int rem = idx % (8 * PL::kSub);
+                        const int sub = rem / 8;
+                        *reinterpret_cast<uint4 *>(vrow + sub * T * 128 + rr * 128 +
+                                                   (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                }
+
+                // ---- S = Q K^T for this warp's TW positions ----
+                float sc[NT][4];
+#pragma unroll
+                for (int n = 0; n < NT; ++n)
+                    sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+                const int mi = lane >> 3;   // which 8x8 matrix this lane addresses
+                const int mr = lane & 7;    // which row of it
+#pragma unroll
+                for (int ks = 0; ks < KS; ++ks) {
+#pragma unroll
+                    for (int n = 0; n < NT; n += 2) {
+                        const int row = row0 + 8 * (n + (mi >> 1)) + mr;
+                        const int chunk = 2 * ks + (mi & 1);
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4(kt + swz<T>(row, chunk), b0, b1, b2, b3);
+                        mma_bf16_16816(sc[n], qa[ks], b0, b1);
+                        mma_bf16_16816(sc[n + 1], qa[ks], b2, b3);
+                    }
+                }
+
+                // ---- online softmax (base 2, scale folded into the exponent) ----
+                float mx[2] = {NEG_INF, NEG_INF};
+                if (valid < TW) {
+#pragma unroll
+                    for (int n = 0; n < NT; ++n) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const int pos_in_slice = 8 * n + qc + (c & 1);
+                            if (pos_in_slice >= valid)
+                                sc[n][c] = NEG_INF;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int n = 0; n < NT; ++n) {
+                    mx[0] = fmaxf(mx[0], fmaxf(sc[n][0], sc[n][1]));
+                    mx[1] = fmaxf(mx[1], fmaxf(sc[n][2], sc[n][3]));
+                }
+                float alpha[2], m_use[2];
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 1));
+                    mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 2));
+                    const float m_new = fmaxf(m_run[hr], mx[hr] * scale);
+                    m_use[hr] = (m_new == NEG_INF) ? 0.f : m_new;
+                    alpha[hr] = fast_exp2(m_run[hr] - m_use[hr]);
+                    m_run[hr] = m_new;
+                    l_run[hr] *= alpha[hr];
+                }
+                // Rescale the accumulators only when some row's running maximum moved.
+                if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
+#pragma unroll
+                    for (int n = 0; n < NO; ++n) {
+                        o[n][0] *= alpha[0];
+                        o[n][1] *= alpha[0];
+                        o[n][2] *= alpha[1];
+                        o[n][3] *= alpha[1];
+                    }
+                }
+                // P in bf16 (the mma A operand); the row sums use the same rounded weights.
+                uint32_t pa[NT / 2][4];
+#pragma unroll
+                for (int n = 0; n < NT; ++n) {
+                    const float p0 = fast_exp2(fmaf(sc[n][0], scale, -m_use[0]));
+                    const float p1 = fast_exp2(fmaf(sc[n][1], scale, -m_use[0]));
+                    const float p2 = fast_exp2(fmaf(sc[n][2], scale, -m_use[1]));
+                    const float p3 = fast_exp2(fmaf(sc[n][3], scale, -m_use[1]));
+                    const uint32_t top = pack_bf16x2(p0, p1);
+                    const uint32_t bot = pack_bf16x2(p2, p3);
+                    l_run[0] += bf16_lo(top) + bf16_hi(top);
+                    l_run[1] += bf16_lo(bot) + bf16_hi(bot);
+                    pa[n >> 1][(n & 1) * 2 + 0] = top;
+                    pa[n >> 1][(n & 1) * 2 + 1] = bot;
+                }
+
+                // ---- O += P V ----
+#pragma unroll
+                for (int kk = 0; kk < NT / 2; ++kk) {
+#pragma unroll
+                    for (int q = 0; q < NO / 2; ++q) {
+                        const int row = row0 + 16 * kk + 8 * (mi & 1) + mr;
+                        const int chunk = 2 * q + (mi >> 1);
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4_trans(vt + swz<T>(row, chunk), b0, b1, b2, b3);
+                        mma_bf16_16816(o[2 * q], pa[kk], b0, b1);
+                        mma_bf16_16816(o[2 * q + 1], pa[kk], b2, b3);
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(bar_empty + 8 * s);
+            wk.next(p, s_len, s_start);
+        }
+
+        // ---------------- end of piece: merge the warps (no atomics) ----------------
+        // Row statistics of every warp -> per-row maximum and total; each warp scales its own
+        // accumulators by 2^(m_w - m*) / l*, then a tree over warps sums them into warp 0.
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
+            l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 2);
+        }
+        if ((lane & 3) == 0) {
+            red_m[warp * 16 + qr] = m_run[0];
+            red_m[warp * 16 + qr + 8] = m_run[1];
+            red_l[warp * 16 + qr] = l_run[0];
+            red_l[warp * 16 + qr + 8] = l_run[1];
+        }
+        consumer_bar_sync<NCW>();
+        float lse[2];
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            const int row = qr + 8 * hr;
+            // every piece holds at least one visible position, so mstar is finite
+            float mstar = NEG_INF;
+#pragma unroll
+            for (int w = 0; w < NCW; ++w)
+                mstar = fmaxf(mstar, red_m[w * 16 + row]);
+            float lsum = 0.f;
+#pragma unroll
+            for (int w = 0; w < NCW; ++w)
+                lsum += red_l[w * 16 + row] * fast_exp2(red_m[w * 16 + row] - mstar);
+            const float f = fast_exp2(m_run[hr] - mstar) * fast_rcp(lsum);
+            lse[hr] = mstar + fast_log2(lsum);
+#pragma unroll
+            for (int n = 0; n < NO; ++n) {
+                o[n][2 * hr] *= f;
+                o[n][2 * hr + 1] *= f;
+            }
+        }
+        // Tree over warps with NCW/2 slots.  First level: warp w in [NCW/2, NCW) writes slot
+        // w - NCW/2 and warp r < NCW/2 adds slot r.  Later levels (half < NCW/2): warp w in
+        // [half, 2 half) writes slot w and warp r < half adds slot r + half.  Every slot is
+        // rewritten only by the warp that read it last, so one barrier per level suffices.
+#pragma unroll
+        for (int half = NCW / 2; half >= 1; half >>= 1) {
+            const bool first = (half == NCW / 2);
+            if (warp >= half && warp < 2 * half) {
+                float *dst = merge + (first ? warp - half : warp) * (NO * 4 * 32);
+#pragma unroll
+                for (int n = 0; n < NO; ++n)
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        dst[(n * 4 + c) * 32 + lane] = o[n][c];
+            }
+            consumer_bar_sync<NCW>();
+            if (warp < half) {
+                const float *src = merge + (first ? warp : warp + half) * (NO * 4 * 32);
+#pragma unroll
+                for (int n = 0; n < NO; ++n)
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        o[n][c] += src[(n * 4 + c) * 32 + lane];
+            }
+        }
+
+        // Warp 0 hands the piece to the epilogue warp through a double-buffered slot and the
+        // consumers move on to the next piece at once.
+        if (warp == 0) {
+            const int rb = npiece & 1;
+            if (npiece >= 2 && !flags[0] &&
+                !mbar_wait(bar_res_empty + 8 * rb, ((npiece >> 1) - 1) & 1)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitEmpty);
+            }
+            uint8_t *slot = smem + PL::kRes + rb * PL::kResBytes;
+            float *ro = reinterpret_cast<float *>(slot);
+            float *rlse = reinterpret_cast<float *>(slot + PL::kResO);
+            int *meta = reinterpret_cast<int *>(slot + PL::kResO + 64);
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                const int row = qr + 8 * hr;
+                if (row < G) {
+#pragma unroll
+                    for (int n = 0; n < NO; ++n)
+                        *reinterpret_cast<float2 *>(ro + row * D + n * 8 + qc) =
+                            make_float2(o[n][2 * hr], o[n][2 * hr + 1]);
+                    if (qc == 0)
+                        rlse[row] = lse[hr];
+                }
+            }
+            if (lane == 0) {
+                meta[kMetaBeta] = beta;
+                meta[kMetaJ] = j;
+                meta[kMetaSeg] = seg;
+                meta[kMetaWhole] = (piece_first == seg_first && piece_end == seg_end) ? 1 : 0;
+                meta[kMetaFirst] = cta_of_tile(seg_first, N, P);
+                meta[kMetaLast] = cta_of_tile(seg_end - 1, N, P);
+                meta[kMetaStop] = 0;
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(bar_res_full + 8 * rb);
+        }
+        ++npiece;
+    }
+    // Tell the epilogue warp that no piece follows.
+    if (warp == 0) {
+        const int rb = npiece & 1;
+        if (npiece >= 2 && !flags[0] && !mbar_wait(bar_res_empty + 8 * rb, ((npiece >> 1) - 1) & 1)) {
+            flags[0] = 1;
+            atomicOr(p.err, kErrWaitEmpty);
+        }
+        if (lane == 0) {
+            int *meta = reinterpret_cast<int *>(smem + PL::kRes + rb * PL::kResBytes + PL::kResO + 64);
+            meta[kMetaStop] = 1;
+            mbar_arrive(bar_res_full + 8 * rb);
+        }
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
+// append kernel: one thread per 16-byte vector of the new token's K/V rows
+// ------------------------------------------------------------------------------------------------
+
+__global__ void append_kernel(const __grid_constant__ AppendParams p)
+{
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int vecs = p.d / 8;
+    const long long total = 2LL * p.b * p.g * vecs;
+    const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= total)
+        return;
+    const int v = static_cast<int>(idx % vecs);
+    long long row = idx / vecs;   // (kv, beta, j)
+    const int j = static_cast<int>(row % p.g);
+    row /= p.g;
+    const int beta = static_cast<int>(row % p.b);
+    const int kv = static_cast<int>(row / p.b);
+    const int pos = p.seq_len[beta] - 1;
+    const uint4 *src = reinterpret_cast<const uint4 *>(kv ? p.V : p.K) +
+                       (static_cast<size_t>(beta) * p.g + j) * vecs + v;
+    uint4 *dst = reinterpret_cast<uint4 *>(p.cache) +
+                 ((((static_cast<size_t>(p.slot) * 2 + kv) * p.b + beta) * p.g + j) *
+                      static_cast<size_t>(p.max_seq) + pos) * vecs + v;
+    *dst = *src;
+}
+
+template <int D, int T, int STAGES, int NCW>
+constexpr DecodeVariant make_variant()
+{
+    using PL = Plan<D, T, STAGES, NCW>;
+    return DecodeVariant{D, T, STAGES, PL::kThreads, static_cast<size_t>(PL::kAlloc),
+                         static_cast<size_t>(PL::kResBytes),
+                         reinterpret_cast<const void *>(&decode_kernel<D, T, STAGES, NCW>)};
+}
+
+// (head_dim, positions per tile, ring stages, consumer warps); the first match of a
+// (head_dim, tile) pair is used.
+const DecodeVariant kVariants[] = {
+    make_variant<64, 128, 6, 8>(),
+    make_variant<64, 256, 3, 8>(),
+    make_variant<64, 64, 4, 4>(),
+    make_variant<128, 64, 5, 4>(),
+    make_variant<128, 128, 2, 4>(),
+};
+
+}  // namespace
+
+const DecodeVariant *find_decode_variant(int head_dim, int tile_tokens)
+{
+    for (const DecodeVariant &v : kVariants)
+        if (v.head_dim == head_dim && v.tile_tokens == tile_tokens)
+            return &v;
+    return nullptr;
+}
+
+cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem)
+{
+    size_t tail = table_bytes(MLKV_MAX_BATCH);
+    if (3 * v.res_bytes > tail)
+        tail = 3 * v.res_bytes;   // cluster mode, k = 4
+    size_t want = v.smem_bytes + tail;
+    if (want > max_smem)
+        want = max_smem;
+    if (v.smem_bytes > want)
+        return cudaErrorInvalidValue;
+    return cudaFuncSetAttribute(v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(want));
+}
+
+cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
+                          const CUtensorMap *tmap, const DecodeParams &p,
+                          const cudaAccessPolicyWindow *window)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(static_cast<unsigned>(v.threads));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[3];
+    int na = 0;
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+    if (p.cluster_k > 1) {
+        attr[na].id = cudaLaunchAttributeClusterDimension;
+        attr[na].val.clusterDim.x = static_cast<unsigned>(p.cluster_k);
+        attr[na].val.clusterDim.y = 1;
+        attr[na].val.clusterDim.z = 1;
+        ++na;
+    }
+    if (window != nullptr) {
+        attr[na].id = cudaLaunchAttributeAccessPolicyWindow;
+        attr[na].val.accessPolicyWindow = *window;
+        ++na;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = na;
+    void *args[] = {const_cast<CUtensorMap *>(tmap), const_cast<DecodeParams *>(&p)};
+    return cudaLaunchKernelExC(&cfg, v.fn, args);
+}
+
+cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(k));
+    cfg.blockDim = dim3(static_cast<unsigned>(v.threads));
+    cfg.dynamicSmemBytes = v.smem_bytes + (k - 1) * v.res_bytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(k);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaOccupancyMaxActiveClusters(out, v.fn, &cfg);
+}
+
+cudaError_t launch_append(const AppendParams &p, cudaStream_t stream)
+{
+    const long long total = 2LL * p.b * p.g * (p.d / 8);
+    const int threads = 256;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>((total + threads - 1) / threads));
+    cfg.blockDim = dim3(threads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void *args[] = {const_cast<AppendParams *>(&p)};
+    return cudaLaunchKernelExC(&cfg, reinterpret_cast<const void *>(&append_kernel), args);
+}
+
+}  // namespace mlkv
