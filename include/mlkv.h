@@ -44,6 +44,7 @@ extern "C" {
 
 #define MLKV_MAX_BATCH 1024       /* largest batch a cache may hold */
 #define MLKV_MAX_GROUP 16         /* largest query group h/g per KV head */
+#define MLKV_STATIC_SCRATCH_BYTES (8u << 20) /* scratch of mlkv_decode_attention_static */
 
 typedef struct mlkv_cache *mlkv_cache_t;
 
@@ -173,6 +174,36 @@ const char *mlkv_last_error(void);
  * n_layers (else MLKV_ERR_MAP).  layer_owner: host int32[n_layers], written on success.
  */
 int mlkv_block_owner_map(int n_layers, int n_owners, int *layer_owner);
+
+/*
+ * mlkv_decode_attention_static - decode attention over one owner slot held by the caller, for
+ * callers that cannot allocate device memory.  It allocates nothing: no cudaMalloc, cudaFree or
+ * allocating library call, on any call.
+ *
+ * The paper has no counterpart; this is a deployment variant of mlkv_decode_attention.  Some
+ * callers may not allocate device memory once they run: a runtime whose own allocator owns all
+ * device memory, or a serving loop that must not call cudaMalloc (it can synchronise the device
+ * and stall every stream).  Such a caller keeps the cache slot itself and passes it here; the
+ * merge scratch of the split-KV kernel (partial outputs, their log-sum-exps, per-(sequence, KV
+ * head) counters, an error word) lives in one array compiled into the library, of
+ * MLKV_STATIC_SCRATCH_BYTES (8 MiB), which every GPU that loads the library holds until exit.
+ *
+ *   kv_slot    device bf16 [2][batch][kv_heads][max_seq][head_dim]: the K block then the V block
+ *              of one owner layer, the layout of mlkv_kv_ptr's k_base (v_base follows it)
+ *   batch, n_q_heads, kv_heads, head_dim, max_seq   as for mlkv_cache_create (kv_heads = g)
+ *   Q, out, seq_lens, cuda_stream                   as for mlkv_decode_attention
+ * Runs on the calling thread's current device.  The first call on a device sets that device up
+ * (looks up the scratch array's device address with cudaGetSymbolAddress and raises the kernels'
+ * shared-memory limits); make that first call before any stream capture.  Every call clears the
+ * part of the array that must start at zero, in stream order.  All calls share the one array:
+ * calls whose work overlaps on the GPU (different streams, no ordering between them) race on it
+ * and must not be issued.  A request whose scratch would exceed the array (roughly
+ * batch * kv_heads * (h/g) * (head_dim + 1) * 4 bytes plus one record per CTA) returns
+ * MLKV_ERR_UNSUPPORTED before any work is queued.
+ */
+int mlkv_decode_attention_static(const void *kv_slot, int batch, int n_q_heads, int kv_heads,
+                                 int head_dim, int max_seq, const void *Q, void *out,
+                                 const int *seq_lens, void *cuda_stream);
 
 /* Library version, major*10000 + minor*100 + patch. */
 int mlkv_version(void);

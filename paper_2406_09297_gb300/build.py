@@ -19,7 +19,7 @@ NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc" if os.path.exists(
     "/usr/local/cuda/bin/nvcc") else "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
-SOURCES = ["mlkv_kernels.cu", "mlkv_host.cpp"]
+SOURCES = ["mlkv_kernels.cu", "mlkv_host.cpp", "mlkv_noalloc.cu"]
 
 
 def _sources():

@@ -225,6 +225,8 @@ int validate_map(int l, int h, int d, const int *owner, int g, int b, int max_se
 
 }  // namespace
 
+void mlkv::set_last_error(const char *msg) { g_last_error = msg; }
+
 extern "C" {
 
 int mlkv_version(void) { return 100; }

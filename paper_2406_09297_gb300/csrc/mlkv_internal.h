@@ -73,6 +73,9 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
                           const CUtensorMap *tmap, const DecodeParams &p,
                           const cudaAccessPolicyWindow *window);
 
+// Sets the calling thread's mlkv_last_error() text.
+void set_last_error(const char *msg);
+
 // How many k-CTA clusters of this variant can be resident at once.
 cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out);
 

@@ -29,7 +29,7 @@ EXPORTED = [
     "mlkv_append_decode_attention",
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
-    "mlkv_block_owner_map", "mlkv_version",
+    "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static",
 ]
 
 
@@ -65,6 +65,7 @@ def _load():
     L.mlkv_last_error.restype = ctypes.c_char_p
     L.mlkv_block_owner_map.argtypes = [ci, ci, ip]
     L.mlkv_version.argtypes = []
+    L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
     return L
 
 
@@ -187,6 +188,15 @@ def mlkv_block_owner_map(n_layers, n_owners):
 
 def mlkv_version():
     return lib.mlkv_version()
+
+
+def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, max_seq, Q, out,
+                                 seq_lens, stream=None):
+    """kv_slot: device address (int) of a [2][batch][kv_heads][max_seq][head_dim] bf16 block."""
+    a, p = _lens_ptr(seq_lens)
+    return _check(lib.mlkv_decode_attention_static(
+        ctypes.c_void_p(kv_slot), batch, n_q_heads, kv_heads, head_dim, max_seq, _ptr(Q),
+        _ptr(out), p, _stream(stream)))
 
 
 class MLKVCache:
