@@ -217,7 +217,6 @@ def run(args, w):
         import torch.distributed as dist
         dist.init_process_group("nccl")
 
-    seq_lens = w.seq_lens()
     cache = mlkv.MLKVCache(w.l, w.h, w.d, w.owner, w.g, w.b, w.max_seq)
     if args.tile:
         cache.set_option("tile_tokens", args.tile)
@@ -226,16 +225,7 @@ def run(args, w):
     if args.l2_persist:
         cache.set_option("l2_persist", 1)
     owners = w.owners()
-    # owner caches: generator values at every position [0, max_seq)
-    for n in owners:
-        slot = cache.owner_slot(n)[1]
-        kp, vp, strides = cache.kv_ptr(slot)
-        device.fill_slot(kp, vp, strides, w.seed, n, w.b, w.g, w.d, w.max_seq, w.sigma_k,
-                         w.sigma_v)
-    Q = [device.q_tensor(w.seed, n, w.b, w.h, w.d, w.sigma_q) for n in range(w.l)]
-    # the new token of every owner: the generator's value at L-1 (re-appending it is idempotent)
-    Kn = {n: device.kv_token(w.seed, n, 0, w.b, w.g, w.d, seq_lens, w.sigma_k) for n in owners}
-    Vn = {n: device.kv_token(w.seed, n, 1, w.b, w.g, w.d, seq_lens, w.sigma_v) for n in owners}
+    seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
     out = [torch.empty((w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda") for _ in range(w.l)]
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     torch.cuda.synchronize()

@@ -71,3 +71,19 @@ def fill_slot(k_base, v_base, strides, seed, owner_layer, b, g, d, length, sigma
     pitch = strides[1]   # elements between consecutive (beta, j) rows
     fill_ptr(k_base, b * g, length * d, pitch, seed, gen.TID_K + owner_layer, sigma_k)
     fill_ptr(v_base, b * g, length * d, pitch, seed, gen.TID_V + owner_layer, sigma_v)
+
+
+def workload_inputs(w, cache):
+    """Device inputs of one decode step of workload `w` on an mlkv cache (the bench's and the
+    full-size tests' set-up): every owner slot holds the generator's K/V at positions
+    [0, max_seq); Q of every layer; the new token of every owner (the generator's value at L-1,
+    so re-appending it is idempotent).  Returns (seq_lens, Q list, K_new dict, V_new dict)."""
+    seq_lens = w.seq_lens()
+    for n in w.owners():
+        slot = cache.owner_slot(n)[1]
+        kp, vp, strides = cache.kv_ptr(slot)
+        fill_slot(kp, vp, strides, w.seed, n, w.b, w.g, w.d, w.max_seq, w.sigma_k, w.sigma_v)
+    Q = [q_tensor(w.seed, n, w.b, w.h, w.d, w.sigma_q) for n in range(w.l)]
+    Kn = {n: kv_token(w.seed, n, 0, w.b, w.g, w.d, seq_lens, w.sigma_k) for n in w.owners()}
+    Vn = {n: kv_token(w.seed, n, 1, w.b, w.g, w.d, seq_lens, w.sigma_v) for n in w.owners()}
+    return seq_lens, Q, Kn, Vn

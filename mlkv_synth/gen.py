@@ -85,10 +85,40 @@ def bf16_bits_to_f32(bits):
     return u.view(np.float32)
 
 
-def gen_bf16(seed, tensor_id, rows, ncols, sigma=1.0, col0=0):
+_host_lib = None
+
+
+def _host():
+    """The C implementation of this generator (synth_host.c), or None if it cannot be built."""
+    global _host_lib
+    if _host_lib is None:
+        import ctypes
+        try:
+            from . import build as _b
+            L = ctypes.CDLL(_b.build_host())
+            L.synth_host_fill_bf16.argtypes = [
+                ctypes.c_void_p, ctypes.c_longlong, ctypes.c_longlong, ctypes.c_longlong,
+                ctypes.c_void_p, ctypes.c_longlong, ctypes.c_ulonglong, ctypes.c_ulonglong,
+                ctypes.c_float]
+            _host_lib = L
+        except Exception:
+            _host_lib = False
+    return _host_lib or None
+
+
+def gen_bf16(seed, tensor_id, rows, ncols, sigma=1.0, col0=0, impl="auto"):
     """bf16 bit patterns [len(rows)][ncols] of the generator at the given row ids and columns
-    [col0, col0 + ncols)."""
+    [col0, col0 + ncols).  impl: "numpy", "c" or "auto" (C when available)."""
     rows = [int(r) for r in np.atleast_1d(rows)]
+    host = _host() if impl in ("auto", "c") else None
+    if impl == "c" and host is None:
+        raise RuntimeError("the C generator is not available")
+    if host is not None:
+        out = np.empty((len(rows), ncols), dtype=np.uint16)
+        ids = np.asarray(rows, dtype=np.int64)
+        host.synth_host_fill_bf16(out.ctypes.data, len(rows), ncols, ncols, ids.ctypes.data,
+                                  col0, seed, tensor_id, sigma)
+        return out
     out = np.empty((len(rows), ncols), dtype=np.uint16)
     k = np.arange(3 * col0, 3 * (col0 + ncols), dtype=np.uint64) + np.uint64(1)
     with np.errstate(over="ignore"):

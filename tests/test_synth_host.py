@@ -12,9 +12,16 @@ def test_splitmix64_published_vectors():
         6457827717110365317, 3203168211198807973, 9817491932198370423]
 
 
+def test_c_generator_matches_numpy_bits():
+    for sigma in (1.0, 0.5):
+        a = gen.gen_bf16(7, 0x305, [0, 3, 1 << 20], 5000, sigma=sigma, col0=11, impl="numpy")
+        b = gen.gen_bf16(7, 0x305, [0, 3, 1 << 20], 5000, sigma=sigma, col0=11, impl="c")
+        assert np.array_equal(a, b)
+
+
 def test_vectorised_generator_matches_scalar_definition():
     seed, tid, row, ncols = 99, 0x201, 5, 17
-    bits = gen.gen_bf16(seed, tid, [row], ncols, sigma=0.5, col0=3)[0]
+    bits = gen.gen_bf16(seed, tid, [row], ncols, sigma=0.5, col0=3, impl="numpy")[0]
     s = gen.row_seed(seed, tid, row)
     for c in range(ncols):
         col = 3 + c
