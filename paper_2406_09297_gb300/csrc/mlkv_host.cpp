@@ -115,7 +115,7 @@ struct mlkv_cache {
     int l2_persist = 0;
     int cluster = 1;            // allow the DSMEM cluster merge
     // the most recent decode launch (read-only options, for tests and tuning)
-    int last_grid = 0, last_tile = 0, last_cluster_k = 0;
+    int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0;
     // per-variant launch state
     struct Variant {
         const mlkv::DecodeVariant *v = nullptr;
@@ -486,7 +486,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
         const long long per = (tiles + wave - 1) / wave;
         grid = static_cast<int>((tiles + per - 1) / per);
     }
-    grid = std::max(grid, 1);
+    grid = std::max(std::min(grid, mlkv::kCombineMaxPiecesHost), 1);
 
     p.Q = static_cast<const __nv_bfloat16 *>(Q);
     p.out = static_cast<__nv_bfloat16 *>(out);
@@ -506,6 +506,14 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     p.slot = c->slot[layer];
     p.num_tiles = static_cast<int>(tiles);
     p.cluster_k = cluster_k;
+    p.tile_tokens = T;
+    p.decode_grid = grid;
+    // Segments split over many CTAs are merged by a separate parallel kernel: one warp merging
+    // dozens of partials would serialise on its loads.
+    p.deferred_merge = (cluster_k <= 1 &&
+                        mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces)
+                           ? 1
+                           : 0;
 
     cudaAccessPolicyWindow win = {};
     const cudaAccessPolicyWindow *winp = nullptr;
@@ -526,9 +534,15 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                                         &var->tmap, p, winp);
     if (e != cudaSuccess)
         return fail_cuda(e, "decode launch");
+    if (p.deferred_merge) {
+        e = mlkv::launch_combine(p, c->d, static_cast<cudaStream_t>(cuda_stream));
+        if (e != cudaSuccess)
+            return fail_cuda(e, "combine launch");
+    }
     c->last_grid = grid;
     c->last_tile = T;
     c->last_cluster_k = cluster_k;
+    c->last_deferred = p.deferred_merge;
     return MLKV_OK;
 }
 
@@ -688,6 +702,10 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "last_cluster_k") == 0) {
         *value = c->last_cluster_k;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_deferred_merge") == 0) {
+        *value = c->last_deferred;
         return MLKV_OK;
     }
     if (std::strcmp(key, "max_grid") == 0) {

@@ -36,6 +36,9 @@ struct DecodeParams {
     int num_tiles;            // total tiles over all (beta, j) segments
     int uniform_len;          // the common length when every sequence has the same, else 0
     int cluster_k;            // > 1: clusters of k CTAs, one segment each, merged over DSMEM
+    int deferred_merge;       // 1: split segments only write partials; combine_kernel merges them
+    int tile_tokens;          // T of the launch (the combine kernel re-derives the piece layout)
+    int decode_grid;          // P of the decode launch
     int seq_len[MLKV_MAX_BATCH];
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };
@@ -75,6 +78,19 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
 
 // Sets the calling thread's mlkv_last_error() text.
 void set_last_error(const char *msg);
+
+// Largest number of CTAs sharing one (sequence, KV head) segment for a stream-K launch of `grid`
+// CTAs over the tiles described by p (tile_start / seq_len / uniform_len, g, b) with tile length T.
+int max_pieces_per_segment(const DecodeParams &p, int T, int grid);
+
+// Merges the partials of every split segment of the decode launch described by p (which must
+// have deferred_merge = 1), launched right after it on the same stream.
+cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream);
+
+// Pieces per segment above which the decode launch defers its merges to combine_kernel.
+constexpr int kInlineMergeMaxPieces = 4;
+// combine_kernel keeps one weight per piece in shared memory.
+constexpr int kCombineMaxPiecesHost = 1024;
 
 // How many k-CTA clusters of this variant can be resident at once.
 cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out);

@@ -439,6 +439,8 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
         *reinterpret_cast<float4 *>(po + i) = *reinterpret_cast<const float4 *>(ro + i);
     if (lane < G)
         p.part_lse[piece * G + lane] = rlse[lane];
+    if (p.deferred_merge)
+        return;   // combine_kernel merges this segment after the launch
     __syncwarp();
     const int c_first = meta[kMetaFirst], c_last = meta[kMetaLast];
     unsigned prev = 0;
@@ -1048,6 +1050,105 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads, 1)
 }
 
 // ------------------------------------------------------------------------------------------------
+// combine kernel: merge of segments split over many CTAs
+// ------------------------------------------------------------------------------------------------
+
+// One CTA per (segment, query row of its group).  The CTA first turns the pieces' log-sum-exps
+// into normalised weights w_c = 2^(lse_c - M) / sum_c' 2^(lse_c' - M) (M = max_c lse_c), then
+// each thread sums w_c * o_c[e] for one column e over a strided subset of the pieces, with up to
+// 16 loads in flight, and the subsets are added through shared memory.
+constexpr int kCombineThreads = 256;
+constexpr int kCombineMaxPieces = 1024;
+
+template <int D>
+__global__ void __launch_bounds__(kCombineThreads)
+    combine_kernel(const __grid_constant__ DecodeParams p)
+{
+    __shared__ float s_w[kCombineMaxPieces];
+    __shared__ float s_red[kCombineThreads];
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int seg = blockIdx.x;
+    const int row = blockIdx.y;
+    const int G = p.G;
+    const int T = p.tile_tokens;
+    const int beta = seg / p.g;
+    const int j = seg - beta * p.g;
+    const int L = p.uniform_len > 0 ? p.uniform_len : p.seq_len[beta];
+    const int nt = (L + T - 1) / T;
+    const int seg_first = p.uniform_len > 0 ? seg * nt : p.tile_start[beta] + j * nt;
+    const int c_first = cta_of_tile(seg_first, p.num_tiles, p.decode_grid);
+    const int c_last = cta_of_tile(seg_first + nt - 1, p.num_tiles, p.decode_grid);
+    if (c_first == c_last)
+        return;   // one CTA held the whole segment and wrote the output itself
+    const int np = c_last - c_first + 1;
+    const size_t rec0 = static_cast<size_t>(seg + c_first);
+    const int tid = threadIdx.x;
+    const float NEG_INF = -__int_as_float(0x7f800000);
+
+    float mx = NEG_INF;
+    for (int k = tid; k < np; k += kCombineThreads) {
+        const float v = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
+        s_w[k] = v;
+        mx = fmaxf(mx, v);
+    }
+    s_red[tid] = mx;
+    __syncthreads();
+    for (int off = kCombineThreads / 2; off > 0; off >>= 1) {
+        if (tid < off)
+            s_red[tid] = fmaxf(s_red[tid], s_red[tid + off]);
+        __syncthreads();
+    }
+    mx = s_red[0];
+    __syncthreads();
+    float tot = 0.f;
+    for (int k = tid; k < np; k += kCombineThreads) {
+        const float w = fast_exp2(s_w[k] - mx);
+        s_w[k] = w;
+        tot += w;
+    }
+    s_red[tid] = tot;
+    __syncthreads();
+    for (int off = kCombineThreads / 2; off > 0; off >>= 1) {
+        if (tid < off)
+            s_red[tid] += s_red[tid + off];
+        __syncthreads();
+    }
+    const float inv = fast_rcp(s_red[0]);
+    __syncthreads();
+
+    constexpr int kGroups = kCombineThreads / D;   // pieces summed side by side per column
+    const int e = tid % D;
+    const int grp = tid / D;
+    const float *src = p.part_o + rec0 * G * D + static_cast<size_t>(row) * D + e;
+    float acc = 0.f;
+    for (int k0 = grp; k0 < np; k0 += kGroups * 16) {
+        float v[16];
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+            const int k = k0 + m * kGroups;
+            v[m] = k < np ? __ldcg(src + static_cast<size_t>(k) * G * D) : 0.f;
+        }
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+            const int k = k0 + m * kGroups;
+            if (k < np)
+                acc += s_w[k] * v[m];
+        }
+    }
+    s_red[tid] = acc;
+    __syncthreads();
+    if (grp == 0) {
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < kGroups; ++q)
+            sum += s_red[q * D + e];
+        p.out[(static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G + row) * D + e] =
+            __float2bfloat16_rn(sum * inv);
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
 // append kernel: one thread per 16-byte vector of the new token's K/V rows
 // ------------------------------------------------------------------------------------------------
 
@@ -1148,6 +1249,51 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
     cfg.numAttrs = na;
     void *args[] = {const_cast<CUtensorMap *>(tmap), const_cast<DecodeParams *>(&p)};
     return cudaLaunchKernelExC(&cfg, v.fn, args);
+}
+
+int max_pieces_per_segment(const DecodeParams &p, int T, int grid)
+{
+    const long long N = p.num_tiles;
+    if (grid <= 1 || N <= 0)
+        return 1;
+    if (p.uniform_len > 0) {
+        // Every CTA holds at least floor(N/grid) tiles, so a segment of nt tiles meets at most
+        // ceil((nt - 1) / floor(N/grid)) + 1 of them.
+        const long long nt = (p.uniform_len + T - 1) / T;
+        const long long per = N / grid;
+        if (per <= 0)
+            return grid;
+        return static_cast<int>((nt - 1 + per - 1) / per + 1);
+    }
+    auto cta_of = [&](long long tile) { return static_cast<int>(((tile + 1) * grid - 1) / N); };
+    int worst = 1;
+    for (int beta = 0; beta < p.b; ++beta) {
+        const int nt = (p.seq_len[beta] + T - 1) / T;
+        for (int j = 0; j < p.g; ++j) {
+            const long long first =
+                static_cast<long long>(p.tile_start[beta]) + static_cast<long long>(j) * nt;
+            const int np = cta_of(first + nt - 1) - cta_of(first) + 1;
+            worst = np > worst ? np : worst;
+        }
+    }
+    return worst;
+}
+
+cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.b * p.g), static_cast<unsigned>(p.G));
+    cfg.blockDim = dim3(kCombineThreads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void *args[] = {const_cast<DecodeParams *>(&p)};
+    const void *fn = head_dim == 64 ? reinterpret_cast<const void *>(&combine_kernel<64>)
+                                    : reinterpret_cast<const void *>(&combine_kernel<128>);
+    return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
 cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out)

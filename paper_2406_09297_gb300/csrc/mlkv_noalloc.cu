@@ -176,7 +176,8 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     long long wave = std::min<long long>(static_cast<long long>(ctas_per_sm) * st.sm_count, tiles);
     wave = std::min(wave, fit);
     const long long per = (tiles + wave - 1) / wave;
-    const int grid = static_cast<int>((tiles + per - 1) / per);
+    const int grid = std::min(static_cast<int>((tiles + per - 1) / per),
+                              mlkv::kCombineMaxPiecesHost);
 
     char *base = static_cast<char *>(st.scratch);
     int *err = reinterpret_cast<int *>(base);
@@ -229,9 +230,15 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.num_tiles = static_cast<int>(tiles);
     p.uniform_len = uniform ? seq_lens[0] : 0;
     p.cluster_k = 0;
+    p.tile_tokens = T;
+    p.decode_grid = grid;
+    p.deferred_merge =
+        mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces ? 1 : 0;
     const size_t smem = v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(batch));
     e = mlkv::launch_decode(*v, grid, smem, stream, &tmap, p, nullptr);
     if (e != cudaSuccess)
         return fail(MLKV_ERR_CUDA, "decode launch failed");
+    if (p.deferred_merge && mlkv::launch_combine(p, head_dim, stream) != cudaSuccess)
+        return fail(MLKV_ERR_CUDA, "combine launch failed");
     return MLKV_OK;
 }

@@ -114,12 +114,26 @@ def test_non_finite_cache_contents_beyond_length_do_not_leak():
         cache.sync_status()
 
 
-def test_merge_of_hundreds_of_pieces():
-    # one segment of 313 tiles over 313 CTAs: more pieces than the shared-memory merge holds
-    run_small_case([0], 16, 1, 64, 1, [20000], 20000, seed=15,
-                   options={"grid": 600, "tile_tokens": 64})
-    run_small_case([0], 16, 1, 64, 1, [20000], 20000, seed=16,
-                   options={"grid": 600, "tile_tokens": 64}, fused=True)
+@pytest.mark.parametrize("d", [64, 128])
+def test_merge_of_hundreds_of_pieces(d):
+    # one segment of 313 tiles over 313 CTAs: the decode launch writes partials only and the
+    # combine kernel merges them
+    run_small_case([0], 16, 1, d, 1, [20000], 20000, seed=15,
+                   options={"grid": 600, "tile_tokens": 64}, expect={"last_deferred_merge": 1})
+    run_small_case([0], 16, 1, d, 1, [20000], 20000, seed=16,
+                   options={"grid": 600, "tile_tokens": 64}, fused=True,
+                   expect={"last_deferred_merge": 1})
+
+
+def test_long_single_segments_default_launch():
+    # batch 2 x 2 KV heads of 30000 positions: four segments over the whole GPU
+    run_small_case([0, 0], 8, 2, 64, 2, [30000, 29999], 30000, seed=19, fused=True,
+                   expect={"last_deferred_merge": 1})
+
+
+def test_few_pieces_merge_inline():
+    run_small_case([0], 8, 2, 64, 4, [700, 1, 129, 1000], 1024, seed=20,
+                   options={"grid": 3, "tile_tokens": 64}, expect={"last_deferred_merge": 0})
 
 
 @pytest.mark.parametrize("b,L,tile,k", [(64, 2048, 0, 2), (64, 256, 64, 4)])
