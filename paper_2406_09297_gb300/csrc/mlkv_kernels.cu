@@ -284,6 +284,8 @@ __device__ __forceinline__ int cta_of_tile(int tile, int N, int P)
 template <int D, int T, int STAGES, int NCW>
 struct Plan {
     static constexpr int kThreads = (NCW + 2) * 32;   // consumers, one producer, one epilogue warp
+    // Variants whose ring fits twice in an SM's shared memory ask for two resident CTAs.
+    static constexpr int kMinBlocks = (STAGES * 2 * T * D * 2 <= 80 * 1024) ? 2 : 1;
     static constexpr int kProducer = NCW;             // warp indices
     static constexpr int kEpilogue = NCW + 1;
     static constexpr int kSub = D / 64;               // 128-byte-wide column blocks per row
@@ -606,7 +608,8 @@ __device__ __forceinline__ void epilogue_cluster(const DecodeParams &p, const fl
 // ------------------------------------------------------------------------------------------------
 
 template <int D, int T, int STAGES, int NCW>
-__global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads, 1)
+__global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
+                                  Plan<D, T, STAGES, NCW>::kMinBlocks)
     decode_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ DecodeParams p)
 {
     using PL = Plan<D, T, STAGES, NCW>;
@@ -748,7 +751,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads, 1)
     const float NEG_INF = -__int_as_float(0x7f800000);
 
     int it = 0;
-    int npiece = 0;
+    int nhand = 0;   // pieces handed to the epilogue warp (all but the CTA's last)
     int tile = tile_lo;
     TileWalk<T> wk;
     if (tile < tile_hi)
@@ -968,76 +971,218 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads, 1)
                 o[n][2 * hr + 1] *= f;
             }
         }
-        // Tree over warps with NCW/2 slots.  First level: warp w in [NCW/2, NCW) writes slot
-        // w - NCW/2 and warp r < NCW/2 adds slot r.  Later levels (half < NCW/2): warp w in
-        // [half, 2 half) writes slot w and warp r < half adds slot r + half.  Every slot is
-        // rewritten only by the warp that read it last, so one barrier per level suffices.
-#pragma unroll
-        for (int half = NCW / 2; half >= 1; half >>= 1) {
-            const bool first = (half == NCW / 2);
-            if (warp >= half && warp < 2 * half) {
-                float *dst = merge + (first ? warp - half : warp) * (NO * 4 * 32);
-#pragma unroll
-                for (int n = 0; n < NO; ++n)
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        dst[(n * 4 + c) * 32 + lane] = o[n][c];
+        if (piece_end != tile_hi) {
+            // Tree over warps with NCW/2 slots.  First level: warp w in [NCW/2, NCW) writes slot
+            // w - NCW/2 and warp r < NCW/2 adds slot r.  Later levels (half < NCW/2): warp w in
+            // [half, 2 half) writes slot w and warp r < half adds slot r + half.  Every slot is
+            // rewritten only by the warp that read it last, so one barrier per level suffices.
+    #pragma unroll
+            for (int half = NCW / 2; half >= 1; half >>= 1) {
+                const bool first = (half == NCW / 2);
+                if (warp >= half && warp < 2 * half) {
+                    float *dst = merge + (first ? warp - half : warp) * (NO * 4 * 32);
+    #pragma unroll
+                    for (int n = 0; n < NO; ++n)
+    #pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            dst[(n * 4 + c) * 32 + lane] = o[n][c];
+                }
+                consumer_bar_sync<NCW>();
+                if (warp < half) {
+                    const float *src = merge + (first ? warp : warp + half) * (NO * 4 * 32);
+    #pragma unroll
+                    for (int n = 0; n < NO; ++n)
+    #pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            o[n][c] += src[(n * 4 + c) * 32 + lane];
+                }
             }
-            consumer_bar_sync<NCW>();
-            if (warp < half) {
-                const float *src = merge + (first ? warp : warp + half) * (NO * 4 * 32);
-#pragma unroll
-                for (int n = 0; n < NO; ++n)
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        o[n][c] += src[(n * 4 + c) * 32 + lane];
-            }
-        }
 
-        // Warp 0 hands the piece to the epilogue warp through a double-buffered slot and the
-        // consumers move on to the next piece at once.
-        if (warp == 0) {
-            const int rb = npiece & 1;
-            if (npiece >= 2 && !flags[0] &&
-                !mbar_wait(bar_res_empty + 8 * rb, ((npiece >> 1) - 1) & 1)) {
-                flags[0] = 1;
-                atomicOr(p.err, kErrWaitEmpty);
+            // Warp 0 hands the piece to the epilogue warp through a double-buffered slot and the
+            // consumers move on to the next piece at once.
+            if (warp == 0) {
+                const int rb = nhand & 1;
+                if (nhand >= 2 && !flags[0] &&
+                    !mbar_wait(bar_res_empty + 8 * rb, ((nhand >> 1) - 1) & 1)) {
+                    flags[0] = 1;
+                    atomicOr(p.err, kErrWaitEmpty);
+                }
+                uint8_t *slot = smem + PL::kRes + rb * PL::kResBytes;
+                float *ro = reinterpret_cast<float *>(slot);
+                float *rlse = reinterpret_cast<float *>(slot + PL::kResO);
+                int *meta = reinterpret_cast<int *>(slot + PL::kResO + 64);
+    #pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    const int row = qr + 8 * hr;
+                    if (row < G) {
+    #pragma unroll
+                        for (int n = 0; n < NO; ++n)
+                            *reinterpret_cast<float2 *>(ro + row * D + n * 8 + qc) =
+                                make_float2(o[n][2 * hr], o[n][2 * hr + 1]);
+                        if (qc == 0)
+                            rlse[row] = lse[hr];
+                    }
+                }
+                if (lane == 0) {
+                    meta[kMetaBeta] = beta;
+                    meta[kMetaJ] = j;
+                    meta[kMetaSeg] = seg;
+                    meta[kMetaWhole] = (piece_first == seg_first && piece_end == seg_end) ? 1 : 0;
+                    meta[kMetaFirst] = cta_of_tile(seg_first, N, P);
+                    meta[kMetaLast] = cta_of_tile(seg_end - 1, N, P);
+                    meta[kMetaStop] = 0;
+                }
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(bar_res_full + 8 * rb);
             }
-            uint8_t *slot = smem + PL::kRes + rb * PL::kResBytes;
-            float *ro = reinterpret_cast<float *>(slot);
-            float *rlse = reinterpret_cast<float *>(slot + PL::kResO);
-            int *meta = reinterpret_cast<int *>(slot + PL::kResO + 64);
+            ++nhand;
+        } else {
+            // ---- the CTA's last piece: every tile has been consumed and no copy is pending, so
+            // the stage ring is free.  All consumer warps finish the piece: one exchange through
+            // the ring instead of the tree, and the output / partial / merge work shared by all
+            // consumer threads instead of the epilogue warp.
+            float *fbuf = reinterpret_cast<float *>(smem);         // [NCW][16][D] f32
+            float *flse = fbuf + NCW * 16 * D;                      // [16]
 #pragma unroll
             for (int hr = 0; hr < 2; ++hr) {
                 const int row = qr + 8 * hr;
                 if (row < G) {
 #pragma unroll
                     for (int n = 0; n < NO; ++n)
-                        *reinterpret_cast<float2 *>(ro + row * D + n * 8 + qc) =
+                        *reinterpret_cast<float2 *>(fbuf + (warp * 16 + row) * D + n * 8 + qc) =
                             make_float2(o[n][2 * hr], o[n][2 * hr + 1]);
-                    if (qc == 0)
-                        rlse[row] = lse[hr];
+                    if (warp == 0 && qc == 0)
+                        flse[row] = lse[hr];
                 }
             }
-            if (lane == 0) {
-                meta[kMetaBeta] = beta;
-                meta[kMetaJ] = j;
-                meta[kMetaSeg] = seg;
-                meta[kMetaWhole] = (piece_first == seg_first && piece_end == seg_end) ? 1 : 0;
-                meta[kMetaFirst] = cta_of_tile(seg_first, N, P);
-                meta[kMetaLast] = cta_of_tile(seg_end - 1, N, P);
-                meta[kMetaStop] = 0;
+            consumer_bar_sync<NCW>();
+            const int ctid = threadIdx.x;
+            const bool whole = (piece_first == seg_first && piece_end == seg_end);
+            __nv_bfloat16 *ob =
+                p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+            constexpr int kPairs = NCW * 32;   // float2 outputs per pass
+            // mode: 0 whole, 1 cluster sender, 2 cluster leader, 3 partial record
+            const int rank = p.cluster_k > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+            const int mode = whole ? 0 : (p.cluster_k > 1 ? (rank != 0 ? 1 : 2) : 3);
+            const uint32_t cslots = sbase + PL::kTables;
+            const uint8_t *cs = smem + PL::kTables;
+            uint32_t remote = 0;
+            if (mode == 1)
+                remote = map_to_rank(cslots + (rank - 1) * PL::kResBytes, 0);
+            if (mode == 2) {
+                if (ctid == 0 && !flags[0] && !mbar_wait_cluster(bar_cluster, 0)) {
+                    flags[0] = 1;
+                    atomicOr(p.err, kErrWaitFull);
+                }
+                consumer_bar_sync<NCW>();
             }
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(bar_res_full + 8 * rb);
+            const size_t piece = static_cast<size_t>(seg + cta);
+            float *po = p.part_o + piece * G * D;
+#pragma unroll 1
+            for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
+                const int row = i / D, e = i - row * D;
+                float2 v = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int w = 0; w < NCW; ++w) {
+                    const float2 x = *reinterpret_cast<const float2 *>(fbuf + (w * 16 + row) * D + e);
+                    v.x += x.x;
+                    v.y += x.y;
+                }
+                if (mode == 0) {
+                    *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(v.x, v.y);
+                } else if (mode == 1) {
+                    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(remote + i * 4),
+                                 "f"(v.x), "f"(v.y)
+                                 : "memory");
+                } else if (mode == 2) {
+                    if (!flags[0]) {
+                        float mx = flse[row];
+                        for (int r = 1; r < p.cluster_k; ++r)
+                            mx = fmaxf(mx, reinterpret_cast<const float *>(
+                                               cs + (r - 1) * PL::kResBytes + PL::kResO)[row]);
+                        float w = fast_exp2(flse[row] - mx);
+                        float tot = w, ax = w * v.x, ay = w * v.y;
+                        for (int r = 1; r < p.cluster_k; ++r) {
+                            const float *sl =
+                                reinterpret_cast<const float *>(cs + (r - 1) * PL::kResBytes);
+                            w = fast_exp2(sl[PL::kResO / 4 + row] - mx);
+                            tot += w;
+                            const float2 x = *reinterpret_cast<const float2 *>(sl + i);
+                            ax += w * x.x;
+                            ay += w * x.y;
+                        }
+                        const float inv = fast_rcp(tot);
+                        *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(ax * inv, ay * inv);
+                    }
+                } else {
+                    *reinterpret_cast<float2 *>(po + i) = v;
+                }
+            }
+            if (mode == 1) {
+                if (ctid < G)
+                    st_cluster_f32(remote + PL::kResO + ctid * 4, flse[ctid]);
+                fence_acq_rel_cluster();
+                consumer_bar_sync<NCW>();
+                if (ctid == 0)
+                    mbar_arrive_remote(map_to_rank(bar_cluster, 0));
+            } else if (mode == 3) {
+                if (ctid < G)
+                    p.part_lse[piece * G + ctid] = flse[ctid];
+                if (!p.deferred_merge) {
+                    const int c_first = cta_of_tile(seg_first, N, P);
+                    const int c_last = cta_of_tile(seg_end - 1, N, P);
+                    __threadfence();
+                    consumer_bar_sync<NCW>();
+                    if (ctid == 0) {
+                        const unsigned prev = atomic_add_acq_rel_gpu(&p.counters[seg], 1u);
+                        flags[1] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
+                    }
+                    consumer_bar_sync<NCW>();
+                    if (flags[1]) {
+                        // Last finisher of the segment: merge its <= 4 records (own included).
+                        const int np = c_last - c_first + 1;
+                        const size_t rec0 = static_cast<size_t>(seg + c_first);
+#pragma unroll 1
+                        for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
+                            const int row = i / D;
+                            float lv[kInlineMergeMaxPieces];
+                            float2 ov[kInlineMergeMaxPieces];
+                            float mx = NEG_INF;
+#pragma unroll
+                            for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
+                                lv[k] = NEG_INF;
+                                ov[k] = make_float2(0.f, 0.f);
+                                if (k < np) {
+                                    lv[k] = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
+                                    ov[k] = __ldcg(reinterpret_cast<const float2 *>(
+                                        p.part_o + (rec0 + k) * G * D + i));
+                                }
+                                mx = fmaxf(mx, lv[k]);
+                            }
+                            float tot = 0.f, ax = 0.f, ay = 0.f;
+#pragma unroll
+                            for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
+                                const float w = fast_exp2(lv[k] - mx);   // 0 past np
+                                tot += w;
+                                ax += w * ov[k].x;
+                                ay += w * ov[k].y;
+                            }
+                            const float inv = fast_rcp(tot);
+                            *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(ax * inv, ay * inv);
+                        }
+                        if (ctid == 0)
+                            p.counters[seg] = 0u;
+                    }
+                    consumer_bar_sync<NCW>();   // flags[1] is reused
+                }
+            }
         }
-        ++npiece;
     }
     // Tell the epilogue warp that no piece follows.
     if (warp == 0) {
-        const int rb = npiece & 1;
-        if (npiece >= 2 && !flags[0] && !mbar_wait(bar_res_empty + 8 * rb, ((npiece >> 1) - 1) & 1)) {
+        const int rb = nhand & 1;
+        if (nhand >= 2 && !flags[0] && !mbar_wait(bar_res_empty + 8 * rb, ((nhand >> 1) - 1) & 1)) {
             flags[0] = 1;
             atomicOr(p.err, kErrWaitEmpty);
         }
