@@ -246,6 +246,8 @@ def run(args, w):
         cache.set_option("grid", args.grid)
     if args.l2_persist:
         cache.set_option("l2_persist", 1)
+    if args.no_pdl:
+        cache.set_option("pdl", 0)
     owners = w.owners()
     seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
     out = [torch.empty((w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda") for _ in range(w.l)]
@@ -419,6 +421,7 @@ def main():
     ap.add_argument("--tile", type=int, default=0)
     ap.add_argument("--grid", type=int, default=0)
     ap.add_argument("--l2-persist", action="store_true")
+    ap.add_argument("--no-pdl", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -154,6 +154,9 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through
  *                  distributed shared memory; 0 = always the global-memory merge
+ *   "pdl"          1 (default) = programmatic dependent launch: a decode launch's set-up overlaps
+ *                  the previous kernel of the stream (it touches no global memory before that
+ *                  kernel has completed); 0 = plain stream order
  * Read-only (mlkv_get_option): "sm_count", "l2_bytes", "max_grid", "ctas_per_sm", and for the most
  * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.

@@ -114,6 +114,7 @@ struct mlkv_cache {
     int grid = 0;
     int l2_persist = 0;
     int cluster = 1;            // allow the DSMEM cluster merge
+    int pdl = 1;                // programmatic dependent launch
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0;
     // per-variant launch state
@@ -531,11 +532,11 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                         (cluster_k > 1 ? (cluster_k - 1) * var->v->res_bytes
                                        : (uniform ? 0 : mlkv::table_bytes(c->b)));
     cudaError_t e = mlkv::launch_decode(*var->v, grid, smem, static_cast<cudaStream_t>(cuda_stream),
-                                        &var->tmap, p, winp);
+                                        &var->tmap, p, winp, c->pdl != 0);
     if (e != cudaSuccess)
         return fail_cuda(e, "decode launch");
     if (p.deferred_merge) {
-        e = mlkv::launch_combine(p, c->d, static_cast<cudaStream_t>(cuda_stream));
+        e = mlkv::launch_combine(p, c->d, static_cast<cudaStream_t>(cuda_stream), c->pdl != 0);
         if (e != cudaSuccess)
             return fail_cuda(e, "combine launch");
     }
@@ -669,6 +670,12 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->cluster = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "pdl") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "pdl must be 0 or 1");
+        c->pdl = static_cast<int>(value);
+        return MLKV_OK;
+    }
     return fail(MLKV_ERR_INVALID_ARG, "unknown option '%s'", key);
 }
 
@@ -690,6 +697,10 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "cluster") == 0) {
         *value = c->cluster;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "pdl") == 0) {
+        *value = c->pdl;
         return MLKV_OK;
     }
     if (std::strcmp(key, "last_grid") == 0) {

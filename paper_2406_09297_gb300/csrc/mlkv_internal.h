@@ -72,9 +72,11 @@ const DecodeVariant *find_decode_variant(int head_dim, int tile_tokens);
 // per-block maximum); call once per device before the first launch.
 cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem);
 
+// pdl: launch with programmatic stream serialization (the kernel's prologue may overlap the
+// previous kernel of the stream; it waits on griddepcontrol.wait before touching global memory).
 cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
                           const CUtensorMap *tmap, const DecodeParams &p,
-                          const cudaAccessPolicyWindow *window);
+                          const cudaAccessPolicyWindow *window, bool pdl = true);
 
 // Sets the calling thread's mlkv_last_error() text.
 void set_last_error(const char *msg);
@@ -85,7 +87,8 @@ int max_pieces_per_segment(const DecodeParams &p, int T, int grid);
 
 // Merges the partials of every split segment of the decode launch described by p (which must
 // have deferred_merge = 1), launched right after it on the same stream.
-cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream);
+cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream,
+                           bool pdl = true);
 
 // Pieces per segment above which the decode launch defers its merges to combine_kernel.
 constexpr int kInlineMergeMaxPieces = 4;

@@ -333,10 +333,16 @@ __device__ __forceinline__ uint32_t cluster_ctarank()
     return r;
 }
 
-__device__ __forceinline__ void cluster_sync_all()
+// Every thread of a cluster launch arrives once, right after set-up, and waits once, late: before
+// its first access to another CTA's shared memory and before it exits.
+__device__ __forceinline__ void cluster_arrive()
 {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
-                 ::: "memory");
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait()
+{
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // Address, in the cluster's shared window, of this CTA's shared address `a` in CTA `rank`.
@@ -347,26 +353,20 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t a, uint32_t rank)
     return r;
 }
 
-__device__ __forceinline__ void st_cluster_v4(uint32_t a, float4 v)
+// Asynchronous store into another CTA's shared memory that completes `bytes` of the transaction
+// count of that CTA's mbarrier `mbar` (both addresses in the cluster window).
+__device__ __forceinline__ void st_async_v2(uint32_t a, float x, float y, uint32_t mbar)
 {
-    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(v.x), "f"(v.y),
-                 "f"(v.z), "f"(v.w)
-                 : "memory");
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(a),
+        "f"(x), "f"(y), "r"(mbar)
+        : "memory");
 }
 
-__device__ __forceinline__ void st_cluster_f32(uint32_t a, float v)
+__device__ __forceinline__ void st_async_f32(uint32_t a, float x, uint32_t mbar)
 {
-    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
-}
-
-__device__ __forceinline__ void fence_acq_rel_cluster()
-{
-    asm volatile("fence.acq_rel.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr)
-{
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];" ::"r"(a),
+                 "f"(x), "r"(mbar)
                  : "memory");
 }
 
@@ -544,65 +544,6 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
         p.counters[seg] = 0u;
 }
 
-// Cluster mode: the k CTAs of a cluster hold the k equal pieces of one segment.  Ranks 1..k-1
-// write their (o, lse) into slot rank-1 of the leader's shared memory over DSMEM and arrive on the
-// leader's cluster barrier; the leader merges the k results from its own shared memory.
-template <int D, int RES_BYTES, int RES_O>
-__device__ __forceinline__ void epilogue_cluster(const DecodeParams &p, const float *ro,
-                                                 const float *rlse, const int *meta,
-                                                 uint8_t *cslots, uint32_t cslots_addr,
-                                                 uint32_t bar_cluster, int lane,
-                                                 volatile int *flags)
-{
-    const int G = p.G;
-    const int k = p.cluster_k;
-    const uint32_t rank = cluster_ctarank();
-    if (rank != 0) {
-        const uint32_t dst = map_to_rank(cslots_addr + (rank - 1) * RES_BYTES, 0);
-        for (int i = lane * 4; i < G * D; i += 128)
-            st_cluster_v4(dst + i * 4, *reinterpret_cast<const float4 *>(ro + i));
-        if (lane < G)
-            st_cluster_f32(dst + RES_O + lane * 4, rlse[lane]);
-        fence_acq_rel_cluster();
-        __syncwarp();
-        if (lane == 0)
-            mbar_arrive_remote(map_to_rank(bar_cluster, 0));
-        return;
-    }
-    if (!mbar_wait_cluster(bar_cluster, 0)) {
-        flags[0] = 1;
-        atomicOr(p.err, kErrWaitFull);
-        return;
-    }
-    const int beta = meta[kMetaBeta], j = meta[kMetaJ];
-    __nv_bfloat16 *ob = p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
-    for (int i = lane * 4; i < G * D; i += 128) {
-        const int row = i / D;
-        float mx = rlse[row];
-        for (int r = 1; r < k; ++r)
-            mx = fmaxf(mx, reinterpret_cast<const float *>(cslots + (r - 1) * RES_BYTES + RES_O)[row]);
-        float w = fast_exp2(rlse[row] - mx);
-        float tot = w;
-        float4 v = *reinterpret_cast<const float4 *>(ro + i);
-        float4 acc = make_float4(w * v.x, w * v.y, w * v.z, w * v.w);
-        for (int r = 1; r < k; ++r) {
-            const float *slot = reinterpret_cast<const float *>(cslots + (r - 1) * RES_BYTES);
-            w = fast_exp2(slot[RES_O / 4 + row] - mx);
-            tot += w;
-            v = *reinterpret_cast<const float4 *>(slot + i);
-            acc.x += w * v.x;
-            acc.y += w * v.y;
-            acc.z += w * v.z;
-            acc.w += w * v.w;
-        }
-        const float inv = fast_rcp(tot);
-        uint2 w2;
-        w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-        w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-        *reinterpret_cast<uint2 *>(ob + i) = w2;
-    }
-}
-
 // ------------------------------------------------------------------------------------------------
 // decode kernel
 // ------------------------------------------------------------------------------------------------
@@ -648,7 +589,12 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             mbar_init(bar_res_full + 8 * r, 1);
             mbar_init(bar_res_empty + 8 * r, 1);
         }
-        mbar_init(bar_cluster, p.cluster_k > 1 ? p.cluster_k - 1 : 1);
+        mbar_init(bar_cluster, 1);
+        if (p.cluster_k > 1 && cluster_ctarank() == 0) {
+            // The leader expects every other rank's result: G*D outputs and G lse values, f32.
+            mbar_arrive_expect_tx(bar_cluster, static_cast<uint32_t>(
+                                                   (p.cluster_k - 1) * (p.G * D + p.G) * 4));
+        }
         flags[0] = 0;   // abort
         fence_barrier_init();
     }
@@ -664,19 +610,22 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     }
     __syncthreads();
     if (p.cluster_k > 1)
-        cluster_sync_all();   // every rank's barriers exist before any remote arrival
+        cluster_arrive();   // this CTA's barriers exist; waited on before any remote access
+    // The tile walk reads only the parameters and the shared tables: set it up before the wait.
+    TileWalk<T> wk;
+    if (tile_lo < tile_hi)
+        wk.init(p, s_len, s_start, tile_lo);
     // Everything above overlaps the previous kernel's tail; global memory is touched only below.
     grid_dependency_wait();
-    grid_dependents_launch();
+    if (warp != PL::kProducer)
+        grid_dependents_launch();
 
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
         if (lane != 0)
-            return;
+            grid_dependents_launch();
+        if (lane == 0) {
         int issued = 0;
-        TileWalk<T> wk;
-        if (tile_lo < tile_hi)
-            wk.init(p, s_len, s_start, tile_lo);
         for (int tile = tile_lo; tile < tile_hi; ++tile) {
             const int s = issued % STAGES;
             if (issued >= STAGES && !flags[0] &&
@@ -699,13 +648,21 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
             }
             ++issued;
+            if (issued == STAGES)
+                grid_dependents_launch();   // the first loads are in flight
             wk.next(p, s_len, s_start);
         }
+        if (issued < STAGES)
+            grid_dependents_launch();
         // No copy may still be in flight when the CTA exits.
         const int first = issued > STAGES ? issued - STAGES : 0;
         for (int k = first; k < issued; ++k)
             if (!mbar_wait(bar_full + 8 * (k % STAGES), (k / STAGES) & 1))
                 atomicOr(p.err, kErrDrain);
+        }
+        __syncwarp();
+        if (p.cluster_k > 1)
+            cluster_wait();
         return;
     }
 
@@ -714,30 +671,31 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         float *s_w = reinterpret_cast<float *>(smem + PL::kEpiW);
         for (int k = 0;; ++k) {
             const int rb = k & 1;
-            if (!mbar_wait(bar_res_full + 8 * rb, (k >> 1) & 1)) {
+            int ok = 1;
+            if (lane == 0 && !mbar_wait(bar_res_full + 8 * rb, (k >> 1) & 1)) {
                 flags[0] = 1;
                 atomicOr(p.err, kErrWaitFull);
-                return;
+                ok = 0;
             }
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok)
+                break;
             const uint8_t *slot = smem + PL::kRes + rb * PL::kResBytes;
             const int *meta = reinterpret_cast<const int *>(slot + PL::kResO + 64);
             if (meta[kMetaStop])
-                return;
-            if (!flags[0]) {
-                if (p.cluster_k > 1)
-                    epilogue_cluster<D, PL::kResBytes, PL::kResO>(
-                        p, reinterpret_cast<const float *>(slot),
-                        reinterpret_cast<const float *>(slot + PL::kResO), meta,
-                        smem + PL::kTables, sbase + PL::kTables, bar_cluster, lane, flags);
-                else
-                    epilogue_piece<D>(p, reinterpret_cast<const float *>(slot),
-                                      reinterpret_cast<const float *>(slot + PL::kResO), meta,
-                                      s_w, PL::kEpiCap, lane, cta);
-            }
+                break;
+            if (!flags[0])
+                epilogue_piece<D>(p, reinterpret_cast<const float *>(slot),
+                                  reinterpret_cast<const float *>(slot + PL::kResO), meta, s_w,
+                                  PL::kEpiCap, lane, cta);
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(bar_res_empty + 8 * rb);
         }
+        __syncwarp();
+        if (p.cluster_k > 1)
+            cluster_wait();
+        return;
     }
 
     // -------------------------------- consumer warps -------------------------------------------
@@ -753,9 +711,6 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     int it = 0;
     int nhand = 0;   // pieces handed to the epilogue warp (all but the CTA's last)
     int tile = tile_lo;
-    TileWalk<T> wk;
-    if (tile < tile_hi)
-        wk.init(p, s_len, s_start, tile);
 
     while (tile < tile_hi) {
         const int beta = wk.beta;
@@ -936,8 +891,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         }
 
         // ---------------- end of piece: merge the warps (no atomics) ----------------
-        // Row statistics of every warp -> per-row maximum and total; each warp scales its own
-        // accumulators by 2^(m_w - m*) / l*, then a tree over warps sums them into warp 0.
+        // Row statistics of every warp -> per-row maximum m* and total l*; each warp's
+        // accumulators are weighted by 2^(m_w - m*) / l* and the warps summed.
 #pragma unroll
         for (int hr = 0; hr < 2; ++hr) {
             l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
@@ -949,6 +904,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             red_l[warp * 16 + qr] = l_run[0];
             red_l[warp * 16 + qr + 8] = l_run[1];
         }
+        // The barrier also guarantees that every warp is done with the ring's tiles.
         consumer_bar_sync<NCW>();
         float lse[2];
 #pragma unroll
@@ -972,6 +928,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             }
         }
         if (piece_end != tile_hi) {
+            // A piece before the CTA's last: tree over warps, result to the epilogue warp, and
+            // the consumers go straight on to the next piece.
             // Tree over warps with NCW/2 slots.  First level: warp w in [NCW/2, NCW) writes slot
             // w - NCW/2 and warp r < NCW/2 adds slot r.  Later levels (half < NCW/2): warp w in
             // [half, 2 half) writes slot w and warp r < half adds slot r + half.  Every slot is
@@ -1039,9 +997,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             ++nhand;
         } else {
             // ---- the CTA's last piece: every tile has been consumed and no copy is pending, so
-            // the stage ring is free.  All consumer warps finish the piece: one exchange through
-            // the ring instead of the tree, and the output / partial / merge work shared by all
-            // consumer threads instead of the epilogue warp.
+            // the stage ring is free.  The warps write their weighted accumulators there (one
+            // barrier) and every consumer thread sums and finishes its share of the outputs.
             float *fbuf = reinterpret_cast<float *>(smem);         // [NCW][16][D] f32
             float *flse = fbuf + NCW * 16 * D;                      // [16]
 #pragma unroll
@@ -1056,6 +1013,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                         flse[row] = lse[hr];
                 }
             }
+            if (p.cluster_k > 1)
+                cluster_wait();   // the partner CTAs' barriers exist
             consumer_bar_sync<NCW>();
             const int ctid = threadIdx.x;
             const bool whole = (piece_first == seg_first && piece_end == seg_end);
@@ -1067,9 +1026,11 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             const int mode = whole ? 0 : (p.cluster_k > 1 ? (rank != 0 ? 1 : 2) : 3);
             const uint32_t cslots = sbase + PL::kTables;
             const uint8_t *cs = smem + PL::kTables;
-            uint32_t remote = 0;
-            if (mode == 1)
+            uint32_t remote = 0, remote_bar = 0;
+            if (mode == 1) {
                 remote = map_to_rank(cslots + (rank - 1) * PL::kResBytes, 0);
+                remote_bar = map_to_rank(bar_cluster, 0);
+            }
             if (mode == 2) {
                 if (ctid == 0 && !flags[0] && !mbar_wait_cluster(bar_cluster, 0)) {
                     flags[0] = 1;
@@ -1082,6 +1043,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
 #pragma unroll 1
             for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
                 const int row = i / D, e = i - row * D;
+                const float lse_row = flse[row];
                 float2 v = make_float2(0.f, 0.f);
 #pragma unroll
                 for (int w = 0; w < NCW; ++w) {
@@ -1092,16 +1054,14 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 if (mode == 0) {
                     *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(v.x, v.y);
                 } else if (mode == 1) {
-                    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(remote + i * 4),
-                                 "f"(v.x), "f"(v.y)
-                                 : "memory");
+                    st_async_v2(remote + i * 4, v.x, v.y, remote_bar);
                 } else if (mode == 2) {
                     if (!flags[0]) {
-                        float mx = flse[row];
+                        float mx = lse_row;
                         for (int r = 1; r < p.cluster_k; ++r)
                             mx = fmaxf(mx, reinterpret_cast<const float *>(
                                                cs + (r - 1) * PL::kResBytes + PL::kResO)[row]);
-                        float w = fast_exp2(flse[row] - mx);
+                        float w = fast_exp2(lse_row - mx);
                         float tot = w, ax = w * v.x, ay = w * v.y;
                         for (int r = 1; r < p.cluster_k; ++r) {
                             const float *sl =
@@ -1120,12 +1080,9 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 }
             }
             if (mode == 1) {
+                // the leader's barrier completes when all these bytes have landed
                 if (ctid < G)
-                    st_cluster_f32(remote + PL::kResO + ctid * 4, flse[ctid]);
-                fence_acq_rel_cluster();
-                consumer_bar_sync<NCW>();
-                if (ctid == 0)
-                    mbar_arrive_remote(map_to_rank(bar_cluster, 0));
+                    st_async_f32(remote + PL::kResO + ctid * 4, flse[ctid], remote_bar);
             } else if (mode == 3) {
                 if (ctid < G)
                     p.part_lse[piece * G + ctid] = flse[ctid];
@@ -1366,7 +1323,7 @@ cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem)
 
 cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
                           const CUtensorMap *tmap, const DecodeParams &p,
-                          const cudaAccessPolicyWindow *window)
+                          const cudaAccessPolicyWindow *window, bool pdl)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -1375,9 +1332,11 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
     cfg.stream = stream;
     cudaLaunchAttribute attr[3];
     int na = 0;
-    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[na].val.programmaticStreamSerializationAllowed = 1;
-    ++na;
+    if (pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
     if (p.cluster_k > 1) {
         attr[na].id = cudaLaunchAttributeClusterDimension;
         attr[na].val.clusterDim.x = static_cast<unsigned>(p.cluster_k);
@@ -1424,7 +1383,7 @@ int max_pieces_per_segment(const DecodeParams &p, int T, int grid)
     return worst;
 }
 
-cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream)
+cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream, bool pdl)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.b * p.g), static_cast<unsigned>(p.G));
@@ -1434,7 +1393,7 @@ cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t str
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 1 : 0;
     void *args[] = {const_cast<DecodeParams *>(&p)};
     const void *fn = head_dim == 64 ? reinterpret_cast<const void *>(&combine_kernel<64>)
                                     : reinterpret_cast<const void *>(&combine_kernel<128>);
