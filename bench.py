@@ -6,11 +6,12 @@ for the others.  Default workload: Pythia-160M-shaped
 MLKV-2 (12 layers, 12 query heads, head_dim 64, owner layers 0 and 6 with one KV head each),
 batch 64, context 2048, bf16 Q/K/V ~ N(0,1) from a seeded generator.
 
-value   decode tokens/s of the whole job = batch * world / step time; device time of a CUDA-graph
-        replay of the step, CUDA events on the launching stream, L2 flushed (a 512 MiB write)
-        before every step outside the timed events.
-e2e     the same metric through the C ABI called from Python per layer, with the step's inputs
-        copied from pinned host memory and its outputs copied back inside the timed region.
+value   decode tokens/s of the whole job = batch * world / step time; device time of one
+        mlkv_decode_step call (the library replays the step's launches from a CUDA graph), CUDA
+        events on the launching stream, L2 flushed (a 512 MiB write) before every step outside
+        the timed events.
+e2e     the same metric end to end: the step's Q and new K/V copied from pinned host memory, one
+        mlkv_decode_step call, every layer's output copied back, all inside the timed region.
 roofline  the decode kernel: logical K/V bytes per launch / mean launch duration (CUDA events
         around each launch) against the measured HBM copy bandwidth.
 cpu_baseline  the fp64 oracle (test infrastructure) on the host cores, on a bounded sample.
@@ -250,32 +251,22 @@ def run(args, w):
         cache.set_option("pdl", 0)
     owners = w.owners()
     seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
-    out = [torch.empty((w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda") for _ in range(w.l)]
+    Qs = torch.stack(Q)                              # [l][b][h][d]
+    Ks = torch.stack([Kn[n] for n in owners])        # [m][b][g][d], slot order
+    Vs = torch.stack([Vn[n] for n in owners])
+    outs = torch.empty((w.l, w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda")
+    out = list(outs.unbind(0))
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     torch.cuda.synchronize()
 
     def step():
-        # owner layers store their new token and attend in one launch; the others only attend
-        for n in range(w.l):
-            if n in Kn:
-                cache.append_decode_attention(n, Kn[n], Vn[n], Q[n], out[n], seq_lens)
-            else:
-                cache.decode_attention(n, Q[n], out[n], seq_lens)
+        # one call: every layer in order, owner layers storing their new token and attending
+        # in one launch; replayed from the CUDA graph the library recorded on the first call
+        cache.decode_step(Qs, Ks, Vs, outs, seq_lens)
 
-    launches_per_step = w.l
     step()
     cache.sync_status()
-
-    # ---- device-timed step: CUDA graph of the whole step --------------------------------------
-    graph = torch.cuda.CUDAGraph()
-    s = torch.cuda.Stream()
-    s.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(s):
-        step()
-    torch.cuda.current_stream().wait_stream(s)
-    with torch.cuda.graph(graph):
-        step()
-    torch.cuda.synchronize()
+    launches_per_step = w.l * (2 if cache.get_option("last_deferred_merge") else 1)
 
     def barrier():
         if dist is not None:
@@ -284,7 +275,7 @@ def run(args, w):
 
     for _ in range(args.warmup):
         flush.zero_()
-        graph.replay()
+        step()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     barrier()
@@ -292,7 +283,7 @@ def run(args, w):
         for k in range(args.steps):
             flush.zero_()
             ev[k][0].record()
-            graph.replay()
+            step()
             ev[k][1].record()
         barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
@@ -324,7 +315,7 @@ def run(args, w):
     torch.cuda.synchronize()
     kms = [[a.elapsed_time(b) for a, b in row] for row in kev]
     layer_ms = [statistics.median(kms[k][n] for k in range(args.steps)) for n in range(w.l)]
-    mean_kernel_ms = ms / launches_per_step
+    mean_kernel_ms = ms / w.l   # decode launches (a combine launch, if any, rides with each)
     kv_layer = kv_bytes_per_layer(w, seq_lens)
     qo_layer = 2 * w.b * w.h * w.d * 2
     alg_bytes = kv_layer + qo_layer
@@ -336,28 +327,24 @@ def run(args, w):
     traffic = _recorded_traffic(w)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
-    host_q = torch.stack(Q).cpu().pin_memory()
-    host_k = {n: Kn[n].cpu().pin_memory() for n in owners}
-    host_v = {n: Vn[n].cpu().pin_memory() for n in owners}
+    host_q = Qs.cpu().pin_memory()
+    host_k = Ks.cpu().pin_memory()
+    host_v = Vs.cpu().pin_memory()
     host_out = torch.empty((w.l, w.b, w.h, w.d), dtype=torch.bfloat16).pin_memory()
     dq = torch.empty_like(host_q, device="cuda")
-    dk = {n: torch.empty_like(host_k[n], device="cuda") for n in owners}
-    dv = {n: torch.empty_like(host_v[n], device="cuda") for n in owners}
+    dk = torch.empty_like(host_k, device="cuda")
+    dv = torch.empty_like(host_v, device="cuda")
     dout = torch.empty_like(host_out, device="cuda")
-    h2d = host_q.numel() * 2 + sum(host_k[n].numel() * 2 * 2 for n in owners)
+    h2d = (host_q.numel() + host_k.numel() + host_v.numel()) * 2
     d2h = host_out.numel() * 2
 
     def e2e_step():
+        # the user's view: this step's inputs from pinned host memory, one library call for the
+        # step, every layer's output back to pinned host memory
         dq.copy_(host_q, non_blocking=True)
-        for n in owners:
-            dk[n].copy_(host_k[n], non_blocking=True)
-            dv[n].copy_(host_v[n], non_blocking=True)
-        for n in range(w.l):
-            if n in dk:
-                mlkv.mlkv_append_decode_attention(cache.handle, n, dk[n], dv[n], dq[n], dout[n],
-                                                  seq_lens)
-            else:
-                mlkv.mlkv_decode_attention(cache.handle, n, dq[n], dout[n], seq_lens)
+        dk.copy_(host_k, non_blocking=True)
+        dv.copy_(host_v, non_blocking=True)
+        mlkv.mlkv_decode_step(cache.handle, dq, dk, dv, dout, seq_lens)
         host_out.copy_(dout, non_blocking=True)
 
     for _ in range(args.warmup):

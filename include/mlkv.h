@@ -120,6 +120,25 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
                                  void *cuda_stream);
 
 /*
+ * mlkv_decode_step - one decode step of the whole model: for every layer n in order, the calls
+ * mlkv_append_decode_attention (layers that own KV heads) or mlkv_decode_attention (the others).
+ *
+ * Paper: Sec. 3 (the layer stack of Eq. 18: owner layers store their token, every layer attends
+ * over its owner's cache) and Sec. 4.5 (autoregressive decoding, one token per step).
+ *
+ *   Q        device bf16 [l][batch][h][d], every layer's queries
+ *   K, V     device bf16 [m][batch][g][d], every owner layer's new token, in slot order
+ *   out      device bf16 [l][batch][h][d]
+ *   seq_lens host int32[batch], as for mlkv_decode_attention
+ * With option "step_graph" = 1 (default) the launches of a step are recorded into a CUDA graph on
+ * the first call and replayed by later calls with the same pointers, lengths and options (new
+ * values in the same buffers are fine); a change re-records.  When cuda_stream is itself being
+ * captured the launches are issued directly, into the caller's graph.
+ */
+int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
+                     const int *seq_lens, void *cuda_stream);
+
+/*
  * mlkv_load_prefix - bulk-stores positions [0, len) of an owner layer's keys and values
  * (prefill).  K, V: device bf16 [batch][g][len][d].  No-op (MLKV_OK) for a non-owner layer.
  * Paper: Sec. 4.5 starts decoding from a pre-filled ("dummy") cache.
@@ -157,8 +176,10 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *   "pdl"          1 (default) = programmatic dependent launch: a decode launch's set-up overlaps
  *                  the previous kernel of the stream (it touches no global memory before that
  *                  kernel has completed); 0 = plain stream order
+ *   "step_graph"   1 (default) = mlkv_decode_step replays a recorded CUDA graph (see there)
  * Read-only (mlkv_get_option): "sm_count", "l2_bytes", "max_grid", "ctas_per_sm", and for the most
- * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge).
+ * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge),
+ * "last_deferred_merge", and "step_graph_replays" (graph launches by mlkv_decode_step).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.
  */
 int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);

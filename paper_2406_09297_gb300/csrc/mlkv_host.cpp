@@ -115,6 +115,23 @@ struct mlkv_cache {
     int l2_persist = 0;
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
+    // mlkv_decode_step's recorded graph and the arguments it was recorded for
+    int step_graph = 1;
+    cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
+    cudaGraphExec_t step_exec = nullptr;
+    struct StepKey {
+        const void *Q = nullptr, *K = nullptr, *V = nullptr;
+        void *out = nullptr;
+        std::vector<int> lens;
+        int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1;
+        bool operator==(const StepKey &o) const
+        {
+            return Q == o.Q && K == o.K && V == o.V && out == o.out && lens == o.lens &&
+                   tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
+                   l2 == o.l2;
+        }
+    } step_key;
+    int step_graph_replays = 0;
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0;
     // per-variant launch state
@@ -368,6 +385,10 @@ int mlkv_cache_destroy(mlkv_cache_t c)
         return MLKV_OK;
     DeviceGuard guard(c->device);
     cudaDeviceSynchronize();
+    if (c->step_exec)
+        cudaGraphExecDestroy(c->step_exec);
+    if (c->record_stream)
+        cudaStreamDestroy(c->record_stream);
     free_all(c);
     delete c;
     return MLKV_OK;
@@ -565,6 +586,106 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
     return decode_impl(c, layer, nullptr, nullptr, Q, out, seq_lens, cuda_stream);
 }
 
+// The layer calls of one decode step, issued on `stream`.
+static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
+                      const int *seq_lens, void *stream)
+{
+    const size_t qo = static_cast<size_t>(c->b) * c->h * c->d * 2;   // bytes of one layer's Q
+    const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
+    for (int n = 0; n < c->l; ++n) {
+        int rc;
+        if (c->owner[n] == n)
+            rc = decode_impl(c, n, K + kv * c->slot[n], V + kv * c->slot[n], Q + qo * n,
+                             out + qo * n, seq_lens, stream);
+        else
+            rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream);
+        if (rc != MLKV_OK)
+            return rc;
+    }
+    return MLKV_OK;
+}
+
+int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
+                     const int *seq_lens, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (Q == nullptr || K == nullptr || V == nullptr || out == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "Q, K, V and out must be non-NULL");
+    int rc = check_seq_lens(c, seq_lens);
+    if (rc != MLKV_OK)
+        return rc;
+    DeviceGuard guard(c->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(stream, &cap);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "cudaStreamIsCapturing");
+    const char *q = static_cast<const char *>(Q);
+    const char *k = static_cast<const char *>(K);
+    const char *v = static_cast<const char *>(V);
+    char *o = static_cast<char *>(out);
+    if (!c->step_graph || cap != cudaStreamCaptureStatusNone)
+        return issue_step(c, q, k, v, o, seq_lens, cuda_stream);   // the caller records us
+
+    mlkv_cache::StepKey key;
+    key.Q = Q;
+    key.K = K;
+    key.V = V;
+    key.out = out;
+    key.lens.assign(seq_lens, seq_lens + c->b);
+    key.tile = c->tile_tokens;
+    key.grid = c->grid;
+    key.cluster = c->cluster;
+    key.pdl = c->pdl;
+    key.l2 = c->l2_persist;
+    if (c->step_exec == nullptr || !(key == c->step_key)) {
+        // Record the step once for these arguments (on a private stream: the caller's may be the
+        // legacy default stream, which cannot be captured), then replay it on the caller's.
+        if (c->record_stream == nullptr &&
+            (e = cudaStreamCreateWithFlags(&c->record_stream, cudaStreamNonBlocking)) != cudaSuccess)
+            return fail_cuda(e, "cudaStreamCreateWithFlags");
+        e = cudaStreamBeginCapture(c->record_stream, cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess)
+            return fail_cuda(e, "cudaStreamBeginCapture");
+        rc = issue_step(c, q, k, v, o, seq_lens, c->record_stream);
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamEndCapture(c->record_stream, &graph);
+        if (rc != MLKV_OK) {
+            if (graph)
+                cudaGraphDestroy(graph);
+            return rc;
+        }
+        if (e != cudaSuccess)
+            return fail_cuda(e, "cudaStreamEndCapture");
+        bool updated = false;
+        if (c->step_exec != nullptr) {
+            cudaGraphExecUpdateResultInfo info;
+            updated = cudaGraphExecUpdate(c->step_exec, graph, &info) == cudaSuccess;
+            if (!updated) {
+                cudaGetLastError();
+                cudaGraphExecDestroy(c->step_exec);
+                c->step_exec = nullptr;
+            }
+        }
+        if (!updated) {
+            e = cudaGraphInstantiate(&c->step_exec, graph, 0);
+            if (e != cudaSuccess) {
+                cudaGraphDestroy(graph);
+                c->step_exec = nullptr;
+                return fail_cuda(e, "cudaGraphInstantiate");
+            }
+        }
+        cudaGraphDestroy(graph);
+        c->step_key = key;
+    }
+    e = cudaGraphLaunch(c->step_exec, stream);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "cudaGraphLaunch");
+    ++c->step_graph_replays;
+    return MLKV_OK;
+}
+
 int mlkv_load_prefix(mlkv_cache_t c, int layer, const void *K, const void *V, int len,
                      void *cuda_stream)
 {
@@ -676,6 +797,12 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->pdl = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "step_graph") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "step_graph must be 0 or 1");
+        c->step_graph = static_cast<int>(value);
+        return MLKV_OK;
+    }
     return fail(MLKV_ERR_INVALID_ARG, "unknown option '%s'", key);
 }
 
@@ -701,6 +828,14 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "pdl") == 0) {
         *value = c->pdl;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "step_graph") == 0) {
+        *value = c->step_graph;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "step_graph_replays") == 0) {
+        *value = c->step_graph_replays;
         return MLKV_OK;
     }
     if (std::strcmp(key, "last_grid") == 0) {

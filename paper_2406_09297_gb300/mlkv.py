@@ -26,7 +26,7 @@ MLKV_MAX_GROUP = 16
 
 EXPORTED = [
     "mlkv_cache_create", "mlkv_cache_destroy", "mlkv_append", "mlkv_decode_attention",
-    "mlkv_append_decode_attention",
+    "mlkv_append_decode_attention", "mlkv_decode_step",
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static",
@@ -51,6 +51,7 @@ def _load():
     L.mlkv_append.argtypes = [vp, ci, vp, vp, ip, vp]
     L.mlkv_decode_attention.argtypes = [vp, ci, vp, vp, ip, vp]
     L.mlkv_append_decode_attention.argtypes = [vp, ci, vp, vp, vp, vp, ip, vp]
+    L.mlkv_decode_step.argtypes = [vp, vp, vp, vp, vp, ip, vp]
     L.mlkv_load_prefix.argtypes = [vp, ci, vp, vp, ci, vp]
     L.mlkv_cache_bytes.argtypes = [vp]
     L.mlkv_cache_bytes.restype = i64
@@ -134,6 +135,12 @@ def mlkv_append_decode_attention(handle, layer, K, V, Q, out, seq_lens, stream=N
     a, p = _lens_ptr(seq_lens)
     return _check(lib.mlkv_append_decode_attention(handle, layer, _ptr(K), _ptr(V), _ptr(Q),
                                                    _ptr(out), p, _stream(stream)))
+
+
+def mlkv_decode_step(handle, Q, K, V, out, seq_lens, stream=None):
+    a, p = _lens_ptr(seq_lens)
+    return _check(lib.mlkv_decode_step(handle, _ptr(Q), _ptr(K), _ptr(V), _ptr(out), p,
+                                       _stream(stream)))
 
 
 def mlkv_load_prefix(handle, layer, K, V, length, stream=None):
@@ -235,6 +242,9 @@ class MLKVCache:
 
     def append_decode_attention(self, layer, K, V, Q, out, seq_lens, stream=None):
         return mlkv_append_decode_attention(self.handle, layer, K, V, Q, out, seq_lens, stream)
+
+    def decode_step(self, Q, K, V, out, seq_lens, stream=None):
+        return mlkv_decode_step(self.handle, Q, K, V, out, seq_lens, stream)
 
     def load_prefix(self, layer, K, V, length, stream=None):
         return mlkv_load_prefix(self.handle, layer, K, V, length, stream)

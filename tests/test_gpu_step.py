@@ -1,0 +1,126 @@
+"""mlkv_decode_step (every layer of a decode step in one call, replayed from a recorded CUDA graph)
+against the per-layer calls and the oracle."""
+import numpy as np
+import pytest
+
+import oracle
+from mlkv_synth import gen
+from tests.mlkv_cases import MAX_ABS, MEAN_ABS, errors, from_dev, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref):
+    m = len(set(owner))
+    for n in sorted(set(owner)):
+        kb = gen.gen_kv(seed, n, 0, b, g, max_seq, d)
+        vb = gen.gen_kv(seed, n, 1, b, g, max_seq, d)
+        cache.load_prefix(n, to_dev(kb), to_dev(vb), max_seq)
+        if ref is not None:
+            ref.load_prefix(n, gen.bf16_bits_to_f64(kb), gen.bf16_bits_to_f64(vb), max_seq)
+    qb = np.stack([gen.gen_q(seed, n, b, h, d) for n in range(len(owner))])
+    owners = sorted(set(owner))
+    kn = np.stack([gen.gen_bf16(seed + 1, gen.TID_K + n, range(b * g), d).reshape(b, g, d)
+                   for n in owners])
+    vn = np.stack([gen.gen_bf16(seed + 1, gen.TID_V + n, range(b * g), d).reshape(b, g, d)
+                   for n in owners])
+    return qb, kn, vn
+
+
+@pytest.mark.parametrize("owner,h,g,d,b,lens,max_seq", [
+    ([0, 0, 2, 2, 2, 5], 12, 2, 64, 5, [1, 300, 1000, 77, 640], 1024),
+    ([0, 0, 0, 0], 12, 1, 64, 64, [2048] * 64, 2048),            # cluster mode
+    ([0, 0, 2], 16, 4, 128, 3, [5000, 20, 4096], 5000),
+])
+def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    seed = 31
+    lens = np.asarray(lens, dtype=np.int32)
+    l = len(owner)
+    with mlkv.MLKVCache(l, h, d, owner, g, b, max_seq) as cache, \
+            mlkv.MLKVCache(l, h, d, owner, g, b, max_seq) as cache2:
+        ref = oracle.OracleCache(owner, h, g, d, b, max_seq)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref)
+        _inputs(owner, h, g, d, b, lens, max_seq, seed, cache2, None)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        out = torch.full((l, b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        for rep in range(3):   # record, then replay twice
+            out.fill_(float("nan"))
+            cache.decode_step(Q, K, V, out, lens)
+        torch.cuda.synchronize()
+        assert cache.get_option("step_graph_replays") == 3
+        # the same layer calls one by one on a second cache
+        owners = sorted(set(owner))
+        out2 = torch.full_like(out, float("nan"))
+        for n in range(l):
+            if owner[n] == n:
+                s = owners.index(n)
+                cache2.append_decode_attention(n, K[s], V[s], Q[n], out2[n], lens)
+            else:
+                cache2.decode_attention(n, Q[n], out2[n], lens)
+        torch.cuda.synchronize()
+        assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
+        for n in range(l):
+            if owner[n] == n:
+                s = owners.index(n)
+                ref.append(n, gen.bf16_bits_to_f64(kn[s]), gen.bf16_bits_to_f64(vn[s]), lens)
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens)
+            mx, mean = errors(from_dev(out[n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
+        cache2.sync_status()
+
+
+def test_step_rerecords_on_new_lengths_and_buffers():
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, g, d, b, max_seq = [0, 0, 2, 2], 8, 2, 64, 4, 700
+    with mlkv.MLKVCache(4, h, d, owner, g, b, max_seq) as cache:
+        qb, kn, vn = _inputs(owner, h, g, d, b, None, max_seq, 41, cache, None)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        outs = []
+        for lens in ([300, 1, 700, 64], [301, 2, 700, 65], [301, 2, 700, 65]):
+            lens = np.asarray(lens, dtype=np.int32)
+            out = torch.empty((4, b, h, d), dtype=torch.bfloat16, device="cuda")
+            cache.decode_step(Q, K, V, out, lens)
+            outs.append((lens, out))
+        torch.cuda.synchronize()
+        with mlkv.MLKVCache(4, h, d, owner, g, b, max_seq) as check:
+            _inputs(owner, h, g, d, b, None, max_seq, 41, check, None)
+            check.set_option("step_graph", 0)
+            for lens, out in outs:
+                ref = torch.empty_like(out)
+                check.decode_step(Q, K, V, ref, lens)
+                torch.cuda.synchronize()
+                assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
+
+
+def test_step_inside_a_caller_graph():
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, g, d, b, max_seq = [0, 0], 12, 1, 64, 8, 512
+    lens = np.full(b, 512, dtype=np.int32)
+    with mlkv.MLKVCache(2, h, d, owner, g, b, max_seq) as cache:
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, max_seq, 51, cache, None)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        out = torch.empty((2, b, h, d), dtype=torch.bfloat16, device="cuda")
+        ref = torch.empty_like(out)
+        cache.set_option("step_graph", 0)
+        cache.decode_step(Q, K, V, ref, lens)
+        cache.set_option("step_graph", 1)
+        graph = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            cache.decode_step(Q, K, V, out, lens)
+        torch.cuda.current_stream().wait_stream(s)
+        with torch.cuda.graph(graph):
+            cache.decode_step(Q, K, V, out, lens)
+        out.zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
