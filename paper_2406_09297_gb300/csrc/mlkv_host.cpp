@@ -426,7 +426,8 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
 }
 
 static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
-                       const void *Q, void *out, const int *seq_lens, void *cuda_stream)
+                       const void *Q, void *out, const int *seq_lens, void *cuda_stream,
+                       int early_fetch = 0)
 {
     if (c == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
@@ -530,6 +531,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     p.cluster_k = cluster_k;
     p.tile_tokens = T;
     p.decode_grid = grid;
+    p.early_fetch = early_fetch;
     // Segments split over many CTAs are merged by a separate parallel kernel: one warp merging
     // dozens of partials would serialise on its loads.
     p.deferred_merge = (cluster_k <= 1 &&
@@ -594,11 +596,14 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
     const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
     for (int n = 0; n < c->l; ++n) {
         int rc;
+        // Layers after the first follow this library's own launch of the preceding layer.
+        const int early = (n > 0 && c->pdl) ? 1 : 0;
         if (c->owner[n] == n)
             rc = decode_impl(c, n, K + kv * c->slot[n], V + kv * c->slot[n], Q + qo * n,
-                             out + qo * n, seq_lens, stream);
+                             out + qo * n, seq_lens, stream, early);
         else
-            rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream);
+            rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream,
+                             early);
         if (rc != MLKV_OK)
             return rc;
     }

@@ -39,6 +39,8 @@ struct DecodeParams {
     int deferred_merge;       // 1: split segments only write partials; combine_kernel merges them
     int tile_tokens;          // T of the launch (the combine kernel re-derives the piece layout)
     int decode_grid;          // P of the decode launch
+    int early_fetch;          // 1: the previous kernel is this library's decode of the preceding
+                              // layer; tiles without a segment's newest row may be fetched first
     int seq_len[MLKV_MAX_BATCH];
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };

@@ -615,18 +615,46 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     TileWalk<T> wk;
     if (tile_lo < tile_hi)
         wk.init(p, s_len, s_start, tile_lo);
-    // Everything above overlaps the previous kernel's tail; global memory is touched only below.
-    grid_dependency_wait();
-    if (warp != PL::kProducer)
+    // Everything above overlaps the previous kernel's tail; global memory is touched only below
+    // (the producer may first fetch tiles the previous kernel cannot have written; see there).
+    if (warp != PL::kProducer) {
+        grid_dependency_wait();
         grid_dependents_launch();
+    }
 
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
-        if (lane != 0)
+        if (lane != 0) {
+            grid_dependency_wait();
             grid_dependents_launch();
+        }
         if (lane == 0) {
         int issued = 0;
-        for (int tile = tile_lo; tile < tile_hi; ++tile) {
+        int tile = tile_lo;
+        // Early fetch: when the previous kernel of the stream is this library's decode of the
+        // preceding layer (mlkv_decode_step), the only cache data it writes is the new token's
+        // row, which lies in the last tile of a segment.  Tiles before that are fetched before
+        // waiting for it to finish.
+        if (p.early_fetch) {
+            while (tile < tile_hi && issued < STAGES && wk.tt != wk.nt - 1) {
+                const uint32_t fb = bar_full + 8 * issued;
+                mbar_arrive_expect_tx(fb, PL::kStageBytes);
+                const int zk = ((p.slot * 2 + 0) * p.b + wk.beta) * p.g + wk.j;
+                const int zv = zk + p.b * p.g;
+                const uint32_t kdst = sbase + issued * PL::kStageBytes;
+#pragma unroll
+                for (int sub = 0; sub < PL::kSub; ++sub) {
+                    tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, wk.tt * T, zk);
+                    tma_load_3d(kdst + PL::kTileBytes + sub * T * 128, &tmap, fb, sub * 64,
+                                wk.tt * T, zv);
+                }
+                ++issued;
+                ++tile;
+                wk.next(p, s_len, s_start);
+            }
+        }
+        grid_dependency_wait();
+        for (; tile < tile_hi; ++tile) {
             const int s = issued % STAGES;
             if (issued >= STAGES && !flags[0] &&
                 !mbar_wait(bar_empty + 8 * s, ((issued / STAGES) & 1) ^ 1)) {

@@ -232,6 +232,7 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.cluster_k = 0;
     p.tile_tokens = T;
     p.decode_grid = grid;
+    p.early_fetch = 0;
     p.deferred_merge =
         mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces ? 1 : 0;
     const size_t smem = v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(batch));
