@@ -427,7 +427,7 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
 
 static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
                        const void *Q, void *out, const int *seq_lens, void *cuda_stream,
-                       int early_fetch = 0)
+                       int early_fetch = 0, const void *Q_next = nullptr)
 {
     if (c == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
@@ -532,6 +532,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.early_fetch = early_fetch;
+    p.Q_next = static_cast<const __nv_bfloat16 *>(Q_next);
     // Segments split over many CTAs are merged by a separate parallel kernel: one warp merging
     // dozens of partials would serialise on its loads.
     p.deferred_merge = (cluster_k <= 1 &&
@@ -598,12 +599,13 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         int rc;
         // Layers after the first follow this library's own launch of the preceding layer.
         const int early = (n > 0 && c->pdl) ? 1 : 0;
+        const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
         if (c->owner[n] == n)
             rc = decode_impl(c, n, K + kv * c->slot[n], V + kv * c->slot[n], Q + qo * n,
-                             out + qo * n, seq_lens, stream, early);
+                             out + qo * n, seq_lens, stream, early, q_next);
         else
             rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream,
-                             early);
+                             early, q_next);
         if (rc != MLKV_OK)
             return rc;
     }

@@ -39,8 +39,11 @@ struct DecodeParams {
     int deferred_merge;       // 1: split segments only write partials; combine_kernel merges them
     int tile_tokens;          // T of the launch (the combine kernel re-derives the piece layout)
     int decode_grid;          // P of the decode launch
+    const __nv_bfloat16 *Q_next;   // the next layer's queries (decode step), prefetched to L2
     int early_fetch;          // 1: the previous kernel is this library's decode of the preceding
-                              // layer; tiles without a segment's newest row may be fetched first
+                              // layer, which writes neither Q nor any cache row but a segment's
+                              // newest: Q and the tiles without that row are read before the
+                              // dependency wait
     int seq_len[MLKV_MAX_BATCH];
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };

@@ -187,6 +187,12 @@ __device__ __forceinline__ void consumer_bar_sync()
 
 // Programmatic dependent launch: wait until the previous kernel of the stream has completed and
 // its memory is visible; allow the next kernel of the stream to start its prologue.
+// Bulk prefetch of [src, src + bytes) into L2 (src 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void grid_dependency_wait()
 {
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -308,12 +314,15 @@ struct Plan {
     // slots for the other ranks' results ([k-1][kResBytes]).
     static constexpr int kTables = kBars + (2 * STAGES + 5) * 8 + 8;
     static constexpr int kBytes = kTables;
+    static constexpr int kFinRow = D + 8;             // row stride (f32) of the last piece's sums
     static constexpr int kAlloc = kBytes + 1024;      // base aligned up to 1024 in the kernel
     static_assert(kTW % 16 == 0, "each warp takes whole 16-position mma steps");
     static_assert(NCW == 4 || NCW == 8, "tree merge over 4 or 8 warps");
     static_assert(D == 64 || D == 128, "head_dim 64 or 128");
     static_assert(T <= 256, "TMA box height");
     static_assert(kResBytes % 16 == 0, "result slots stay 16-byte aligned");
+    static_assert((NCW * 16 * kFinRow + 16) * 4 <= STAGES * kStageBytes,
+                  "the last piece's per-warp sums fit in the stage ring");
 };
 
 // Byte offset of 16-byte chunk `chunk` (0 .. D/8-1) of row `row` inside a K or V tile laid out by
@@ -335,9 +344,11 @@ __device__ __forceinline__ uint32_t cluster_ctarank()
 
 // Every thread of a cluster launch arrives once, right after set-up, and waits once, late: before
 // its first access to another CTA's shared memory and before it exits.
+// Relaxed: what the partners need from this arrival are the barrier initialisations, which
+// fence.mbarrier_init.release.cluster has already published.
 __device__ __forceinline__ void cluster_arrive()
 {
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ void cluster_wait()
@@ -544,6 +555,27 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
         p.counters[seg] = 0u;
 }
 
+// Query fragments of one (sequence, KV head) group: the A operand of S = Q K^T in the
+// mma.m16n8k16 layout, rows >= G (the padding of the group to 16 rows) zero.
+template <int D>
+__device__ __forceinline__ void load_q_frag(uint32_t (&qa)[D / 16][4], const DecodeParams &p,
+                                            int beta, int j, int lane)
+{
+    const int G = p.G;
+    const int qr = lane >> 2, qc = (lane & 3) * 2;
+    const __nv_bfloat16 *qb =
+        p.Q + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+    const bool r0 = qr < G, r1 = qr + 8 < G;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        const int c = ks * 16 + qc;
+        qa[ks][0] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c) : 0u;
+        qa[ks][1] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c) : 0u;
+        qa[ks][2] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c + 8) : 0u;
+        qa[ks][3] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c + 8) : 0u;
+    }
+}
+
 // ------------------------------------------------------------------------------------------------
 // decode kernel
 // ------------------------------------------------------------------------------------------------
@@ -615,46 +647,54 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     TileWalk<T> wk;
     if (tile_lo < tile_hi)
         wk.init(p, s_len, s_start, tile_lo);
-    // Everything above overlaps the previous kernel's tail; global memory is touched only below
-    // (the producer may first fetch tiles the previous kernel cannot have written; see there).
+    // Everything above overlaps the previous kernel's tail.  Normally global memory is touched only
+    // after the dependency wait.  When the previous kernel is this library's decode of the
+    // preceding layer (p.early_fetch, inside mlkv_decode_step), that kernel writes nothing this one
+    // reads except the newest row (position L-1) of the slot it appended to, which lies in the
+    // last tile of a segment, and the merge scratch (partials, counters).  So the queries and
+    // every other tile are read at once; the producer waits before it fetches a segment's last
+    // tile, the epilogue warp before it writes its first record, and the consumers before they
+    // write the last piece (scratch) or, at the latest, before they exit -- so this grid finishes
+    // only after the previous one, as the next layer's wait expects.  The fused append writes
+    // the newest row of this layer's own slot, which no earlier layer reads.
+    const bool early = p.early_fetch != 0;
+    uint32_t qa[KS][4];
+    const bool q_early = early && warp < NCW && tile_lo < tile_hi;
+    if (q_early)
+        load_q_frag<D>(qa, p, wk.beta, wk.j, lane);
     if (warp != PL::kProducer) {
-        grid_dependency_wait();
+        if (!early)
+            grid_dependency_wait();
         grid_dependents_launch();
     }
 
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
-        if (lane != 0) {
-            grid_dependency_wait();
-            grid_dependents_launch();
-        }
+        if (lane != 0)
+            grid_dependents_launch();   // only lane 0 touches global memory
         if (lane == 0) {
         int issued = 0;
         int tile = tile_lo;
-        // Early fetch: when the previous kernel of the stream is this library's decode of the
-        // preceding layer (mlkv_decode_step), the only cache data it writes is the new token's
-        // row, which lies in the last tile of a segment.  Tiles before that are fetched before
-        // waiting for it to finish.
-        if (p.early_fetch) {
-            while (tile < tile_hi && issued < STAGES && wk.tt != wk.nt - 1) {
-                const uint32_t fb = bar_full + 8 * issued;
-                mbar_arrive_expect_tx(fb, PL::kStageBytes);
-                const int zk = ((p.slot * 2 + 0) * p.b + wk.beta) * p.g + wk.j;
-                const int zv = zk + p.b * p.g;
-                const uint32_t kdst = sbase + issued * PL::kStageBytes;
-#pragma unroll
-                for (int sub = 0; sub < PL::kSub; ++sub) {
-                    tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, wk.tt * T, zk);
-                    tma_load_3d(kdst + PL::kTileBytes + sub * T * 128, &tmap, fb, sub * 64,
-                                wk.tt * T, zv);
-                }
-                ++issued;
-                ++tile;
-                wk.next(p, s_len, s_start);
-            }
+        bool waited = !early;
+        if (!early)
+            grid_dependency_wait();
+        // The next layer's queries (an input of the whole step) go to L2 now: its CTAs load
+        // them first thing, while this layer still streams.  Each CTA takes a 128-byte-aligned
+        // share.
+        if (p.Q_next != nullptr) {
+            const size_t qbytes = static_cast<size_t>(p.b) * p.h * D * 2;   // a multiple of 128
+            const size_t lo = (qbytes * cta / P) & ~static_cast<size_t>(127);
+            const size_t hi =
+                cta + 1 == P ? qbytes : (qbytes * (cta + 1) / P) & ~static_cast<size_t>(127);
+            if (hi > lo)
+                bulk_prefetch_l2(reinterpret_cast<const uint8_t *>(p.Q_next) + lo,
+                                 static_cast<uint32_t>(hi - lo));
         }
-        grid_dependency_wait();
         for (; tile < tile_hi; ++tile) {
+            if (!waited && wk.tt == wk.nt - 1) {
+                grid_dependency_wait();   // this tile holds the newest row
+                waited = true;
+            }
             const int s = issued % STAGES;
             if (issued >= STAGES && !flags[0] &&
                 !mbar_wait(bar_empty + 8 * s, ((issued / STAGES) & 1) ^ 1)) {
@@ -712,6 +752,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             const int *meta = reinterpret_cast<const int *>(slot + PL::kResO + 64);
             if (meta[kMetaStop])
                 break;
+            if (early && k == 0)
+                grid_dependency_wait();   // records and merges use the shared scratch
             if (!flags[0])
                 epilogue_piece<D>(p, reinterpret_cast<const float *>(slot),
                                   reinterpret_cast<const float *>(slot + PL::kResO), meta, s_w,
@@ -750,22 +792,9 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         const int piece_first = tile;
         const int piece_end = seg_end < tile_hi ? seg_end : tile_hi;
 
-        // Query fragments of the group's heads (rows >= G are zero): A operand of S = Q K^T.
-        uint32_t qa[KS][4];
-        {
-            const __nv_bfloat16 *qb =
-                p.Q + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
-            const bool r0 = qr < G, r1 = qr + 8 < G;
-#pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                const int c = ks * 16 + qc;
-                qa[ks][0] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c) : 0u;
-                qa[ks][1] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c) : 0u;
-                qa[ks][2] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * D + c + 8) : 0u;
-                qa[ks][3] =
-                    r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * D + c + 8) : 0u;
-            }
-        }
+        // The first piece's query fragments may already be loaded (before the dependency wait).
+        if (!(q_early && tile == tile_lo))
+            load_q_frag<D>(qa, p, beta, j, lane);
 
         float o[NO][4];
 #pragma unroll
@@ -934,30 +963,30 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         }
         // The barrier also guarantees that every warp is done with the ring's tiles.
         consumer_bar_sync<NCW>();
-        float lse[2];
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            const int row = qr + 8 * hr;
-            // every piece holds at least one visible position, so mstar is finite
-            float mstar = NEG_INF;
-#pragma unroll
-            for (int w = 0; w < NCW; ++w)
-                mstar = fmaxf(mstar, red_m[w * 16 + row]);
-            float lsum = 0.f;
-#pragma unroll
-            for (int w = 0; w < NCW; ++w)
-                lsum += red_l[w * 16 + row] * fast_exp2(red_m[w * 16 + row] - mstar);
-            const float f = fast_exp2(m_run[hr] - mstar) * fast_rcp(lsum);
-            lse[hr] = mstar + fast_log2(lsum);
-#pragma unroll
-            for (int n = 0; n < NO; ++n) {
-                o[n][2 * hr] *= f;
-                o[n][2 * hr + 1] *= f;
-            }
-        }
         if (piece_end != tile_hi) {
             // A piece before the CTA's last: tree over warps, result to the epilogue warp, and
             // the consumers go straight on to the next piece.
+            float lse[2];
+    #pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                const int row = qr + 8 * hr;
+                // every piece holds at least one visible position, so mstar is finite
+                float mstar = NEG_INF;
+    #pragma unroll
+                for (int w = 0; w < NCW; ++w)
+                    mstar = fmaxf(mstar, red_m[w * 16 + row]);
+                float lsum = 0.f;
+    #pragma unroll
+                for (int w = 0; w < NCW; ++w)
+                    lsum += red_l[w * 16 + row] * fast_exp2(red_m[w * 16 + row] - mstar);
+                const float f = fast_exp2(m_run[hr] - mstar) * fast_rcp(lsum);
+                lse[hr] = mstar + fast_log2(lsum);
+    #pragma unroll
+                for (int n = 0; n < NO; ++n) {
+                    o[n][2 * hr] *= f;
+                    o[n][2 * hr + 1] *= f;
+                }
+            }
             // Tree over warps with NCW/2 slots.  First level: warp w in [NCW/2, NCW) writes slot
             // w - NCW/2 and warp r < NCW/2 adds slot r.  Later levels (half < NCW/2): warp w in
             // [half, 2 half) writes slot w and warp r < half adds slot r + half.  Every slot is
@@ -1025,20 +1054,23 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             ++nhand;
         } else {
             // ---- the CTA's last piece: every tile has been consumed and no copy is pending, so
-            // the stage ring is free.  The warps write their weighted accumulators there (one
-            // barrier) and every consumer thread sums and finishes its share of the outputs.
-            float *fbuf = reinterpret_cast<float *>(smem);         // [NCW][16][D] f32
-            float *flse = fbuf + NCW * 16 * D;                      // [16]
+            // the stage ring is free.  Each warp stores its raw accumulators there; after one
+            // barrier each consumer warp finishes one row per pass from every warp's statistics
+            // of the row: m* = max_w m_w, l* = sum_w l_w 2^(m_w - m*), o = sum_w 2^(m_w - m*) o_w
+            // / l*, lse = m* + log2 l*.
+            // Rows padded to D + 8 floats: the fragment stores of a warp's 8 rows then fall in
+            // distinct banks.
+            constexpr int FS = PL::kFinRow;
+            float *fbuf = reinterpret_cast<float *>(smem);         // [NCW][16][FS] f32
+            float *flse = fbuf + NCW * 16 * FS;                     // [16]
 #pragma unroll
             for (int hr = 0; hr < 2; ++hr) {
                 const int row = qr + 8 * hr;
                 if (row < G) {
 #pragma unroll
                     for (int n = 0; n < NO; ++n)
-                        *reinterpret_cast<float2 *>(fbuf + (warp * 16 + row) * D + n * 8 + qc) =
+                        *reinterpret_cast<float2 *>(fbuf + (warp * 16 + row) * FS + n * 8 + qc) =
                             make_float2(o[n][2 * hr], o[n][2 * hr + 1]);
-                    if (warp == 0 && qc == 0)
-                        flse[row] = lse[hr];
                 }
             }
             if (p.cluster_k > 1)
@@ -1049,9 +1081,12 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             __nv_bfloat16 *ob =
                 p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
             constexpr int kPairs = NCW * 32;   // float2 outputs per pass
+            static_assert(D == 2 * 32 || D == 4 * 32, "a warp's pass covers 64 elements of one row");
             // mode: 0 whole, 1 cluster sender, 2 cluster leader, 3 partial record
             const int rank = p.cluster_k > 1 ? static_cast<int>(cluster_ctarank()) : 0;
             const int mode = whole ? 0 : (p.cluster_k > 1 ? (rank != 0 ? 1 : 2) : 3);
+            if (early && mode == 3)
+                grid_dependency_wait();   // partial records and counters are shared scratch
             const uint32_t cslots = sbase + PL::kTables;
             const uint8_t *cs = smem + PL::kTables;
             uint32_t remote = 0, remote_bar = 0;
@@ -1059,111 +1094,145 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 remote = map_to_rank(cslots + (rank - 1) * PL::kResBytes, 0);
                 remote_bar = map_to_rank(bar_cluster, 0);
             }
-            if (mode == 2) {
-                if (ctid == 0 && !flags[0] && !mbar_wait_cluster(bar_cluster, 0)) {
-                    flags[0] = 1;
-                    atomicOr(p.err, kErrWaitFull);
-                }
-                consumer_bar_sync<NCW>();
-            }
             const size_t piece = static_cast<size_t>(seg + cta);
             float *po = p.part_o + piece * G * D;
-#pragma unroll 1
+#pragma unroll 2
             for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
-                const int row = i / D, e = i - row * D;
-                const float lse_row = flse[row];
+                const int row = i / D, e = i - row * D;   // row is the same across the warp
+                // independent broadcast loads of the row's statistics of every warp
+                float mw[NCW], lw[NCW];
+#pragma unroll
+                for (int w = 0; w < NCW; ++w) {
+                    mw[w] = red_m[w * 16 + row];
+                    lw[w] = red_l[w * 16 + row];
+                }
+                float ms = mw[0];   // finite: the piece holds a visible position
+#pragma unroll
+                for (int w = 1; w < NCW; ++w)
+                    ms = fmaxf(ms, mw[w]);
+                float ls = 0.f;
                 float2 v = make_float2(0.f, 0.f);
 #pragma unroll
                 for (int w = 0; w < NCW; ++w) {
-                    const float2 x = *reinterpret_cast<const float2 *>(fbuf + (w * 16 + row) * D + e);
-                    v.x += x.x;
-                    v.y += x.y;
+                    const float ew = fast_exp2(mw[w] - ms);
+                    ls = fmaf(lw[w], ew, ls);
+                    const float2 x =
+                        *reinterpret_cast<const float2 *>(fbuf + (w * 16 + row) * FS + e);
+                    v.x = fmaf(ew, x.x, v.x);
+                    v.y = fmaf(ew, x.y, v.y);
                 }
+                const float inv = fast_rcp(ls);
+                v.x *= inv;
+                v.y *= inv;
+                const float lse_row = ms + fast_log2(ls);
+                const bool row_head = (e == 0 && lane == 0);   // one lane per row
                 if (mode == 0) {
                     *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(v.x, v.y);
                 } else if (mode == 1) {
+                    // the leader's barrier completes when all these bytes have landed
                     st_async_v2(remote + i * 4, v.x, v.y, remote_bar);
+                    if (row_head)
+                        st_async_f32(remote + PL::kResO + row * 4, lse_row, remote_bar);
                 } else if (mode == 2) {
-                    if (!flags[0]) {
-                        float mx = lse_row;
-                        for (int r = 1; r < p.cluster_k; ++r)
-                            mx = fmaxf(mx, reinterpret_cast<const float *>(
-                                               cs + (r - 1) * PL::kResBytes + PL::kResO)[row]);
-                        float w = fast_exp2(lse_row - mx);
-                        float tot = w, ax = w * v.x, ay = w * v.y;
-                        for (int r = 1; r < p.cluster_k; ++r) {
-                            const float *sl =
-                                reinterpret_cast<const float *>(cs + (r - 1) * PL::kResBytes);
-                            w = fast_exp2(sl[PL::kResO / 4 + row] - mx);
+                    // each element is read and rewritten by this thread alone
+                    *reinterpret_cast<float2 *>(fbuf + row * FS + e) = v;
+                    if (row_head)
+                        flse[row] = lse_row;
+                } else {
+                    *reinterpret_cast<float2 *>(po + i) = v;
+                    if (row_head)
+                        p.part_lse[piece * G + row] = lse_row;
+                }
+            }
+            if (mode == 2) {
+                // Leader: its own result is in warp 0's rows; merge the other ranks' once landed.
+                if (!flags[0] && !mbar_wait_cluster(bar_cluster, 0)) {
+                    flags[0] = 1;
+                    atomicOr(p.err, kErrWaitFull);
+                }
+                consumer_bar_sync<NCW>();   // flse is complete
+                const int k = p.cluster_k;   // 2 or 4
+#pragma unroll 2
+                for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
+                    const int row = i / D, e = i - row * D;
+                    float lr[4];
+                    float2 x[4];
+                    lr[0] = flse[row];
+                    x[0] = *reinterpret_cast<const float2 *>(fbuf + row * FS + e);
+#pragma unroll
+                    for (int r = 1; r < 4; ++r) {
+                        lr[r] = NEG_INF;
+                        x[r] = make_float2(0.f, 0.f);
+                        if (r < k) {
+                            const uint8_t *sl = cs + (r - 1) * PL::kResBytes;
+                            lr[r] = reinterpret_cast<const float *>(sl + PL::kResO)[row];
+                            x[r] = *reinterpret_cast<const float2 *>(sl + static_cast<size_t>(i) * 4);
+                        }
+                    }
+                    const float mx = fmaxf(fmaxf(lr[0], lr[1]), fmaxf(lr[2], lr[3]));
+                    float tot = 0.f, ax = 0.f, ay = 0.f;
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const float w = fast_exp2(lr[r] - mx);   // 0 past k
+                        tot += w;
+                        ax = fmaf(w, x[r].x, ax);
+                        ay = fmaf(w, x[r].y, ay);
+                    }
+                    const float inv = fast_rcp(tot);
+                    if (!flags[0])
+                        *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(ax * inv, ay * inv);
+                }
+            } else if (mode == 3 && !p.deferred_merge) {
+                const int c_first = cta_of_tile(seg_first, N, P);
+                const int c_last = cta_of_tile(seg_end - 1, N, P);
+                __threadfence();
+                consumer_bar_sync<NCW>();
+                if (ctid == 0) {
+                    const unsigned prev = atomic_add_acq_rel_gpu(&p.counters[seg], 1u);
+                    flags[1] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
+                }
+                consumer_bar_sync<NCW>();
+                if (flags[1]) {
+                    // Last finisher of the segment: merge its <= 4 records (own included).
+                    const int np = c_last - c_first + 1;
+                    const size_t rec0 = static_cast<size_t>(seg + c_first);
+#pragma unroll 1
+                    for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
+                        const int row = i / D;
+                        float lv[kInlineMergeMaxPieces];
+                        float2 ov[kInlineMergeMaxPieces];
+                        float mx = NEG_INF;
+#pragma unroll
+                        for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
+                            lv[k] = NEG_INF;
+                            ov[k] = make_float2(0.f, 0.f);
+                            if (k < np) {
+                                lv[k] = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
+                                ov[k] = __ldcg(reinterpret_cast<const float2 *>(
+                                    p.part_o + (rec0 + k) * G * D + i));
+                            }
+                            mx = fmaxf(mx, lv[k]);
+                        }
+                        float tot = 0.f, ax = 0.f, ay = 0.f;
+#pragma unroll
+                        for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
+                            const float w = fast_exp2(lv[k] - mx);   // 0 past np
                             tot += w;
-                            const float2 x = *reinterpret_cast<const float2 *>(sl + i);
-                            ax += w * x.x;
-                            ay += w * x.y;
+                            ax += w * ov[k].x;
+                            ay += w * ov[k].y;
                         }
                         const float inv = fast_rcp(tot);
                         *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(ax * inv, ay * inv);
                     }
-                } else {
-                    *reinterpret_cast<float2 *>(po + i) = v;
+                    if (ctid == 0)
+                        p.counters[seg] = 0u;
                 }
-            }
-            if (mode == 1) {
-                // the leader's barrier completes when all these bytes have landed
-                if (ctid < G)
-                    st_async_f32(remote + PL::kResO + ctid * 4, flse[ctid], remote_bar);
-            } else if (mode == 3) {
-                if (ctid < G)
-                    p.part_lse[piece * G + ctid] = flse[ctid];
-                if (!p.deferred_merge) {
-                    const int c_first = cta_of_tile(seg_first, N, P);
-                    const int c_last = cta_of_tile(seg_end - 1, N, P);
-                    __threadfence();
-                    consumer_bar_sync<NCW>();
-                    if (ctid == 0) {
-                        const unsigned prev = atomic_add_acq_rel_gpu(&p.counters[seg], 1u);
-                        flags[1] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
-                    }
-                    consumer_bar_sync<NCW>();
-                    if (flags[1]) {
-                        // Last finisher of the segment: merge its <= 4 records (own included).
-                        const int np = c_last - c_first + 1;
-                        const size_t rec0 = static_cast<size_t>(seg + c_first);
-#pragma unroll 1
-                        for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
-                            const int row = i / D;
-                            float lv[kInlineMergeMaxPieces];
-                            float2 ov[kInlineMergeMaxPieces];
-                            float mx = NEG_INF;
-#pragma unroll
-                            for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
-                                lv[k] = NEG_INF;
-                                ov[k] = make_float2(0.f, 0.f);
-                                if (k < np) {
-                                    lv[k] = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
-                                    ov[k] = __ldcg(reinterpret_cast<const float2 *>(
-                                        p.part_o + (rec0 + k) * G * D + i));
-                                }
-                                mx = fmaxf(mx, lv[k]);
-                            }
-                            float tot = 0.f, ax = 0.f, ay = 0.f;
-#pragma unroll
-                            for (int k = 0; k < kInlineMergeMaxPieces; ++k) {
-                                const float w = fast_exp2(lv[k] - mx);   // 0 past np
-                                tot += w;
-                                ax += w * ov[k].x;
-                                ay += w * ov[k].y;
-                            }
-                            const float inv = fast_rcp(tot);
-                            *reinterpret_cast<uint32_t *>(ob + i) = pack_bf16x2(ax * inv, ay * inv);
-                        }
-                        if (ctid == 0)
-                            p.counters[seg] = 0u;
-                    }
-                    consumer_bar_sync<NCW>();   // flags[1] is reused
-                }
+                consumer_bar_sync<NCW>();   // flags[1] is reused
             }
         }
     }
+    if (early)
+        grid_dependency_wait();   // no-op if already waited; this grid ends after the previous
     // Tell the epilogue warp that no piece follows.
     if (warp == 0) {
         const int rb = nhand & 1;
@@ -1319,7 +1388,7 @@ constexpr DecodeVariant make_variant()
 // (head_dim, tile) pair is used.
 const DecodeVariant kVariants[] = {
     make_variant<64, 128, 6, 8>(),
-    make_variant<64, 256, 3, 8>(),
+    make_variant<64, 256, 3, 4>(),
     make_variant<64, 64, 4, 4>(),
     make_variant<128, 64, 5, 4>(),
     make_variant<128, 128, 2, 4>(),

@@ -233,6 +233,7 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.early_fetch = 0;
+    p.Q_next = nullptr;
     p.deferred_merge =
         mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces ? 1 : 0;
     const size_t smem = v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(batch));
