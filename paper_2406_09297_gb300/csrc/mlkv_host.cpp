@@ -137,7 +137,8 @@ struct mlkv_cache {
     // per-variant launch state
     struct Variant {
         const mlkv::DecodeVariant *v = nullptr;
-        CUtensorMap tmap;
+        CUtensorMap tmap;        // boxes of tile_tokens positions
+        CUtensorMap tmap_rows;   // boxes of 64 positions (a partly visible last tile)
         int ctas_per_sm = 0;
         int clusters[5] = {0, 0, 0, 0, 0};   // resident k-CTA clusters, k = 2, 4
     };
@@ -179,7 +180,7 @@ mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0)
     return nullptr;
 }
 
-int encode_tmap(mlkv_cache *c, const mlkv::DecodeVariant *v, CUtensorMap *out)
+int encode_tmap(mlkv_cache *c, int rows, CUtensorMap *out)
 {
     static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
     if (encode == nullptr)
@@ -188,7 +189,7 @@ int encode_tmap(mlkv_cache *c, const mlkv::DecodeVariant *v, CUtensorMap *out)
                                 static_cast<cuuint64_t>(c->m) * 2 * c->b * c->g};
     const cuuint64_t strides[2] = {static_cast<cuuint64_t>(c->d) * 2,
                                    static_cast<cuuint64_t>(c->max_seq) * c->d * 2};
-    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(v->tile_tokens), 1u};
+    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(rows), 1u};
     const cuuint32_t estr[3] = {1u, 1u, 1u};
     CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, c->cache, dims, strides, box,
                         estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -367,7 +368,9 @@ int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_d
         return fail_cuda(e, "initialising the cache");
     }
     for (auto &var : c->variants) {
-        rc = encode_tmap(c, var.v, &var.tmap);
+        rc = encode_tmap(c, var.v->tile_tokens, &var.tmap);
+        if (rc == MLKV_OK)
+            rc = encode_tmap(c, 64, &var.tmap_rows);
         if (rc != MLKV_OK) {
             free_all(c);
             delete c;
@@ -556,7 +559,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                         (cluster_k > 1 ? (cluster_k - 1) * var->v->res_bytes
                                        : (uniform ? 0 : mlkv::table_bytes(c->b)));
     cudaError_t e = mlkv::launch_decode(*var->v, grid, smem, static_cast<cudaStream_t>(cuda_stream),
-                                        &var->tmap, p, winp, c->pdl != 0);
+                                        &var->tmap, &var->tmap_rows, p, winp, c->pdl != 0);
     if (e != cudaSuccess)
         return fail_cuda(e, "decode launch");
     if (p.deferred_merge) {

@@ -79,9 +79,12 @@ cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem);
 
 // pdl: launch with programmatic stream serialization (the kernel's prologue may overlap the
 // previous kernel of the stream; it waits on griddepcontrol.wait before touching global memory).
+// tmap: the cache with boxes of {64 channels, tile_tokens positions}; tmap_rows: the same tensor
+// with boxes of 64 positions, used for a segment's last tile when it is only partly visible.
 cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
-                          const CUtensorMap *tmap, const DecodeParams &p,
-                          const cudaAccessPolicyWindow *window, bool pdl = true);
+                          const CUtensorMap *tmap, const CUtensorMap *tmap_rows,
+                          const DecodeParams &p, const cudaAccessPolicyWindow *window,
+                          bool pdl = true);
 
 // Sets the calling thread's mlkv_last_error() text.
 void set_last_error(const char *msg);

@@ -126,6 +126,17 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// Plain bulk copy global -> this CTA's shared memory, completing `bytes` on the mbarrier (both
+// addresses 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes,
+                                          uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map)
 {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -312,7 +323,12 @@ struct Plan {
     static constexpr int kBars = kFlags + 16;
     // Dynamic tail: per-sequence tables (lengths differ) or, in cluster mode, the leader's
     // slots for the other ranks' results ([k-1][kResBytes]).
-    static constexpr int kTables = kBars + (2 * STAGES + 5) * 8 + 8;
+    // Per-stage query slots: the G rows of the segment whose first tile the stage holds, each row
+    // padded by 16 bytes so that the fragment loads (8 rows apart) fall in distinct banks.
+    static constexpr int kQRow = D * 2 + 16;
+    static constexpr int kQSlot = 16 * kQRow;
+    static constexpr int kQ = (kBars + (2 * STAGES + 5) * 8 + 8 + 127) / 128 * 128;
+    static constexpr int kTables = kQ + STAGES * kQSlot;
     static constexpr int kBytes = kTables;
     static constexpr int kFinRow = D + 8;             // row stride (f32) of the last piece's sums
     static constexpr int kAlloc = kBytes + 1024;      // base aligned up to 1024 in the kernel
@@ -555,8 +571,8 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
         p.counters[seg] = 0u;
 }
 
-// Query fragments of one (sequence, KV head) group: the A operand of S = Q K^T in the
-// mma.m16n8k16 layout, rows >= G (the padding of the group to 16 rows) zero.
+// Query fragments of one (sequence, KV head) group from global memory: the A operand of
+// S = Q K^T in the mma.m16n8k16 layout, rows >= G (the padding of the group to 16 rows) zero.
 template <int D>
 __device__ __forceinline__ void load_q_frag(uint32_t (&qa)[D / 16][4], const DecodeParams &p,
                                             int beta, int j, int lane)
@@ -576,6 +592,26 @@ __device__ __forceinline__ void load_q_frag(uint32_t (&qa)[D / 16][4], const Dec
     }
 }
 
+// Query fragments of one (sequence, KV head) group from its shared-memory slot (16 rows of
+// D bf16, row stride RS elements, rows >= G unused): the A operand of S = Q K^T in the
+// mma.m16n8k16 layout, rows >= G zero.
+template <int D, int RS>
+__device__ __forceinline__ void load_q_frag_smem(uint32_t (&qa)[D / 16][4], const uint8_t *slot,
+                                                 int G, int lane)
+{
+    const int qr = lane >> 2, qc = (lane & 3) * 2;
+    const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(slot);
+    const bool r0 = qr < G, r1 = qr + 8 < G;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        const int c = ks * 16 + qc;
+        qa[ks][0] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * RS + c) : 0u;
+        qa[ks][1] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * RS + c) : 0u;
+        qa[ks][2] = r0 ? *reinterpret_cast<const uint32_t *>(qb + qr * RS + c + 8) : 0u;
+        qa[ks][3] = r1 ? *reinterpret_cast<const uint32_t *>(qb + (qr + 8) * RS + c + 8) : 0u;
+    }
+}
+
 // ------------------------------------------------------------------------------------------------
 // decode kernel
 // ------------------------------------------------------------------------------------------------
@@ -583,7 +619,9 @@ __device__ __forceinline__ void load_q_frag(uint32_t (&qa)[D / 16][4], const Dec
 template <int D, int T, int STAGES, int NCW>
 __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                                   Plan<D, T, STAGES, NCW>::kMinBlocks)
-    decode_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ DecodeParams p)
+    decode_kernel(const __grid_constant__ CUtensorMap tmap,
+                  const __grid_constant__ CUtensorMap tmap_rows,
+                  const __grid_constant__ DecodeParams p)
 {
     using PL = Plan<D, T, STAGES, NCW>;
     constexpr int TW = PL::kTW;
@@ -630,8 +668,10 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         flags[0] = 0;   // abort
         fence_barrier_init();
     }
-    if (threadIdx.x == PL::kProducer * 32)
-        prefetch_tensormap(&tmap);   // a kernel parameter: safe before the dependency wait
+    if (threadIdx.x == PL::kProducer * 32) {
+        prefetch_tensormap(&tmap);   // kernel parameters: safe before the dependency wait
+        prefetch_tensormap(&tmap_rows);
+    }
     if (p.uniform_len <= 0) {
         for (int i = threadIdx.x; i < p.b; i += blockDim.x) {
             s_len[i] = p.seq_len[i];
@@ -652,15 +692,16 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // preceding layer (p.early_fetch, inside mlkv_decode_step), that kernel writes nothing this one
     // reads except the newest row (position L-1) of the slot it appended to, which lies in the
     // last tile of a segment, and the merge scratch (partials, counters).  So the queries and
-    // every other tile are read at once; the producer waits before it fetches a segment's last
+    // every other tile are fetched at once; the producer waits before it fetches a segment's last
     // tile, the epilogue warp before it writes its first record, and the consumers before they
     // write the last piece (scratch) or, at the latest, before they exit -- so this grid finishes
     // only after the previous one, as the next layer's wait expects.  The fused append writes
     // the newest row of this layer's own slot, which no earlier layer reads.
     const bool early = p.early_fetch != 0;
+    // The first piece's query fragments come straight from global memory, before the wait when
+    // the queries cannot be the previous kernel's output; later pieces find theirs in a slot.
     uint32_t qa[KS][4];
-    const bool q_early = early && warp < NCW && tile_lo < tile_hi;
-    if (q_early)
+    if (early && warp < NCW && tile_lo < tile_hi)
         load_q_frag<D>(qa, p, wk.beta, wk.j, lane);
     if (warp != PL::kProducer) {
         if (!early)
@@ -704,16 +745,44 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             if (flags[0])
                 break;
             const uint32_t fb = bar_full + 8 * s;
-            mbar_arrive_expect_tx(fb, PL::kStageBytes);
+            // A later piece starts here: its query rows come with the tile.
+            const bool with_q = (wk.tt == 0 && tile != tile_lo);
+            const uint32_t qbytes = static_cast<uint32_t>(p.G) * D * 2;
+            // A segment's last tile may be partly visible: only its boxes of 64 positions that
+            // hold visible rows are fetched (the rest of the stage keeps stale rows, which the
+            // consumers mask in S and zero in V).
+            const int vis = wk.L - wk.tt * T;
+            const int nbox = vis < T ? (vis + 63) / 64 : 0;
+            const uint32_t kv_bytes =
+                nbox > 0 ? static_cast<uint32_t>(nbox) * 64u * D * 2u * 2u : PL::kStageBytes;
+            mbar_arrive_expect_tx(fb, kv_bytes + (with_q ? qbytes : 0u));
+            if (with_q) {
+                const __nv_bfloat16 *q0 = p.Q + (static_cast<size_t>(wk.beta) * p.h +
+                                                 static_cast<size_t>(wk.j) * p.G) * D;
+                for (int r = 0; r < p.G; ++r)
+                    bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2,
+                              fb);
+            }
             const int zk = ((p.slot * 2 + 0) * p.b + wk.beta) * p.g + wk.j;
             const int zv = zk + p.b * p.g;
             const int y = wk.tt * T;
             const uint32_t kdst = sbase + s * PL::kStageBytes;
             const uint32_t vdst = kdst + PL::kTileBytes;
+            if (nbox == 0) {
 #pragma unroll
-            for (int sub = 0; sub < PL::kSub; ++sub) {
-                tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
-                tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
+                for (int sub = 0; sub < PL::kSub; ++sub) {
+                    tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
+                    tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
+                }
+            } else {
+                for (int bx = 0; bx < nbox; ++bx) {
+#pragma unroll
+                    for (int sub = 0; sub < PL::kSub; ++sub) {
+                        const uint32_t off = sub * T * 128 + bx * 64 * 128;
+                        tma_load_3d(kdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zk);
+                        tma_load_3d(vdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zv);
+                    }
+                }
             }
             ++issued;
             if (issued == STAGES)
@@ -792,9 +861,19 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         const int piece_first = tile;
         const int piece_end = seg_end < tile_hi ? seg_end : tile_hi;
 
-        // The first piece's query fragments may already be loaded (before the dependency wait).
-        if (!(q_early && tile == tile_lo))
-            load_q_frag<D>(qa, p, beta, j, lane);
+        if (tile == tile_lo) {
+            if (!early)
+                load_q_frag<D>(qa, p, beta, j, lane);
+        } else {
+            // A later piece: its query rows arrive with its first tile (the loop's wait for that
+            // tile then returns at once).
+            const int s0 = it % STAGES;
+            if (!flags[0] && !mbar_wait(bar_full + 8 * s0, (it / STAGES) & 1)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitFull);
+            }
+            load_q_frag_smem<D, PL::kQRow / 2>(qa, smem + PL::kQ + s0 * PL::kQSlot, G, lane);
+        }
 
         float o[NO][4];
 #pragma unroll
@@ -1387,7 +1466,7 @@ constexpr DecodeVariant make_variant()
 // (head_dim, positions per tile, ring stages, consumer warps); the first match of a
 // (head_dim, tile) pair is used.
 const DecodeVariant kVariants[] = {
-    make_variant<64, 128, 6, 8>(),
+    make_variant<64, 128, 5, 8>(),
     make_variant<64, 256, 3, 4>(),
     make_variant<64, 64, 4, 4>(),
     make_variant<128, 64, 5, 4>(),
@@ -1419,8 +1498,8 @@ cudaError_t prepare_decode_variant(const DecodeVariant &v, size_t max_smem)
 }
 
 cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStream_t stream,
-                          const CUtensorMap *tmap, const DecodeParams &p,
-                          const cudaAccessPolicyWindow *window, bool pdl)
+                          const CUtensorMap *tmap, const CUtensorMap *tmap_rows,
+                          const DecodeParams &p, const cudaAccessPolicyWindow *window, bool pdl)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -1448,7 +1527,8 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
     }
     cfg.attrs = attr;
     cfg.numAttrs = na;
-    void *args[] = {const_cast<CUtensorMap *>(tmap), const_cast<DecodeParams *>(&p)};
+    void *args[] = {const_cast<CUtensorMap *>(tmap), const_cast<CUtensorMap *>(tmap_rows),
+                    const_cast<DecodeParams *>(&p)};
     return cudaLaunchKernelExC(&cfg, v.fn, args);
 }
 

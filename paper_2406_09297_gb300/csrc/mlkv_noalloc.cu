@@ -197,19 +197,22 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     EncodeTiledFn encode = encode_fn();
     if (encode == nullptr)
         return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
-    CUtensorMap tmap;
+    CUtensorMap tmap, tmap_rows;
     const cuuint64_t dims[3] = {static_cast<cuuint64_t>(head_dim),
                                 static_cast<cuuint64_t>(max_seq),
                                 static_cast<cuuint64_t>(2 * S)};
     const cuuint64_t strides[2] = {static_cast<cuuint64_t>(head_dim) * 2,
                                    static_cast<cuuint64_t>(max_seq) * head_dim * 2};
-    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(T), 1u};
     const cuuint32_t estr[3] = {1u, 1u, 1u};
-    if (encode(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(kv_slot), dims,
-               strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
-        CUDA_SUCCESS)
-        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    for (int k = 0; k < 2; ++k) {
+        const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(k == 0 ? T : 64), 1u};
+        if (encode(k == 0 ? &tmap : &tmap_rows, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                   const_cast<void *>(kv_slot), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+            CUDA_SUCCESS)
+            return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    }
 
     p.Q = static_cast<const __nv_bfloat16 *>(Q);
     p.out = static_cast<__nv_bfloat16 *>(out);
@@ -237,7 +240,7 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.deferred_merge =
         mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces ? 1 : 0;
     const size_t smem = v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(batch));
-    e = mlkv::launch_decode(*v, grid, smem, stream, &tmap, p, nullptr);
+    e = mlkv::launch_decode(*v, grid, smem, stream, &tmap, &tmap_rows, p, nullptr);
     if (e != cudaSuccess)
         return fail(MLKV_ERR_CUDA, "decode launch failed");
     if (p.deferred_merge && mlkv::launch_combine(p, head_dim, stream) != cudaSuccess)
