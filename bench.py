@@ -201,17 +201,23 @@ def _config_dict(w):
             "l2": "flushed before every timed step (512 MiB write)", "parallelism": "replicas"}
 
 
+KERNEL_SOURCES = ("mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_device.cuh")
+
+
 def _kernel_source_hash():
+    """sha256[:16] over the kernel sources, in KERNEL_SOURCES order."""
     import hashlib
-    path = os.path.join(ROOT, "paper_2406_09297_gb300", "csrc", "mlkv_kernels.cu")
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2406_09297_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
-def _recorded_traffic(w):
+def _recorded_traffic(w, kernel):
     """DRAM bytes per decode launch (dram__bytes_read.sum + dram__bytes_write.sum) from the ncu
-    capture recorded in profiles/decode_traffic.json for this workload, or None when there is none
-    or the kernel source changed since it was taken."""
+    capture recorded in profiles/decode_traffic.json for this workload and kernel, or None when
+    there is none or the kernel source changed since it was taken."""
     try:
         with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
             rec = json.load(f)
@@ -219,6 +225,8 @@ def _recorded_traffic(w):
         return None
     entry = rec.get(w.name)
     if not entry or entry.get("kernel_source_sha256_16") != _kernel_source_hash():
+        return None
+    if entry.get("kernel", "decode_kernel") != kernel:
         return None
     return entry.get("dram_bytes_per_launch")
 
@@ -249,6 +257,7 @@ def run(args, w):
         cache.set_option("l2_persist", 1)
     if args.no_pdl:
         cache.set_option("pdl", 0)
+    cache.set_option("tc", args.tc)
     owners = w.owners()
     seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
     Qs = torch.stack(Q)                              # [l][b][h][d]
@@ -324,7 +333,8 @@ def run(args, w):
     cold = [layer_ms[n] for n in range(w.l) if w.owner[n] == n]
     cold_gbs = alg_bytes / (statistics.mean(cold) / 1e3) / 1e9
     del big_flush
-    traffic = _recorded_traffic(w)
+    kernel_name = "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel"
+    traffic = _recorded_traffic(w, kernel_name)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
     host_q = Qs.cpu().pin_memory()
@@ -382,7 +392,7 @@ def run(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind,
-                         "kernel": "decode_kernel", "alg_bytes_per_launch": alg_bytes,
+                         "kernel": kernel_name, "alg_bytes_per_launch": alg_bytes,
                          "mean_launch_ms": mean_kernel_ms,
                          "owner_launch_gbs": cold_gbs, "owner_launch_frac": cold_gbs / peak},
             "step_kv_gbs": kv_layer * w.l / (ms / 1e3) / 1e9,
@@ -409,6 +419,8 @@ def main():
     ap.add_argument("--grid", type=int, default=0)
     ap.add_argument("--l2-persist", action="store_true")
     ap.add_argument("--no-pdl", action="store_true")
+    ap.add_argument("--tc", type=int, default=0, choices=[0, 1],
+                    help="0: the mma.sync decode kernel (default); 1: the tcgen05 kernel")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

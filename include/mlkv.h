@@ -177,9 +177,14 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  the previous kernel of the stream (it touches no global memory before that
  *                  kernel has completed); 0 = plain stream order
  *   "step_graph"   1 (default) = mlkv_decode_step replays a recorded CUDA graph (see there)
+ *   "tc"           0 (default) = the decode kernel on mma.sync tensor-core instructions; 1 = the
+ *                  tcgen05 kernel (tensor-memory accumulators) for 128- and 256-position tiles,
+ *                  the mma.sync kernel otherwise.  Same results within the tolerance; the tcgen05
+ *                  kernel is slower for query groups of <= 16 heads (see the design notes).
  * Read-only (mlkv_get_option): "sm_count", "l2_bytes", "max_grid", "ctas_per_sm", and for the most
  * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge),
- * "last_deferred_merge", and "step_graph_replays" (graph launches by mlkv_decode_step).
+ * "last_deferred_merge", "last_tc" (1 if it ran the tcgen05 kernel), and "step_graph_replays"
+ * (graph launches by mlkv_decode_step).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.
  */
 int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);

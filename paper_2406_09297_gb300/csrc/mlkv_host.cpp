@@ -115,6 +115,7 @@ struct mlkv_cache {
     int l2_persist = 0;
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
+    int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     // mlkv_decode_step's recorded graph and the arguments it was recorded for
     int step_graph = 1;
     cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
@@ -123,17 +124,17 @@ struct mlkv_cache {
         const void *Q = nullptr, *K = nullptr, *V = nullptr;
         void *out = nullptr;
         std::vector<int> lens;
-        int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1;
+        int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1, tc = -1;
         bool operator==(const StepKey &o) const
         {
             return Q == o.Q && K == o.K && V == o.V && out == o.out && lens == o.lens &&
                    tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
-                   l2 == o.l2;
+                   l2 == o.l2 && tc == o.tc;
         }
     } step_key;
     int step_graph_replays = 0;
     // the most recent decode launch (read-only options, for tests and tuning)
-    int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0;
+    int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0, last_tc = 0;
     // per-variant launch state
     struct Variant {
         const mlkv::DecodeVariant *v = nullptr;
@@ -174,10 +175,16 @@ int default_tile_tokens(int d, double mean_len)
 mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0)
 {
     const int T = c->tile_tokens > 0 ? c->tile_tokens : default_tile_tokens(c->d, mean_len);
-    for (auto &v : c->variants)
-        if (v.v->tile_tokens == T)
+    mlkv_cache::Variant *plain = nullptr;
+    for (auto &v : c->variants) {
+        if (v.v->tile_tokens != T)
+            continue;
+        if (v.v->tc == c->tc)
             return &v;
-    return nullptr;
+        if (!v.v->tc)
+            plain = &v;
+    }
+    return plain;   // no tcgen05 variant for this tile: the mma.sync kernel
 }
 
 int encode_tmap(mlkv_cache *c, int rows, CUtensorMap *out)
@@ -312,8 +319,9 @@ int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_d
     c->window_max = prop.accessPolicyMaxWindowSize;
     c->max_smem = prop.sharedMemPerBlockOptin;
 
-    for (int T : {64, 128, 256}) {
-        const mlkv::DecodeVariant *v = mlkv::find_decode_variant(c->d, T);
+    for (int vi = 0; vi < 6; ++vi) {
+        const int T = 64 << (vi % 3);
+        const mlkv::DecodeVariant *v = mlkv::find_decode_variant(c->d, T, vi / 3);
         if (v == nullptr)
             continue;
         e = mlkv::prepare_decode_variant(*v, c->max_smem);
@@ -570,6 +578,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     c->last_grid = grid;
     c->last_tile = T;
     c->last_cluster_k = cluster_k;
+    c->last_tc = var->v->tc;
     c->last_deferred = p.deferred_merge;
     return MLKV_OK;
 }
@@ -648,6 +657,7 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
     key.grid = c->grid;
     key.cluster = c->cluster;
     key.pdl = c->pdl;
+    key.tc = c->tc;
     key.l2 = c->l2_persist;
     if (c->step_exec == nullptr || !(key == c->step_key)) {
         // Record the step once for these arguments (on a private stream: the caller's may be the
@@ -813,6 +823,12 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->step_graph = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "tc") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "tc must be 0 or 1");
+        c->tc = static_cast<int>(value);
+        return MLKV_OK;
+    }
     return fail(MLKV_ERR_INVALID_ARG, "unknown option '%s'", key);
 }
 
@@ -842,6 +858,14 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "step_graph") == 0) {
         *value = c->step_graph;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "tc") == 0) {
+        *value = c->tc;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_tc") == 0) {
+        *value = c->last_tc;
         return MLKV_OK;
     }
     if (std::strcmp(key, "step_graph_replays") == 0) {

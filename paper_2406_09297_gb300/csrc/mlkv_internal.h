@@ -65,13 +65,19 @@ struct DecodeVariant {
     size_t smem_bytes;        // without the per-sequence tables (see table_bytes)
     size_t res_bytes;         // one piece result slot (cluster mode adds k-1 of them)
     const void *fn;
+    int tc = 0;               // 1: decode_tc_kernel (tcgen05, TMEM), 0: decode_kernel (mma.sync)
 };
+
+// The tcgen05 variants (mlkv_decode_tc.cu).
+extern const DecodeVariant kTcVariants[];
+extern const int kNumTcVariants;
 
 // Shared memory a launch adds for the per-sequence tables (only when lengths differ).
 inline size_t table_bytes(int batch) { return ((8 * static_cast<size_t>(batch) + 4) + 15) & ~15ull; }
 
-// Returns the compiled variant for (head_dim, tile_tokens), or nullptr.
-const DecodeVariant *find_decode_variant(int head_dim, int tile_tokens);
+// Returns the compiled variant for (head_dim, tile_tokens) of the tcgen05 kernel (tc = 1) or of
+// the mma.sync kernel (tc = 0), or nullptr.
+const DecodeVariant *find_decode_variant(int head_dim, int tile_tokens, int tc = 0);
 
 // Raises the variant's dynamic shared-memory limit (capped at max_smem, the device's opt-in
 // per-block maximum); call once per device before the first launch.

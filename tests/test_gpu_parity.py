@@ -22,6 +22,38 @@ def test_tile_edges_single_layer(d, tile, fused):
                    fused=fused)
 
 
+# The tcgen05 kernel (option "tc"): 128- and 256-position tiles, both head sizes, ragged lengths,
+# split segments (stream-K records, inline and deferred merges) and DSMEM clusters.
+@pytest.mark.parametrize("d,tile", [(64, 128), (64, 256), (128, 128)])
+@pytest.mark.parametrize("fused", [False, True])
+def test_tc_tile_edges(d, tile, fused):
+    b = len(TILE_EDGE_LENS)
+    run_small_case([0], 4, 2, d, b, TILE_EDGE_LENS, 300, seed=21,
+                   options={"tile_tokens": tile, "tc": 1}, fused=fused, expect={"last_tc": 1})
+
+
+@pytest.mark.parametrize("grid", [3, 7, 64, 600])
+def test_tc_split_merges(grid):
+    lens = [700, 1, 129, 1000]
+    run_small_case([0, 0], 16, 1, 64, len(lens), lens, 1024, seed=22,
+                   options={"grid": grid, "tile_tokens": 128, "tc": 1}, fused=True,
+                   expect={"last_tc": 1})
+
+
+@pytest.mark.parametrize("name,owner,h,g,d", [
+    ("mha", [0, 1, 2], 4, 4, 64), ("gqa-mlkv", [0, 0, 0, 3, 3, 3], 12, 4, 64),
+    ("mqa-g16", [0, 1], 16, 1, 128), ("non-uniform", [0, 0, 0, 3, 4, 4], 8, 2, 128)])
+def test_tc_maps(name, owner, h, g, d):
+    lens = [5, 130, 77, 260]
+    run_small_case(owner, h, g, d, len(lens), lens, 320, seed=23,
+                   options={"tc": 1, "tile_tokens": 128}, expect={"last_tc": 1})
+
+
+def test_tc_cluster_merge():
+    run_small_case([0, 0, 2], 12, 1, 64, 64, [2048] * 64, 2048, seed=24, fused=True,
+                   options={"tc": 1}, expect={"last_tc": 1, "last_cluster_k": 2})
+
+
 @pytest.mark.parametrize("lens", [[2048] * 4, [512, 1, 77, 2048], [600] * 3])
 def test_default_tile_choice(lens):
     # the default tile length depends on the mean length; both choices are checked
