@@ -408,6 +408,81 @@ def run(args, w):
     return result
 
 
+# The nine Pythia-160M variants of Table 2 (Sec. 4.2): (name, owner layers m, KV heads g), block map
+# of Eq. 18.
+TABLE2_VARIANTS = [("baseline", 12, 12), ("gqa-48", 12, 4), ("mlkv-48", 4, 12), ("mqa-12", 12, 1),
+                   ("mlkv-12", 4, 3), ("mlkv-6", 6, 1), ("mlkv-4", 4, 1), ("mlkv-2", 2, 1),
+                   ("mlkv-1", 1, 1)]
+LOOP_PREFIX, LOOP_STEPS = 2000, 48
+
+
+def run_loop(args):
+    """The paper's throughput measurement (Sec. 4.5) on this library: a cache pre-filled with 2000
+    positions, then 48 autoregressive decode steps -- every step appends a new token per owner
+    layer (lengths grow by one) and attends in all 12 layers, one mlkv_decode_step call per step.
+    Timed on the device over whole 48-step loops (host work between steps included, as it is in
+    a decode loop), L2 flushed before each loop; tokens/s = batch * 48 / loop time, per variant.
+    Attention only (the paper times the whole model)."""
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device
+
+    torch.cuda.set_device(0)
+    l, h, d, b = 12, 12, 64, args.loop_batch
+    max_seq = LOOP_PREFIX + LOOP_STEPS
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    results, per_step_us = {}, {}
+    for name, m, g in TABLE2_VARIANTS:
+        owner = [int(x) for x in mlkv.mlkv_block_owner_map(l, m)]
+        owners = sorted(set(owner))
+        seed = 2000 + m * 16 + g
+        with mlkv.MLKVCache(l, h, d, owner, g, b, max_seq) as cache:
+            cache.set_option("tc", args.tc)
+            if args.grid:
+                cache.set_option("grid", args.grid)
+            for n in owners:
+                kp, vp, strides = cache.kv_ptr(cache.owner_slot(n)[1])
+                device.fill_slot(kp, vp, strides, seed, n, b, g, d, max_seq)
+            lens = [np.full(b, LOOP_PREFIX + s + 1, dtype=np.int32) for s in range(LOOP_STEPS)]
+            # per step: every layer's queries (another seed per step) and every owner's new token
+            Qs = [torch.stack([device.q_tensor(seed + 1 + s, n, b, h, d) for n in range(l)])
+                  for s in range(LOOP_STEPS)]
+            Ks = [torch.stack([device.kv_token(seed, n, 0, b, g, d, lens[s]) for n in owners])
+                  for s in range(LOOP_STEPS)]
+            Vs = [torch.stack([device.kv_token(seed, n, 1, b, g, d, lens[s]) for n in owners])
+                  for s in range(LOOP_STEPS)]
+            out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+
+            def loop():
+                for s in range(LOOP_STEPS):
+                    cache.decode_step(Qs[s], Ks[s], Vs[s], out, lens[s])
+
+            for _ in range(max(args.warmup, 1)):
+                loop()
+            cache.sync_status()
+            times = []
+            for _ in range(args.loop_reps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                loop()
+                e1.record()
+                torch.cuda.synchronize()
+                times.append(e0.elapsed_time(e1))
+            cache.sync_status()
+            ms = statistics.median(times)
+            results[name] = b * LOOP_STEPS / (ms / 1e3)
+            per_step_us[name] = ms * 1e3 / LOOP_STEPS
+    line = {"metric": "decode-loop tokens/s (prefix 2000, 48 decode steps, attention only)",
+            "unit": "tokens/s", "higher_is_better": True, "batch": b, "layers": l, "q_heads": h,
+            "head_dim": d, "reps": args.loop_reps, "dtype": "bf16", "data": "synthetic",
+            "kernel": "decode_tc_kernel" if args.tc else "decode_kernel",
+            "results": {k: round(v, 1) for k, v in results.items()},
+            "us_per_step": {k: round(v, 2) for k, v in per_step_us.items()}}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -422,8 +497,15 @@ def main():
     ap.add_argument("--tc", type=int, default=0, choices=[0, 1],
                     help="0: the mma.sync decode kernel (default); 1: the tcgen05 kernel")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--loop", action="store_true",
+                    help="the decode-loop measurement over the nine Table 2 variants")
+    ap.add_argument("--loop-batch", type=int, default=8)
+    ap.add_argument("--loop-reps", type=int, default=5)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.loop:
+        run_loop(args)
+        return
 
     from mlkv_synth import workloads
     w = workloads.by_name(args.config)

@@ -130,10 +130,12 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
  *   K, V     device bf16 [m][batch][g][d], every owner layer's new token, in slot order
  *   out      device bf16 [l][batch][h][d]
  *   seq_lens host int32[batch], as for mlkv_decode_attention
- * With option "step_graph" = 1 (default) the launches of a step are recorded into a CUDA graph on
- * the first call and replayed by later calls with the same pointers, lengths and options (new
- * values in the same buffers are fine); a change re-records.  When cuda_stream is itself being
- * captured the launches are issued directly, into the caller's graph.
+ * With option "step_graph" = 1 (default) a call whose pointers, lengths and options equal those of
+ * the previous call replays a CUDA graph of the step's launches (recorded on the second such call;
+ * new values in the same buffers are fine); a call with arguments different from the previous
+ * call's issues the launches directly, which costs the host about half of recording them -- the
+ * case of a decode loop, whose lengths grow every step.  When cuda_stream is itself being captured
+ * the launches are issued directly, into the caller's graph.
  */
 int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
                      const int *seq_lens, void *cuda_stream);

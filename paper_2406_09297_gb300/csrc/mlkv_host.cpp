@@ -131,7 +131,7 @@ struct mlkv_cache {
                    tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
                    l2 == o.l2 && tc == o.tc;
         }
-    } step_key;
+    } step_key, pending_key;   // recorded arguments; arguments seen once, not yet recorded
     int step_graph_replays = 0;
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0, last_tc = 0;
@@ -491,34 +491,45 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     if (tiles > 0x7fffffffLL)
         return fail(MLKV_ERR_UNSUPPORTED, "%lld tiles exceed the int32 tile index", tiles);
     p.tile_start[c->b] = static_cast<int>(tiles);
-    // Cluster mode: every segment splits into k equal pieces held by one k-CTA cluster, merged over
-    // DSMEM; taken when it keeps the one-wave makespan and every cluster is resident at once.
+    // The launch shape.  A one-wave stream-K grid (the fewest CTAs with the makespan of one wave
+    // of resident CTAs) fits large layers, where every SM streams many tiles and the merge of the
+    // few split segments is amortised.  When every sequence has one length two more shapes can
+    // be better for a small layer: whole segments per CTA (no merge at all), or each segment in k
+    // equal pieces run as one k-CTA cluster and merged over DSMEM.  They are chosen with a cost
+    // model in units of one tile's consumer work (~0.5 us on GB300 when the tile is in L2):
+    // a DSMEM cluster merge costs ~2 tiles, the last-CTA merge of up to 4 partial records ~6 (a
+    // global write, an atomic and the reads, after the previous layer has finished) and the
+    // separate combine launch ~7.
+    const long long wave = std::min<long long>(
+        std::min(var->ctas_per_sm * c->sm_count, c->max_ctas), tiles);
+    const long long per_wave = (tiles + wave - 1) / wave;
     int cluster_k = 0;
-    if (uniform && c->grid == 0 && c->cluster) {
-        const long long nt = (seq_lens[0] + T - 1) / T;
-        const long long S = static_cast<long long>(c->b) * c->g;
-        const long long wave = std::min<long long>(
-            std::min(var->ctas_per_sm * c->sm_count, c->max_ctas), tiles);
-        const long long makespan = (tiles + wave - 1) / wave;
-        for (int k : {2, 4}) {
-            if (nt % k == 0 && S * k <= wave && nt / k <= makespan && var->clusters[k] >= S) {
-                cluster_k = k;
-                break;
-            }
-        }
-    }
     int grid;
-    if (cluster_k > 1) {
-        grid = static_cast<int>(static_cast<long long>(c->b) * c->g * cluster_k);
-    } else if (c->grid > 0) {
+    if (c->grid > 0) {
         grid = static_cast<int>(std::min<long long>(std::min(c->grid, c->max_ctas), tiles));
     } else {
-        // One wave of resident CTAs sets the makespan ceil(tiles / wave); the fewest CTAs with
-        // that makespan split fewer segments (e.g. 512 tiles over 152 SMs: 128 CTAs of 4).
-        const long long wave = std::min<long long>(
-            std::min(var->ctas_per_sm * c->sm_count, c->max_ctas), tiles);
-        const long long per = (tiles + wave - 1) / wave;
-        grid = static_cast<int>((tiles + per - 1) / per);
+        grid = static_cast<int>((tiles + per_wave - 1) / per_wave);
+        if (uniform) {
+            const long long nt = (seq_lens[0] + T - 1) / T;
+            const long long S = static_cast<long long>(c->b) * c->g;
+            const long long per = tiles / grid;
+            const long long pieces = per > 0 ? (nt - 1 + per - 1) / per + 1 : grid;
+            long long best = per_wave + (pieces <= 1 ? 0 : pieces <= mlkv::kInlineMergeMaxPieces ? 6 : 7);
+            if (S <= wave && nt < best) {
+                best = nt;   // whole segments: grid S, each CTA exactly one segment
+                grid = static_cast<int>(S);
+            }
+            if (c->cluster) {
+                for (int k : {2, 4}) {
+                    if (nt % k == 0 && S * k <= wave && var->clusters[k] >= S && nt / k + 2 < best) {
+                        best = nt / k + 2;
+                        cluster_k = k;
+                    }
+                }
+                if (cluster_k > 1)
+                    grid = static_cast<int>(S * cluster_k);
+            }
+        }
     }
     grid = std::max(std::min(grid, mlkv::kCombineMaxPiecesHost), 1);
 
@@ -660,6 +671,13 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
     key.tc = c->tc;
     key.l2 = c->l2_persist;
     if (c->step_exec == nullptr || !(key == c->step_key)) {
+        if (!(key == c->pending_key)) {
+            // Arguments not seen on the previous call: issue the launches directly (about half the
+            // host time of recording them), since in a decode loop lengths change every step.
+            // Arguments that come back on the next call are recorded then.
+            c->pending_key = key;
+            return issue_step(c, q, k, v, o, seq_lens, cuda_stream);
+        }
         // Record the step once for these arguments (on a private stream: the caller's may be the
         // legacy default stream, which cannot be captured), then replay it on the caller's.
         if (c->record_stream == nullptr &&

@@ -46,7 +46,7 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
         _inputs(owner, h, g, d, b, lens, max_seq, seed, cache2, None)
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.full((l, b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
-        for rep in range(3):   # record, then replay twice
+        for rep in range(4):   # direct, record, then replay twice
             out.fill_(float("nan"))
             cache.decode_step(Q, K, V, out, lens)
         torch.cuda.synchronize()
@@ -124,3 +124,46 @@ def test_step_inside_a_caller_graph():
         graph.replay()
         torch.cuda.synchronize()
         assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
+
+
+@pytest.mark.parametrize("owner,h,g,d,b,prefix", [
+    ([0, 0, 2, 2], 8, 2, 64, 3, [100, 257, 512]),
+    ([0, 0, 0, 0, 0, 0], 12, 1, 64, 8, [2000] * 8),   # the decode-loop benchmark's shape, shortened
+])
+def test_decode_loop_growing_lengths(owner, h, g, d, b, prefix):
+    # Autoregressive decode as in the paper's throughput measurement (Sec. 4.5): from a
+    # pre-filled cache, every step appends a new token per owner layer (lengths grow by one) and
+    # attends over the cache in every layer; every step of every layer is checked.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    seed, steps = 41, 5
+    l = len(owner)
+    owners = sorted(set(owner))
+    max_seq = max(prefix) + steps
+    with mlkv.MLKVCache(l, h, d, owner, g, b, max_seq) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, max_seq)
+        for n in owners:
+            kb = gen.gen_kv(seed, n, 0, b, g, max_seq, d)
+            vb = gen.gen_kv(seed, n, 1, b, g, max_seq, d)
+            cache.load_prefix(n, to_dev(kb), to_dev(vb), max_seq)
+            ref.load_prefix(n, gen.bf16_bits_to_f64(kb), gen.bf16_bits_to_f64(vb), max_seq)
+        out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        for s in range(steps):
+            lens = np.asarray(prefix, dtype=np.int32) + s + 1
+            qb = np.stack([gen.gen_q(seed + 100 + s, n, b, h, d) for n in range(l)])
+            kn = np.stack([gen.gen_bf16(seed + 200 + s, gen.TID_K + n, range(b * g), d)
+                           .reshape(b, g, d) for n in owners])
+            vn = np.stack([gen.gen_bf16(seed + 200 + s, gen.TID_V + n, range(b * g), d)
+                           .reshape(b, g, d) for n in owners])
+            out.fill_(float("nan"))
+            cache.decode_step(to_dev(qb), to_dev(kn), to_dev(vn), out, lens)
+            torch.cuda.synchronize()
+            for n in range(l):
+                if owner[n] == n:
+                    k = owners.index(n)
+                    ref.append(n, gen.bf16_bits_to_f64(kn[k]), gen.bf16_bits_to_f64(vn[k]), lens)
+                expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens)
+                mx, mean = errors(from_dev(out[n]), expect)
+                assert mx <= MAX_ABS and mean <= MEAN_ABS, (s, n, mx, mean)
+        cache.sync_status()
