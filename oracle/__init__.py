@@ -39,6 +39,10 @@ def load(path):
         ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, ctypes.c_int,
         ctypes.c_int, _ip, ctypes.c_int, _dp, ctypes.POINTER(_dp), ctypes.POINTER(_dp), _dp,
         ctypes.c_int]
+    L.oracle_prefill_layer.argtypes = [
+        ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+        ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, _dp, ctypes.POINTER(_dp),
+        ctypes.POINTER(_dp), _dp, ctypes.c_int]
     L.oracle_append.argtypes = [
         ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, ctypes.c_int, _ip,
         ctypes.c_int, _dp, _dp, ctypes.POINTER(_dp), ctypes.POINTER(_dp)]
@@ -157,6 +161,23 @@ class OracleCache:
                                        out.ctypes.data_as(_dp), nthreads)
         if rc != ORACLE_OK:
             raise ValueError(f"oracle_decode_layer failed ({rc})")
+        return out
+
+
+    def prefill(self, layer, Q, prompt_lens, nthreads=1):
+        """Causal prefill of one layer; Q [b][s_max][h][d] -> out [b][s_max][h][d] (rows past a
+        prompt's length stay zero).  The owner's cache must hold the prompt's K/V."""
+        pl, pp = _ints(prompt_lens)
+        Q, qp = _f64(Q)
+        b, s_max, h, d = Q.shape
+        assert b == self.b and h == self.h and d == self.d
+        out = np.zeros((b, s_max, h, d), dtype=np.float64)
+        karr, varr = self._ptr_arrays()
+        rc = lib().oracle_prefill_layer(layer, self.l, self.owner.ctypes.data_as(_ip), self.h,
+                                        self.g, self.d, self.b, pp, s_max, self.max_seq, qp,
+                                        karr, varr, out.ctypes.data_as(_dp), nthreads)
+        if rc != ORACLE_OK:
+            raise ValueError(f"oracle_prefill_layer failed ({rc})")
         return out
 
 

@@ -1,5 +1,5 @@
 /*
- * MLKV decode-attention oracle.
+ * MLKV decode- and prefill-attention oracle.
  *
  * TEST INFRASTRUCTURE ONLY.  This file states, in plain double-precision C, what the MLKV decode
  * path computes, so that the CUDA library can be checked against it.  Only the test suite,
@@ -239,6 +239,112 @@ int oracle_decode_layer(int layer, int l, const int *owner, int h, int g, int d,
     /* any job whose thread could not be started runs here */
     for (int w = started + 1; w < nthreads; ++w)
         run_layer_job(&jobs[w]);
+    rc = ORACLE_OK;
+    for (int w = 0; w < nthreads; ++w)
+        if (jobs[w].status != ORACLE_OK)
+            rc = jobs[w].status;
+    free(jobs);
+    free(tids);
+    return rc;
+}
+
+typedef struct {
+    int layer, h, g, d, max_seq, s_max;
+    const int *owner;
+    const int *prompt_lens;
+    const double *Q;
+    const double *const *Kc;
+    const double *const *Vc;
+    double *out;
+    int beta_lo, beta_hi;
+    int status;
+} prefill_job;
+
+static void *run_prefill_job(void *arg)
+{
+    prefill_job *jb = (prefill_job *)arg;
+    int h = jb->h, g = jb->g, d = jb->d;
+    int k_owner = jb->owner[jb->layer];                                /* Eqs. 13-18 */
+    const double *Kown = jb->Kc[k_owner];
+    const double *Vown = jb->Vc[k_owner];
+    double *work = (double *)malloc(sizeof(double) * (size_t)(jb->s_max > 0 ? jb->s_max : 1));
+    if (work == NULL) {
+        jb->status = ORACLE_ERR_OOM;
+        return NULL;
+    }
+    for (int beta = jb->beta_lo; beta < jb->beta_hi; ++beta) {
+        int S = jb->prompt_lens[beta];
+        for (int t = 0; t < S; ++t) {
+            int L = t + 1;                     /* position t sees positions 0 .. t */
+            for (int i = 0; i < h; ++i) {
+                int j = oracle_kv_head_of(h, g, i);                    /* Eq. 15 */
+                const double *q = jb->Q + (((size_t)beta * jb->s_max + t) * h + i) * d;
+                size_t kv_row = ((size_t)beta * g + j) * (size_t)jb->max_seq * d;
+                double *o = jb->out + (((size_t)beta * jb->s_max + t) * h + i) * d;
+                attention_one_query(q, Kown + kv_row, Vown + kv_row, L, d, work, o);
+            }
+        }
+    }
+    free(work);
+    jb->status = ORACLE_OK;
+    return NULL;
+}
+
+/* Prefill of one layer: the prompt processed at once.  A decoder-only model (Sec. 2.1; the
+ * autoregressive order of Sec. 4.5) lets prompt position t attend to positions 0 .. t only, so
+ * every row is Eqs. 2-3 over the owner's KV head j(i) (Eqs. 13-18) at visible length t + 1 --
+ * the decode of Sec. 3 at that length.
+ *   Q    [b][s_max][h][d]   the prompt's queries, position-major
+ *   Kc,Vc as for oracle_decode_layer (the owner's cache holds the prompt's K/V)
+ *   out  [b][s_max][h][d]   rows t >= prompt_lens[beta] are left untouched
+ * nthreads > 1 splits the batch across POSIX threads. */
+int oracle_prefill_layer(int layer, int l, const int *owner, int h, int g, int d, int b,
+                         const int *prompt_lens, int s_max, int max_seq, const double *Q,
+                         const double *const *Kc, const double *const *Vc, double *out,
+                         int nthreads)
+{
+    int rc = oracle_validate(l, owner, h, g, d);
+    if (rc != ORACLE_OK)
+        return rc;
+    if (layer < 0 || layer >= l || b < 0 || s_max <= 0 || s_max > max_seq || Q == NULL ||
+        out == NULL)
+        return ORACLE_ERR_ARG;
+    if (Kc == NULL || Vc == NULL || Kc[owner[layer]] == NULL || Vc[owner[layer]] == NULL)
+        return ORACLE_ERR_ARG;
+    for (int beta = 0; beta < b; ++beta)
+        if (prompt_lens[beta] < 1 || prompt_lens[beta] > s_max)
+            return ORACLE_ERR_RANGE;
+    if (nthreads < 1)
+        nthreads = 1;
+    if (nthreads > b)
+        nthreads = b > 0 ? b : 1;
+    prefill_job *jobs = (prefill_job *)calloc((size_t)nthreads, sizeof(prefill_job));
+    pthread_t *tids = (pthread_t *)calloc((size_t)nthreads, sizeof(pthread_t));
+    if (jobs == NULL || tids == NULL) {
+        free(jobs);
+        free(tids);
+        return ORACLE_ERR_OOM;
+    }
+    for (int w = 0; w < nthreads; ++w) {
+        prefill_job *jb = &jobs[w];
+        jb->layer = layer; jb->h = h; jb->g = g; jb->d = d; jb->max_seq = max_seq;
+        jb->s_max = s_max; jb->owner = owner; jb->prompt_lens = prompt_lens; jb->Q = Q;
+        jb->Kc = Kc; jb->Vc = Vc; jb->out = out;
+        jb->beta_lo = (int)((long long)b * w / nthreads);
+        jb->beta_hi = (int)((long long)b * (w + 1) / nthreads);
+        jb->status = ORACLE_ERR_ARG;
+    }
+    int started = 0;
+    for (int w = 1; w < nthreads; ++w) {
+        if (pthread_create(&tids[w], NULL, run_prefill_job, &jobs[w]) != 0)
+            break;
+        started = w;
+    }
+    run_prefill_job(&jobs[0]);
+    for (int w = 1; w <= started; ++w)
+        pthread_join(tids[w], NULL);
+    for (int w = started + 1; w < nthreads; ++w)
+        run_prefill_job(&jobs[w]);
     rc = ORACLE_OK;
     for (int w = 0; w < nthreads; ++w)
         if (jobs[w].status != ORACLE_OK)

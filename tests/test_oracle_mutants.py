@@ -1,7 +1,8 @@
 """Plants plausible mistakes in a copy of the oracle (on the CPU) and checks that the pin suite of
 test_oracle_pins.py rejects every one of them: a dropped scale, a wrong group map, a block map
 that picks the wrong layer, an off-by-one visible length, a missing normalisation, a flipped sign,
-a wrong query row, a dropped factor in the cache size, a mis-numbered slot and a misplaced append.
+a wrong query row, a dropped factor in the cache size, a mis-numbered slot, a misplaced append,
+a prefill row that does not see its own position and prefill queries read head-major.
 """
 import os
 import subprocess
@@ -25,6 +26,10 @@ MUTANTS = [
     ("cache-size-drops-g", "return 2LL * b * s * m * g * dk;", "return 2LL * b * s * m * dk;"),
     ("slot-from-one", "slot[q] = m;", "slot[q] = m + 1;"),
     ("append-at-zero", "(size_t)(L - 1)) * d;", "(size_t)0) * d;"),
+    ("prefill-excludes-self", "int L = t + 1;                     /* position t sees positions 0 .. t */",
+     "int L = t > 0 ? t : 1;"),
+    ("prefill-head-major-rows", "const double *q = jb->Q + (((size_t)beta * jb->s_max + t) * h + i) * d;",
+     "const double *q = jb->Q + (((size_t)beta * h + i) * jb->s_max + t) * d;"),
 ]
 
 PIN_TESTS = [
@@ -40,6 +45,8 @@ PIN_TESTS = [
     pins.test_dominant_key_selects_its_value,
     pins.test_brute_force_decimal,
     pins.test_append_only_for_owner_layers,
+    lambda: [pins.test_prefill_matches_causal_sdpa(*m) for m in pins.MAPS],
+    pins.test_prefill_first_position_returns_value_row,
 ]
 
 

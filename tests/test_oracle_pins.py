@@ -8,6 +8,8 @@
 * MLKV (Sec. 3) equals MHA run on explicitly duplicated K/V, bit for bit.
 * Closed forms: one visible position, equal keys, zero query, one dominant key.
 * Brute force on tiny inputs in 50-digit decimal arithmetic, without max subtraction.
+* Prefill: torch's scaled_dot_product_attention with its causal mask, in float64, per prompt; the
+  first prompt position returns its value row; MLKV prefill equals MHA prefill on duplicated K/V.
 """
 import decimal
 import os
@@ -300,3 +302,64 @@ def test_append_only_for_owner_layers():
         c.V[2][beta, :, t] = 0.0
     assert not c.K[2].any() and not c.V[2].any()               # nothing else was written
     assert not c.K[0].any()
+
+
+# ----------------------------------------------------------------------------------------------
+# prefill (causal attention over a whole prompt)
+# ----------------------------------------------------------------------------------------------
+
+def _prefill_problem(rng, owner, h, g, d, b, s_max, prompt_lens):
+    c = oracle.OracleCache(owner, h, g, d, b, s_max)
+    for n in sorted(set(owner)):
+        c.load_prefix(n, rng.standard_normal((b, g, s_max, d)), rng.standard_normal((b, g, s_max, d)),
+                      s_max)
+    Q = rng.standard_normal((len(owner), b, s_max, h, d))
+    return c, Q
+
+
+@pytest.mark.parametrize("name,owner,h,g", MAPS)
+def test_prefill_matches_causal_sdpa(name, owner, h, g):
+    rng = np.random.default_rng(17)
+    d, b, s_max = 16, 3, 23
+    prompt_lens = np.array([1, 9, 23], dtype=np.int32)
+    c, Q = _prefill_problem(rng, owner, h, g, d, b, s_max, prompt_lens)
+    G = h // g
+    for layer in range(len(owner)):
+        got = c.prefill(layer, Q[layer], prompt_lens)
+        own = owner[layer]
+        for beta in range(b):
+            S = int(prompt_lens[beta])
+            k = torch.repeat_interleave(torch.from_numpy(c.K[own][beta, :, :S, :]), G, dim=0)
+            v = torch.repeat_interleave(torch.from_numpy(c.V[own][beta, :, :S, :]), G, dim=0)
+            q = torch.from_numpy(np.ascontiguousarray(Q[layer][beta, :S].transpose(1, 0, 2)))
+            o = torch.nn.functional.scaled_dot_product_attention(q[None], k[None], v[None],
+                                                                 is_causal=True)
+            np.testing.assert_allclose(got[beta, :S], o[0].numpy().transpose(1, 0, 2), rtol=0,
+                                       atol=1e-13)
+            assert not got[beta, S:].any()
+
+
+def test_prefill_first_position_returns_value_row():
+    rng = np.random.default_rng(19)
+    owner, h, g, d, b, s_max = [0, 0], 4, 2, 8, 2, 6
+    c, Q = _prefill_problem(rng, owner, h, g, d, b, s_max, None)
+    prompt_lens = np.array([6, 3], dtype=np.int32)
+    for layer in range(2):
+        got = c.prefill(layer, Q[layer], prompt_lens)
+        for i in range(h):
+            np.testing.assert_array_equal(got[:, 0, i], c.V[0][:, i // 2, 0])
+
+
+def test_prefill_mlkv_equals_mha_on_duplicated_kv():
+    rng = np.random.default_rng(23)
+    owner, h, g, d, b, s_max = [0, 0, 2, 2], 6, 3, 8, 2, 11
+    prompt_lens = np.array([11, 5], dtype=np.int32)
+    c, Q = _prefill_problem(rng, owner, h, g, d, b, s_max, prompt_lens)
+    mha = oracle.OracleCache(list(range(4)), h, h, d, b, s_max)
+    G = h // g
+    for n in range(4):
+        for i in range(h):
+            mha.K[n][:, i] = c.K[owner[n]][:, i // G]
+            mha.V[n][:, i] = c.V[owner[n]][:, i // G]
+    for n in range(4):
+        assert np.array_equal(c.prefill(n, Q[n], prompt_lens), mha.prefill(n, Q[n], prompt_lens))
