@@ -201,7 +201,7 @@ def _config_dict(w):
             "l2": "flushed before every timed step (512 MiB write)", "parallelism": "replicas"}
 
 
-KERNEL_SOURCES = ("mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_device.cuh")
+KERNEL_SOURCES = ("mlkv_kernels.cu", "mlkv_device.cuh")   # what decode_kernel is built from
 
 
 def _kernel_source_hash():
@@ -483,6 +483,79 @@ def run_loop(args):
     print(json.dumps(line), flush=True)
 
 
+def _tensor_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def run_prefill(args, w):
+    """Prefill of a whole prompt per sequence through every layer of the workload's model, in layer
+    order (owner layers store the prompt's K/V, every layer attends causally over its owner's
+    slot): one mlkv_prefill per layer, timed on the device, L2 flushed before each repetition.
+    tokens/s = batch * prompt / time; TFLOP/s counts the useful causal work
+    4 * h * d * sum_beta S (S + 1) / 2 per layer (QK^T and PV, 2 flops a multiply-add)."""
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device
+
+    torch.cuda.set_device(0)
+    b, S = args.prefill_batch, args.prefill_len
+    owners = w.owners()
+    with mlkv.MLKVCache(w.l, w.h, w.d, w.owner, w.g, b, S) as cache:
+        Q = [torch.empty((b, S, w.h, w.d), dtype=torch.bfloat16, device="cuda") for _ in range(w.l)]
+        for n in range(w.l):
+            device.fill_(Q[n].view(b * S, w.h * w.d), w.seed + 1, 0x100 + n, w.sigma_q)
+        KV = {}
+        for n in owners:
+            k = torch.empty((b, w.g, S, w.d), dtype=torch.bfloat16, device="cuda")
+            v = torch.empty_like(k)
+            device.fill_(k.view(b * w.g, S * w.d), w.seed + 1, 0x200 + n, w.sigma_k)
+            device.fill_(v.view(b * w.g, S * w.d), w.seed + 1, 0x300 + n, w.sigma_v)
+            KV[n] = (k, v)
+        out = torch.empty((b, S, w.h, w.d), dtype=torch.bfloat16, device="cuda")
+        lens = np.full(b, S, dtype=np.int32)
+        flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+        def prefill_model():
+            for n in range(w.l):
+                k, v = KV.get(n, (None, None))
+                cache.prefill(n, Q[n], k, v, out, lens)
+
+        for _ in range(args.warmup):
+            prefill_model()
+        cache.sync_status()
+        times = []
+        with Clocks(0) as clocks:
+            for _ in range(args.steps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                prefill_model()
+                e1.record()
+                torch.cuda.synchronize()
+                times.append(e0.elapsed_time(e1))
+        cache.sync_status()
+    ms = statistics.median(times)
+    flops = 4.0 * w.h * w.d * b * S * (S + 1) / 2 * w.l
+    tflops = flops / (ms / 1e3) / 1e12
+    peak, kind = _tensor_peak()
+    line = {"metric": "prefill tokens/s (all layers, causal)", "value": b * S / (ms / 1e3),
+            "unit": "tokens/s", "higher_is_better": True, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "layers": w.l, "q_heads": w.h, "head_dim": w.d,
+                       "layer_owner": list(w.owner), "kv_heads_per_owner": w.g, "batch": b,
+                       "prompt": S, "l2": "flushed before every timed repetition"},
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+                         "frac": tflops / peak, "peak_source": kind, "kernel": "prefill_kernel",
+                         "flops_per_step": flops},
+            "clocks": clocks.summary()}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -501,10 +574,18 @@ def main():
                     help="the decode-loop measurement over the nine Table 2 variants")
     ap.add_argument("--loop-batch", type=int, default=8)
     ap.add_argument("--loop-reps", type=int, default=5)
+    ap.add_argument("--prefill", action="store_true",
+                    help="prefill throughput of the --config model (prompt of --prefill-len)")
+    ap.add_argument("--prefill-batch", type=int, default=8)
+    ap.add_argument("--prefill-len", type=int, default=2048)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.loop:
         run_loop(args)
+        return
+    if args.prefill:
+        from mlkv_synth import workloads
+        run_prefill(args, workloads.by_name(args.config))
         return
 
     from mlkv_synth import workloads

@@ -141,6 +141,27 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
                      const int *seq_lens, void *cuda_stream);
 
 /*
+ * mlkv_prefill - the prompt of every sequence through one layer at once (prefill): owner layers
+ * first store the prompt's K/V at positions [0, s_max) of their slot (Sec. 3: only a layer with KV
+ * heads of its own stores them); then prompt position t of query head i attends, causally, to
+ * positions 0 .. t of KV head i / (h/g) of the layer's owner (Eqs. 2-3 at every prompt position,
+ * maps of Eqs. 13-18).  A later mlkv_decode_step continues each sequence at length
+ * prompt_lens[beta] + 1.  Runs on the tcgen05 tensor cores.
+ *
+ *   Q            device bf16 [batch][s_max][h][d], position-major (a token's heads contiguous)
+ *   K, V         device bf16 [batch][g][s_max][d], the prompt's keys / values; read only for an
+ *                owner layer (may be NULL otherwise)
+ *   out          device bf16 [batch][s_max][h][d]; rows past a prompt's length are not written
+ *   prompt_lens  host int32[batch], 1 <= prompt_lens[beta] <= s_max
+ *   s_max        1 <= s_max <= max_seq
+ * The caller keeps the buffers valid until the stream reaches the call.  Errors:
+ * MLKV_ERR_INVALID_ARG (null or unaligned pointer, out overlapping Q), MLKV_ERR_RANGE (lengths),
+ * MLKV_ERR_CUDA.
+ */
+int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const void *V, void *out,
+                 const int *prompt_lens, int s_max, void *cuda_stream);
+
+/*
  * mlkv_load_prefix - bulk-stores positions [0, len) of an owner layer's keys and values
  * (prefill).  K, V: device bf16 [batch][g][len][d].  No-op (MLKV_OK) for a non-owner layer.
  * Paper: Sec. 4.5 starts decoding from a pre-filled ("dummy") cache.

@@ -19,7 +19,8 @@ NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc" if os.path.exists(
     "/usr/local/cuda/bin/nvcc") else "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
-SOURCES = ["mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_host.cpp", "mlkv_noalloc.cu"]
+SOURCES = ["mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_prefill.cu", "mlkv_host.cpp",
+           "mlkv_noalloc.cu"]
 
 
 def _sources():
@@ -28,6 +29,7 @@ def _sources():
 
 def _deps():
     deps = _sources() + [os.path.join(CSRC, "mlkv_internal.h"), os.path.join(CSRC, "mlkv_device.cuh"),
+                         os.path.join(CSRC, "mlkv_tcgen05.cuh"),
                          os.path.join(INCLUDE, "mlkv.h"),
                          os.path.abspath(__file__)]
     return deps

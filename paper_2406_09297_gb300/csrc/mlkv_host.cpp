@@ -116,6 +116,7 @@ struct mlkv_cache {
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
+    int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
     // mlkv_decode_step's recorded graph and the arguments it was recorded for
     int step_graph = 1;
     cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
@@ -752,6 +753,112 @@ int mlkv_load_prefix(mlkv_cache_t c, int layer, const void *K, const void *V, in
                               cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess)
         return fail_cuda(e, "prefix copy");
+    return MLKV_OK;
+}
+
+int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const void *V, void *out,
+                 const int *prompt_lens, int s_max, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (layer < 0 || layer >= c->l)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->l);
+    if (s_max < 1 || s_max > c->max_seq)
+        return fail(MLKV_ERR_RANGE, "s_max %d outside [1, %d]", s_max, c->max_seq);
+    if (Q == nullptr || out == nullptr || !aligned16(Q) || !aligned16(out))
+        return fail(MLKV_ERR_INVALID_ARG, "Q and out must be non-NULL and 16-byte aligned");
+    if (prompt_lens == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "prompt_lens must be non-NULL");
+    int max_len = 0;
+    for (int beta = 0; beta < c->b; ++beta) {
+        if (prompt_lens[beta] < 1 || prompt_lens[beta] > s_max)
+            return fail(MLKV_ERR_RANGE, "prompt length %d of sequence %d outside [1, %d]",
+                        prompt_lens[beta], beta, s_max);
+        max_len = std::max(max_len, prompt_lens[beta]);
+    }
+    const size_t qbytes = static_cast<size_t>(c->b) * s_max * c->h * c->d * 2;
+    const char *qs = static_cast<const char *>(Q);
+    const char *os = static_cast<const char *>(out);
+    if (os < qs + qbytes && qs < os + qbytes)
+        return fail(MLKV_ERR_INVALID_ARG, "out overlaps Q");
+    const bool owner = c->owner[layer] == layer;
+    if (owner && (K == nullptr || V == nullptr || !aligned16(K) || !aligned16(V)))
+        return fail(MLKV_ERR_INVALID_ARG, "K and V must be non-NULL and 16-byte aligned");
+    DeviceGuard guard(c->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    // Sec. 3: only an owner layer stores K/V -- the prompt's, at positions [0, s_max).
+    if (owner) {
+        int rc = mlkv_load_prefix(c, layer, K, V, s_max, cuda_stream);
+        if (rc != MLKV_OK)
+            return rc;
+    }
+    cudaError_t e;
+    if (!c->prefill_ready) {
+        if ((e = mlkv::prepare_prefill(c->d)) != cudaSuccess)
+            return fail_cuda(e, "cudaFuncSetAttribute(prefill)");
+        c->prefill_ready = 1;
+    }
+    // The queries, position-major [b][s_max][h][d]: boxes of 64 channels x 1 head x 128 positions.
+    static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
+    if (encode == nullptr)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+    CUtensorMap tmap_q;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->h),
+                                static_cast<cuuint64_t>(s_max), static_cast<cuuint64_t>(c->b)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(c->d) * 2,
+                                   static_cast<cuuint64_t>(c->h) * c->d * 2,
+                                   static_cast<cuuint64_t>(s_max) * c->h * c->d * 2};
+    const cuuint32_t box[4] = {64u, 1u, 128u, 1u};
+    const cuuint32_t estr[4] = {1u, 1u, 1u, 1u};
+    CUresult r = encode(&tmap_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(Q), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled(Q) failed (CUresult %d)",
+                    static_cast<int>(r));
+    // The cache, with boxes of 128 positions (the map of the 128-position decode variant).
+    const CUtensorMap *tmap_kv = nullptr;
+    for (auto &v : c->variants)
+        if (v.v->tile_tokens == 128)
+            tmap_kv = &v.tmap;
+    if (tmap_kv == nullptr)
+        return fail(MLKV_ERR_UNSUPPORTED, "no 128-position cache map for d=%d", c->d);
+
+    static thread_local mlkv::PrefillParams p;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.err = c->err;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
+    p.b = c->b;
+    p.h = c->h;
+    p.g = c->g;
+    p.G = c->G;
+    p.s_max = s_max;
+    p.slot = c->slot[layer];
+    for (int beta = 0; beta < c->b; ++beta)
+        p.prompt_len[beta] = prompt_lens[beta];
+    // Work items (sequence, block of 128 positions), the blocks that see the most keys first.
+    const int max_blocks = (max_len + 127) / 128;
+    int n = 0;
+    for (int qb = max_blocks - 1; qb >= 0; --qb) {
+        for (int beta = 0; beta < c->b; ++beta) {
+            if (qb * 128 >= prompt_lens[beta])
+                continue;
+            p.item_beta[n] = beta;
+            p.item_qb[n] = qb;
+            if (++n == mlkv::kPrefillMaxItems) {
+                p.n_items = n;
+                if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+                    return fail_cuda(e, "prefill launch");
+                n = 0;
+            }
+        }
+    }
+    if (n > 0) {
+        p.n_items = n;
+        if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+            return fail_cuda(e, "prefill launch");
+    }
     return MLKV_OK;
 }
 

@@ -48,6 +48,26 @@ struct DecodeParams {
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };
 
+// Causal prefill of one layer (mlkv_prefill.cu): one CTA per (work item, query head), a work item
+// being one block of 128 prompt positions of one sequence.  Passed by value.
+constexpr int kPrefillMaxItems = 2048;   // work items per launch (more: several launches)
+struct PrefillParams {
+    __nv_bfloat16 *out;       // [b][s_max][h][D]
+    int *err;                 // device error word
+    float scale_log2;         // log2(e) / sqrt(D)
+    int b, h, g, G, s_max, slot, n_items;
+    int prompt_len[MLKV_MAX_BATCH];
+    int item_beta[kPrefillMaxItems];
+    int item_qb[kPrefillMaxItems];
+};
+
+// Dynamic shared memory of the prefill kernel; sets its limit (once per device); launches it with
+// programmatic dependent launch on `stream`.
+size_t prefill_smem_bytes(int head_dim);
+cudaError_t prepare_prefill(int head_dim);
+cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
+                           const PrefillParams &p, cudaStream_t stream);
+
 struct AppendParams {
     const __nv_bfloat16 *K;   // [b][g][D]
     const __nv_bfloat16 *V;

@@ -29,7 +29,7 @@ EXPORTED = [
     "mlkv_append_decode_attention", "mlkv_decode_step",
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
-    "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static",
+    "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
 ]
 
 
@@ -67,6 +67,7 @@ def _load():
     L.mlkv_block_owner_map.argtypes = [ci, ci, ip]
     L.mlkv_version.argtypes = []
     L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
+    L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
     return L
 
 
@@ -141,6 +142,12 @@ def mlkv_decode_step(handle, Q, K, V, out, seq_lens, stream=None):
     a, p = _lens_ptr(seq_lens)
     return _check(lib.mlkv_decode_step(handle, _ptr(Q), _ptr(K), _ptr(V), _ptr(out), p,
                                        _stream(stream)))
+
+
+def mlkv_prefill(handle, layer, Q, K, V, out, prompt_lens, s_max, stream=None):
+    a, p = _lens_ptr(prompt_lens)
+    return _check(lib.mlkv_prefill(handle, layer, _ptr(Q), _ptr(K), _ptr(V), _ptr(out), p, s_max,
+                                   _stream(stream)))
 
 
 def mlkv_load_prefix(handle, layer, K, V, length, stream=None):
@@ -245,6 +252,10 @@ class MLKVCache:
 
     def decode_step(self, Q, K, V, out, seq_lens, stream=None):
         return mlkv_decode_step(self.handle, Q, K, V, out, seq_lens, stream)
+
+    def prefill(self, layer, Q, K, V, out, prompt_lens, stream=None):
+        """Causal prefill of one layer; Q / out [b][s_max][h][d], K / V [b][g][s_max][d]."""
+        return mlkv_prefill(self.handle, layer, Q, K, V, out, prompt_lens, int(Q.shape[1]), stream)
 
     def load_prefix(self, layer, K, V, length, stream=None):
         return mlkv_load_prefix(self.handle, layer, K, V, length, stream)
