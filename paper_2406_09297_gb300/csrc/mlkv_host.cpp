@@ -769,6 +769,9 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
         return fail(MLKV_ERR_INVALID_ARG, "Q and out must be non-NULL and 16-byte aligned");
     if (prompt_lens == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "prompt_lens must be non-NULL");
+    if (c->h > mlkv::kPrefillMaxHeads || s_max > mlkv::kPrefillMaxBlocks * 128)
+        return fail(MLKV_ERR_UNSUPPORTED, "prefill handles at most %d query heads and %d positions",
+                    mlkv::kPrefillMaxHeads, mlkv::kPrefillMaxBlocks * 128);
     int max_len = 0;
     for (int beta = 0; beta < c->b; ++beta) {
         if (prompt_lens[beta] < 1 || prompt_lens[beta] > s_max)
@@ -837,25 +840,32 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
     p.slot = c->slot[layer];
     for (int beta = 0; beta < c->b; ++beta)
         p.prompt_len[beta] = prompt_lens[beta];
-    // Work items (sequence, block of 128 positions), the blocks that see the most keys first.
+    // Work units, those that see the most keys first: two heads of a group at the same block when
+    // the group size is even, else the blocks 2p and 2p+1 of one head (the unit of block 2p+1).
+    p.head_pairs = (c->G % 2 == 0) ? 1 : 0;
+    const int sels = p.head_pairs ? c->h / 2 : c->h;
     const int max_blocks = (max_len + 127) / 128;
     int n = 0;
     for (int qb = max_blocks - 1; qb >= 0; --qb) {
         for (int beta = 0; beta < c->b; ++beta) {
-            if (qb * 128 >= prompt_lens[beta])
+            const int nb = (prompt_lens[beta] + 127) / 128;
+            if (qb >= nb || (!p.head_pairs && qb % 2 == 0 && qb != nb - 1))
                 continue;
-            p.item_beta[n] = beta;
-            p.item_qb[n] = qb;
-            if (++n == mlkv::kPrefillMaxItems) {
-                p.n_items = n;
-                if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
-                    return fail_cuda(e, "prefill launch");
-                n = 0;
+            for (int sel = 0; sel < sels; ++sel) {
+                p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(qb) << 10) |
+                             (static_cast<uint32_t>(sel) << 24);
+                if (++n == mlkv::kPrefillMaxUnits) {
+                    p.n_units = n;
+                    if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) !=
+                        cudaSuccess)
+                        return fail_cuda(e, "prefill launch");
+                    n = 0;
+                }
             }
         }
     }
     if (n > 0) {
-        p.n_items = n;
+        p.n_units = n;
         if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
             return fail_cuda(e, "prefill launch");
     }

@@ -48,17 +48,21 @@ struct DecodeParams {
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };
 
-// Causal prefill of one layer (mlkv_prefill.cu): one CTA per (work item, query head), a work item
-// being one block of 128 prompt positions of one sequence.  Passed by value.
-constexpr int kPrefillMaxItems = 2048;   // work items per launch (more: several launches)
+// Causal prefill of one layer (mlkv_prefill.cu): one CTA per work unit, a unit being two query
+// tiles of 128 prompt positions over one KV head.  Passed by value.
+//   units[u] = beta | qb_b << 10 | sel << 24, qb_b the block (of 128 positions) of tile B.
+//   head_pairs = 1 (G even): tiles A and B are heads 2 sel and 2 sel + 1 at block qb_b.
+//   head_pairs = 0 (G odd):  both are head sel; A is block qb_b - 1 when qb_b is odd, else absent.
+constexpr int kPrefillMaxUnits = 6144;   // units per launch (more: several launches)
+constexpr int kPrefillMaxHeads = 256;    // sel has 8 bits
+constexpr int kPrefillMaxBlocks = 1 << 14;
 struct PrefillParams {
     __nv_bfloat16 *out;       // [b][s_max][h][D]
     int *err;                 // device error word
     float scale_log2;         // log2(e) / sqrt(D)
-    int b, h, g, G, s_max, slot, n_items;
+    int b, h, g, G, s_max, slot, n_units, head_pairs;
     int prompt_len[MLKV_MAX_BATCH];
-    int item_beta[kPrefillMaxItems];
-    int item_qb[kPrefillMaxItems];
+    uint32_t units[kPrefillMaxUnits];
 };
 
 // Dynamic shared memory of the prefill kernel; sets its limit (once per device); launches it with

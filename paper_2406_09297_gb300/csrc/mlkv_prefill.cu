@@ -5,29 +5,39 @@
 // attention, Eqs. 2-3 with the MLKV maps of Eqs. 13-18).  Owner layers first store the prompt's
 // K/V in their slot (mlkv_host.cpp); every layer of the block then attends over it.
 //
-// Work split: one CTA per (sequence, query head, block of 128 prompt positions), longest blocks
-// (those near the end of a prompt, which see the most keys) first.  Each CTA walks the key tiles
-// 0 .. qb of its block's causal triangle, 128 keys per tile.
+// Work unit (one CTA): two query tiles A and B of 128 prompt positions that read the same KV head,
+// so that every K/V tile is loaded once for both.  With an even group size G they are two heads of
+// one group at the same positions (identical causal triangles); otherwise they are the blocks
+// 2p and 2p+1 of one head (B sees one tile more; a last block without a partner runs alone as B).
+// Units that see the most keys run first.
 //
-// Math, per key tile (all MMAs tcgen05.mma kind::f16, bf16 in, fp32 accumulate in TMEM):
-//   S = Q K^T       M = 128 queries (A = the query tile, loaded once by TMA, K-major with the
-//                   128-byte swizzle), N = 128 keys (B = the K tile as TMA left it), K = head_dim;
-//                   double-buffered in TMEM, one query row per TMEM lane.
-//   softmax         four warps, one thread per query row: the thread owns its row's 128 scores
-//                   (tcgen05.ld), so the online maximum needs no exchange between threads.  The
-//                   row's reference maximum is raised only when a score exceeds it by more than
-//                   2^8 in the exponent; then the thread rescales its O row in TMEM (after the
-//                   previous tile's product has landed).  p = 2^(s log2(e)/sqrt(d) - m) is written
-//                   as bf16 to smem in the A-operand layout (K-major, 128-byte swizzle).
-//   O += P V        M = 128 queries, N = head_dim (B = the V tile read MN-major), K = 128 keys;
-//                   O stays in TMEM for the whole block.
-// The diagonal tile masks keys after the query; keys past the prompt's end only meet such
-// masked scores, and their V rows are zeroed in smem so that 0 * V stays 0.
+// Per key tile t and query tile X (all MMAs tcgen05.mma kind::f16, bf16 in, fp32 accumulate):
+//   S_X = Q_X K_t^T  M = 128 queries (A = Q_X, K-major, 128-byte swizzle as TMA wrote it),
+//                    N = 128 keys (B = the K tile), K = head_dim; one query row per TMEM lane.
+//   softmax          a warpgroup per query tile, one thread per row: the thread owns its row's
+//                    128 scores, so the running maximum needs no exchange between threads.  The
+//                    reference maximum is raised only when a score exceeds it by more than 2^8
+//                    (then the thread rescales its O row in TMEM); p = 2^(s log2(e)/sqrt(d) - m)
+//                    goes back to TMEM as bf16 pairs.
+//   O_X += P_X V_t   A = P_X read from TMEM, B = the V tile read MN-major from shared memory,
+//                    N = head_dim, K = 128 keys; O_X stays in TMEM for the whole unit.
+// While one warpgroup turns S into P, the tensor core works on the other query tile.
 //
-// Warp roles (192 threads): warps 0-3 softmax and output, warp 4 TMA producer (query tile, then a
-// ring of K/V tiles), warp 5 MMA issuer (event-driven: S of the next tile as soon as its K/V and a
-// TMEM buffer are ready, P V as soon as a tile's P is written).  Every wait is bounded; on expiry
-// the kernel records an error bit, stops, lets its copies and MMAs land and frees its TMEM.
+// TMEM (512 columns): S_A, S_B (128 each), O_A, O_B (head_dim each).  For head_dim 64, P has
+// columns of its own (so S of the next tile can be computed while P of this one is being written);
+// for head_dim 128, P overwrites the first 64 columns of its S (tcgen05.mma of one thread execute
+// in order, so S of the next tile is written after P V has read P).
+//
+// The diagonal tile masks keys after the query; keys past the prompt's end only meet such masked
+// scores, and their V rows are zeroed in shared memory so that 0 * V stays 0.
+//
+// Warp roles (384 threads): warps 0-3 query tile A, 4-7 query tile B (softmax and output), warp 8
+// TMA producer (both query tiles, then K_0, V_0, K_1, V_1, ... through a ring), warp 9 MMA issuer,
+// warps 10-11 idle.  The block launches with 168 registers a thread (three warps per SM
+// sub-partition); the last warpgroup gives registers back (64) and the softmax warpgroups take
+// them (216): 128 * 64 + 256 * 216 <= 384 * 168.
+// Every wait is bounded; on expiry the kernel records an error bit, stops, lets its copies and MMAs
+// land and frees its TMEM.
 #include "mlkv_device.cuh"
 #include "mlkv_tcgen05.cuh"
 
@@ -36,28 +46,49 @@ namespace {
 
 template <int D>
 struct PrefillPlan {
-    static constexpr int kThreads = 6 * 32;
-    static constexpr int kProducer = 4, kMma = 5;
-    static constexpr int kSub = D / 64;                   // 64-channel blocks of a row
-    static constexpr int kStages = D == 64 ? 4 : 2;
-    static constexpr int kTileBytes = 128 * D * 2;        // a Q, K or V tile of 128 rows
-    static constexpr int kStageBytes = 2 * kTileBytes;    // K and V
-    static constexpr int kPBytes = 128 * 128 * 2;         // P: [2 key blocks][128 rows][64] bf16
-    static constexpr int kQ = 0;
-    static constexpr int kRing = kQ + kTileBytes;
-    static constexpr int kP = kRing + kStages * kStageBytes;   // [2][kPBytes]
-    static constexpr int kFlags = kP + 2 * kPBytes;            // int [4], TMEM base at +16
-    // u64 barriers: q_full, full[S], empty[S], s_ready[2], s_free[2], p_ready[2], p_free[2],
-    // o_ready, fin
+    static constexpr int kThreads = 12 * 32;
+    static constexpr int kRegsLaunch = 168, kRegsLow = 64, kRegsHigh = 216;
+    static constexpr int kProducer = 8, kMma = 9;
+    static constexpr int kSub = D / 64;                      // 64-channel blocks of a row
+    static constexpr int kTileBytes = 128 * D * 2;           // 128 rows of Q, K or V
+    static constexpr int kRingTiles = D == 64 ? 8 : 4;       // K_t and V_t alternate in the ring
+    static constexpr int kQ = 0;                             // [2] query tiles
+    static constexpr int kRing = kQ + 2 * kTileBytes;
+    static constexpr int kFlags = kRing + kRingTiles * kTileBytes;   // int [4], TMEM base at +16
+    // u64 barriers: q, full[R], empty[R], s_ready[2], s_free[2], p_ready[2], pv_done[2], fin
     static constexpr int kBars = kFlags + 32;
-    static constexpr int kNumBars = 1 + 2 * kStages + 10;
+    static constexpr int kNumBars = 1 + 2 * kRingTiles + 8 + 1;
     static constexpr int kBytes = kBars + kNumBars * 8;
-    static constexpr int kAlloc = kBytes + 1024;               // base aligned up to 1024
-    static constexpr int kTmemCols = 512;                      // S: 2 x 128, O: D
-    static constexpr int kColS = 0, kColO = 256;
+    static constexpr int kAlloc = kBytes + 1024;             // base aligned up to 1024
+    static constexpr int kTmemCols = 512;
+    static constexpr bool kPSep = D == 64;                   // P in columns of its own
+    static constexpr int kColS = 0;                          // + 128 per query tile
+    static constexpr int kColO = 256;                        // + D per query tile
+    static constexpr int kColP = 384;                        // + 64 per query tile (kPSep)
     static_assert(D == 64 || D == 128, "head_dim 64 or 128");
-    static_assert(kRing % 1024 == 0 && kP % 1024 == 0, "swizzled tiles stay 1024-byte aligned");
+    static_assert(kRing % 1024 == 0 && kTileBytes % 1024 == 0, "swizzled tiles 1024-aligned");
+    static_assert(kColO + 2 * D <= (kPSep ? kColP : kTmemCols), "TMEM columns overlap");
+    static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kRegsLaunch, "register split");
 };
+
+template <int N>
+__device__ __forceinline__ void setmaxnreg_inc()
+{
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
+template <int N>
+__device__ __forceinline__ void setmaxnreg_dec()
+{
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
 
 template <int D>
 __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
@@ -66,48 +97,49 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                    const __grid_constant__ PrefillParams p)
 {
     using PL = PrefillPlan<D>;
-    constexpr int ST = PL::kStages;
+    constexpr int R = PL::kRingTiles;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const uint32_t sbase = smem_addr(smem);
     const uint32_t bar_q = sbase + PL::kBars;
     const uint32_t bar_full = bar_q + 8;
-    const uint32_t bar_empty = bar_full + 8 * ST;
-    const uint32_t bar_s_ready = bar_empty + 8 * ST;   // [2]
-    const uint32_t bar_s_free = bar_s_ready + 16;       // [2]
-    const uint32_t bar_p_ready = bar_s_free + 16;       // [2]
-    const uint32_t bar_p_free = bar_p_ready + 16;       // [2]
-    const uint32_t bar_o_ready = bar_p_free + 16;
-    const uint32_t bar_fin = bar_o_ready + 8;
+    const uint32_t bar_empty = bar_full + 8 * R;
+    const uint32_t bar_s_ready = bar_empty + 8 * R;   // [2] per query tile
+    const uint32_t bar_s_free = bar_s_ready + 16;
+    const uint32_t bar_p_ready = bar_s_free + 16;
+    const uint32_t bar_pv_done = bar_p_ready + 16;
+    const uint32_t bar_fin = bar_pv_done + 16;
     volatile int *flags = reinterpret_cast<volatile int *>(smem + PL::kFlags);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int item = blockIdx.x / p.h;
-    const int head = blockIdx.x - item * p.h;
-    const int beta = p.item_beta[item];
-    const int qb = p.item_qb[item];
+    // The unit: sequence, last query block of B, head pair or head (see PrefillParams::units).
+    const uint32_t u = p.units[blockIdx.x];
+    const int beta = static_cast<int>(u & 0x3FFu);
+    const int qb_b = static_cast<int>((u >> 10) & 0x3FFFu);
+    const int sel = static_cast<int>(u >> 24);
+    const int head_a = p.head_pairs ? 2 * sel : sel;
+    const int head_b = p.head_pairs ? 2 * sel + 1 : sel;
+    const int n_b = qb_b + 1;                                   // key tiles 0 .. qb_b
+    const int n_a = p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0);   // 0: no tile A
     const int S = p.prompt_len[beta];
-    const int q0 = qb * 128;
-    const int n_kt = qb + 1;                         // key tiles 0 .. qb (causal)
-    const int j = head / p.G;                        // Eq. 15
+    const int j = head_b / p.G;                                 // Eq. 15
     const int zk = ((p.slot * 2 + 0) * p.b + beta) * p.g + j;
     const int zv = zk + p.b * p.g;
 
     if (threadIdx.x == 0) {
         mbar_init(bar_q, 1);
-        for (int s = 0; s < ST; ++s) {
+        for (int s = 0; s < R; ++s) {
             mbar_init(bar_full + 8 * s, 1);
             mbar_init(bar_empty + 8 * s, 1);
         }
-        for (int r = 0; r < 2; ++r) {
-            mbar_init(bar_s_ready + 8 * r, 1);
-            mbar_init(bar_s_free + 8 * r, 4);
-            mbar_init(bar_p_ready + 8 * r, 4);
-            mbar_init(bar_p_free + 8 * r, 1);
+        for (int g = 0; g < 2; ++g) {
+            mbar_init(bar_s_ready + 8 * g, 1);
+            mbar_init(bar_s_free + 8 * g, 4);
+            mbar_init(bar_p_ready + 8 * g, 4);
+            mbar_init(bar_pv_done + 8 * g, 1);
         }
-        mbar_init(bar_o_ready, 1);
         mbar_init(bar_fin, 1);
         flags[0] = 0;
         fence_barrier_init();
@@ -130,246 +162,283 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     // The owner's K/V may have just been stored by the previous kernel of the stream.
     grid_dependency_wait();
     grid_dependents_launch();
-
     if (warp == PL::kProducer) {
         // ------------------------------------ producer ------------------------------------------
+        setmaxnreg_dec<PL::kRegsLow>();
         if (lane == 0) {
-            mbar_arrive_expect_tx(bar_q, PL::kTileBytes);
+            mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kTileBytes);
 #pragma unroll
-            for (int sub = 0; sub < PL::kSub; ++sub)
-                tma_load_4d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64, head, q0, beta);
-            int kt = 0;
-            for (; kt < n_kt; ++kt) {
-                const int s = kt % ST;
-                if (kt >= ST && !flags[0] &&
-                    !mbar_wait(bar_empty + 8 * s, ((kt / ST) & 1) ^ 1)) {
+            for (int sub = 0; sub < PL::kSub; ++sub) {
+                if (n_a > 0)
+                    tma_load_4d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64, head_a,
+                                (n_a - 1) * 128, beta);
+                tma_load_4d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
+                            sub * 64, head_b, qb_b * 128, beta);
+            }
+            const int n_idx = 2 * n_b;   // K_0, V_0, K_1, V_1, ...
+            int idx = 0;
+            for (; idx < n_idx; ++idx) {
+                const int s = idx % R;
+                if (idx >= R && !flags[0] &&
+                    !mbar_wait(bar_empty + 8 * s, ((idx / R) & 1) ^ 1)) {
                     flags[0] = 1;
                     atomicOr(p.err, kErrWaitEmpty);
                 }
                 if (flags[0])
                     break;
                 const uint32_t fb = bar_full + 8 * s;
-                mbar_arrive_expect_tx(fb, PL::kStageBytes);
-                const uint32_t kdst = sbase + PL::kRing + s * PL::kStageBytes;
+                mbar_arrive_expect_tx(fb, PL::kTileBytes);
+                const uint32_t dst = sbase + PL::kRing + s * PL::kTileBytes;
+                const int z = (idx & 1) ? zv : zk;
 #pragma unroll
-                for (int sub = 0; sub < PL::kSub; ++sub) {
-                    tma_load_3d(kdst + sub * 16384, &tmap_kv, fb, sub * 64, kt * 128, zk);
-                    tma_load_3d(kdst + PL::kTileBytes + sub * 16384, &tmap_kv, fb, sub * 64,
-                                kt * 128, zv);
-                }
+                for (int sub = 0; sub < PL::kSub; ++sub)
+                    tma_load_3d(dst + sub * 16384, &tmap_kv, fb, sub * 64, (idx >> 1) * 128, z);
             }
             // No copy may still be in flight when the CTA exits.
             if (!mbar_wait(bar_q, 0))
                 atomicOr(p.err, kErrDrain);
-            for (int k = kt > ST ? kt - ST : 0; k < kt; ++k)
-                if (!mbar_wait(bar_full + 8 * (k % ST), (k / ST) & 1))
+            for (int k = idx > R ? idx - R : 0; k < idx; ++k)
+                if (!mbar_wait(bar_full + 8 * (k % R), (k / R) & 1))
                     atomicOr(p.err, kErrDrain);
         }
         __syncwarp();
     } else if (warp == PL::kMma) {
         // ------------------------------------ MMA issuer ----------------------------------------
-        constexpr uint32_t kIdS = umma_idesc(128, 128, 0, 0);
-        constexpr uint32_t kIdPV = umma_idesc(128, D, 0, 1);
-        int si = 0, pi = 0;
-        bool ok = true;
-        uint64_t idle_since = 0;
-        while (pi < n_kt && ok) {
-            int act = 0;   // 1: O += P V of tile pi, 2: S of tile si
-            if (lane == 0) {
-                if (pi < si && mbar_test_wait(bar_p_ready + 8 * (pi & 1), (pi >> 1) & 1))
-                    act = 1;
-                else if (si < n_kt && (si > 0 || mbar_test_wait(bar_q, 0)) &&
-                         mbar_test_wait(bar_full + 8 * (si % ST), (si / ST) & 1) &&
-                         (si < 2 || mbar_test_wait(bar_s_free + 8 * (si & 1), ((si >> 1) & 1) ^ 1)))
-                    act = 2;
-            }
-            act = __shfl_sync(0xffffffffu, act, 0);
-            if (act == 0) {
-                if (lane == 0) {
-                    const uint64_t now = global_timer_ns();
-                    if (idle_since == 0)
-                        idle_since = now;
-                    else if (now - idle_since > kWaitLimitNs)
-                        ok = false;
-                }
-                ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-                if (ok && flags[0])
+        setmaxnreg_dec<PL::kRegsLow>();
+        if (lane == 0) {
+            constexpr uint32_t kIdS = umma_idesc(128, 128, 0, 0);
+            constexpr uint32_t kIdPV = umma_idesc(128, D, 0, 1);
+            const int n[2] = {n_a, n_b};
+            bool ok = true;
+            auto wait = [&](uint32_t bar, int parity) {
+                if (ok && (flags[0] || !mbar_wait(bar, static_cast<uint32_t>(parity) & 1u)))
                     ok = false;
-                continue;
-            }
-            idle_since = 0;
-            tmem_fence_after();
-            if (act == 2) {
-                if (lane == 0) {
-                    const uint32_t kt = sbase + PL::kRing + (si % ST) * PL::kStageBytes;
+                return ok;
+            };
+            auto ring = [&](int idx) { return sbase + PL::kRing + (idx % R) * PL::kTileBytes; };
+            auto tile_full = [&](int idx) { return wait(bar_full + 8 * (idx % R), idx / R); };
+            auto issue_s = [&](int g, int t) {
+                const uint32_t qt = sbase + PL::kQ + g * PL::kTileBytes;
+                const uint32_t kt = ring(2 * t);
 #pragma unroll
-                    for (int k = 0; k < D / 16; ++k)
-                        umma_f16(tmem + PL::kColS + (si & 1) * 128,
-                                 umma_desc(sbase + PL::kQ + (k >> 2) * 16384 + (k & 3) * 32, 16,
-                                           1024, kLayoutSw128),
-                                 umma_desc(kt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
-                                           kLayoutSw128),
-                                 kIdS, k > 0 ? 1 : 0);
-                    umma_commit(bar_s_ready + 8 * (si & 1));
-                }
-                __syncwarp();
-                ++si;
-            } else {
-                if (lane == 0) {
-                    const uint32_t vt =
-                        sbase + PL::kRing + (pi % ST) * PL::kStageBytes + PL::kTileBytes;
-                    const uint32_t pt = sbase + PL::kP + (pi & 1) * PL::kPBytes;
+                for (int k = 0; k < D / 16; ++k)
+                    umma_f16(tmem + PL::kColS + 128 * g,
+                             umma_desc(qt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
+                                       kLayoutSw128),
+                             umma_desc(kt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
+                                       kLayoutSw128),
+                             kIdS, k > 0 ? 1 : 0);
+                umma_commit(bar_s_ready + 8 * g);
+            };
+            auto issue_pv = [&](int g, int t) {
+                const uint32_t vt = ring(2 * t + 1);
+                const uint32_t pc = tmem + (PL::kPSep ? PL::kColP + 64 * g : PL::kColS + 128 * g);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k)
-                        umma_f16(tmem + PL::kColO,
-                                 umma_desc(pt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
-                                           kLayoutSw128),
-                                 umma_desc(vt + k * 2048, 16384, 1024, kLayoutSw128), kIdPV,
-                                 (pi == 0 && k == 0) ? 0 : 1);
-                    umma_commit(bar_empty + 8 * (pi % ST));   // the K/V stage may be refilled
-                    umma_commit(bar_p_free + 8 * (pi & 1));   // the P buffer may be rewritten
-                    if (pi == n_kt - 1)
-                        umma_commit(bar_o_ready);
-                }
-                __syncwarp();
-                ++pi;
+                for (int k = 0; k < 8; ++k)
+                    umma_f16_ts(tmem + PL::kColO + D * g, pc + 8 * k,
+                                umma_desc(vt + k * 2048, 16384, 1024, kLayoutSw128), kIdPV,
+                                (t > 0 || k > 0) ? 1 : 0);
+                umma_commit(bar_pv_done + 8 * g);
+            };
+            if (wait(bar_q, 0) && tile_full(0)) {
+                tmem_fence_after();
+                for (int g = 0; g < 2; ++g)
+                    if (n[g] > 0)
+                        issue_s(g, 0);
+                umma_commit(bar_empty);   // K_0 (ring slot 0)
             }
-        }
-        if (!ok) {
-            flags[0] = 1;
-            if (lane == 0)
-                atomicOr(p.err, kErrWaitFull);
-        }
-        if (lane == 0)
-            umma_commit(bar_fin);
-        __syncwarp();
-        if (!mbar_wait(bar_fin, 0) && lane == 0)
-            atomicOr(p.err, kErrDrain);
-        __syncwarp();
-    } else {
-        // ------------------------------------ softmax warps -------------------------------------
-        const int r = threadIdx.x;   // query row of the block = TMEM lane
-        const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-        const float scale = p.scale_log2;
-        const float NEG_INF = -__int_as_float(0x7f800000);
-        float m_run = NEG_INF, l_run = 0.f;
-        for (int t = 0; t < n_kt; ++t) {
-            if (!flags[0] && !mbar_wait(bar_s_ready + 8 * (t & 1), (t >> 1) & 1)) {
+            for (int t = 0; ok && t < n_b; ++t) {
+                for (int g = 0; g < 2 && ok; ++g) {
+                    if (t >= n[g])
+                        continue;
+                    const bool next = t + 1 < n[g];
+                    if (PL::kPSep && next) {
+                        // S of the next tile as soon as this one's S has been read.
+                        if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
+                            break;
+                        tmem_fence_after();
+                        issue_s(g, t + 1);
+                    }
+                    if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
+                        break;
+                    tmem_fence_after();
+                    issue_pv(g, t);
+                    if (!PL::kPSep && next) {
+                        if (!tile_full(2 * t + 2))
+                            break;
+                        issue_s(g, t + 1);
+                    }
+                }
+                if (!ok)
+                    break;
+                umma_commit(bar_empty + 8 * ((2 * t + 1) % R));       // V_t, read by both
+                if (t + 1 < n_b)
+                    umma_commit(bar_empty + 8 * ((2 * t + 2) % R));   // K_{t+1}, read by both
+            }
+            if (!ok) {
                 flags[0] = 1;
                 atomicOr(p.err, kErrWaitFull);
             }
+            umma_commit(bar_fin);
+            if (!mbar_wait(bar_fin, 0))
+                atomicOr(p.err, kErrDrain);
+        }
+        __syncwarp();
+    } else if (warp < 8) {
+        // ------------------------------------ softmax warpgroups --------------------------------
+        setmaxnreg_inc<PL::kRegsHigh>();
+        const int grp = warp >> 2;                  // 0: query tile A, 1: query tile B
+        const int r = threadIdx.x & 127;            // query row of the tile = TMEM lane
+        const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const int n_g = grp ? n_b : n_a;
+        const int head = grp ? head_b : head_a;
+        const int q0 = (n_g - 1) * 128;
+        const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * grp;
+        const uint32_t col_o = tmem + lane_off + PL::kColO + D * grp;
+        const uint32_t col_p =
+            tmem + lane_off + (PL::kPSep ? PL::kColP + 64 * grp : PL::kColS + 128 * grp);
+        const uint32_t s_ready = bar_s_ready + 8 * grp, s_free = bar_s_free + 8 * grp;
+        const uint32_t p_ready = bar_p_ready + 8 * grp, pv_done = bar_pv_done + 8 * grp;
+        // The prompt's last block holds keys past its end; the first tile to reach it zeroes them.
+        const bool zero_v = n_g > 0 && n_g == (S + 127) / 128 && (grp == 0 || n_a != n_b);
+        const float scale = p.scale_log2;
+        const float NEG_INF = -__int_as_float(0x7f800000);
+        auto wait = [&](uint32_t bar, int parity) {
+            if (!flags[0] && !mbar_wait(bar, static_cast<uint32_t>(parity) & 1u)) {
+                flags[0] = 1;
+                atomicOr(p.err, kErrWaitFull);
+            }
+        };
+        float m_run = NEG_INF, l_run = 0.f;
+        for (int t = 0; t < n_g; ++t) {
+            wait(s_ready, t);
             tmem_fence_after();
             float sv[4][32];
 #pragma unroll
             for (int c = 0; c < 4; ++c)
-                tmem_ld32_nowait(tmem + lane_base + PL::kColS + (t & 1) * 128 + c * 32, sv[c]);
+                tmem_ld32_nowait(col_s + c * 32, sv[c]);
             tmem_wait_ld();
-            tmem_fence_before();
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(bar_s_free + 8 * (t & 1));
-            const bool diag = (t == qb);
-            float mx = NEG_INF;
+            if (PL::kPSep) {
+                tmem_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(s_free);
+            }
+            const bool diag = t == n_g - 1;
+            if (diag) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
+                for (int c = 0; c < 4; ++c)
 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    if (diag && c * 32 + k > r)
-                        sv[c][k] = NEG_INF;   // a later position: causal mask
-                    mx = fmaxf(mx, sv[c][k]);
+                    for (int k = 0; k < 32; ++k)
+                        if (c * 32 + k > r)
+                            sv[c][k] = NEG_INF;   // a later position: causal mask
+            }
+            float mx[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float a = max3f(sv[c][0], sv[c][1], sv[c][2]);
+                float b = max3f(sv[c][3], sv[c][4], sv[c][5]);
+#pragma unroll
+                for (int k = 6; k < 30; k += 4) {
+                    a = max3f(a, sv[c][k], sv[c][k + 1]);
+                    b = max3f(b, sv[c][k + 2], sv[c][k + 3]);
                 }
-            const float m_tile = mx * scale;
+                mx[c] = max3f(a, b, fmaxf(sv[c][30], sv[c][31]));
+            }
+            const float m_tile = max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * scale;
             const bool raise = (m_run == NEG_INF) || (m_tile > m_run + 8.f);
             if (__any_sync(0xffffffffu, raise)) {
                 const float m_new = raise ? fmaxf(m_run, m_tile) : m_run;
                 const float alpha = fast_exp2(m_run - m_new);   // 0 while nothing is summed
                 if (t > 0) {
                     // Rescale this row of O once the previous tile's product has landed.
-                    const int pt = t - 1;
-                    if (!flags[0] && !mbar_wait(bar_p_free + 8 * (pt & 1), (pt >> 1) & 1)) {
-                        flags[0] = 1;
-                        atomicOr(p.err, kErrWaitFull);
-                    }
+                    if (PL::kPSep)
+                        wait(pv_done, t - 1);
                     tmem_fence_after();
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         float ov[32];
-                        tmem_ld32_nowait(tmem + lane_base + PL::kColO + c * 32, ov);
+                        tmem_ld32_nowait(col_o + c * 32, ov);
                         tmem_wait_ld();
 #pragma unroll
                         for (int k = 0; k < 32; ++k)
                             ov[k] *= alpha;
-                        tmem_st32(tmem + lane_base + PL::kColO + c * 32, ov);
+                        tmem_st32(col_o + c * 32, ov);
                     }
-                    tmem_fence_before();
                 }
                 l_run *= alpha;
                 m_run = m_new;
             }
-            // P row, bf16, into the A-operand layout; the row sum takes the same rounding.
-            if (t >= 2 && !flags[0] &&
-                !mbar_wait(bar_p_free + 8 * (t & 1), ((t >> 1) & 1) ^ 1)) {
-                flags[0] = 1;
-                atomicOr(p.err, kErrWaitFull);
-            }
-            uint8_t *prow = smem + PL::kP + (t & 1) * PL::kPBytes + r * 128;
+            // The P buffer of the previous tile must have been read by its P V.
+            if (PL::kPSep && t > 0)
+                wait(pv_done, t - 1);
+            tmem_fence_after();
+            const float2 sc2 = make_float2(scale, scale);
+            const float2 nm2 = make_float2(-m_run, -m_run);
+            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                             make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int half = 0; half < 2; ++half) {
+                uint32_t w[32];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float p0 = fast_exp2(fmaf(sv[c][q * 8 + 2 * u], scale, -m_run));
-                        const float p1 = fast_exp2(fmaf(sv[c][q * 8 + 2 * u + 1], scale, -m_run));
-                        w[u] = pack_bf16x2(p0, p1);
-                        l_run += bf16_lo(w[u]) + bf16_hi(w[u]);
-                    }
-                    const int chunk = c * 4 + q;   // keys 8*chunk .. 8*chunk+7
-                    *reinterpret_cast<uint4 *>(prow + (chunk >> 3) * 16384 +
-                                               (((chunk & 7) ^ (r & 7)) << 4)) =
-                        make_uint4(w[0], w[1], w[2], w[3]);
+                for (int i = 0; i < 32; ++i) {
+                    const int c = half * 64 + 2 * i;   // keys c, c + 1
+                    const float2 x =
+                        __ffma2_rn(make_float2(sv[c >> 5][c & 31], sv[c >> 5][(c & 31) + 1]), sc2,
+                                   nm2);
+                    const float2 pr = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+                    acc[i & 3] = __fadd2_rn(acc[i & 3], pr);
+                    w[i] = pack_bf16x2(pr.x, pr.y);
                 }
+                tmem_st32_nowait(col_p + half * 32, w);
             }
-            if (diag && q0 + r >= S) {
+            const float2 s01 = __fadd2_rn(acc[0], acc[1]), s23 = __fadd2_rn(acc[2], acc[3]);
+            const float2 s4 = __fadd2_rn(s01, s23);
+            l_run += s4.x + s4.y;
+            tmem_wait_st();
+            if (diag && zero_v && q0 + r >= S) {
                 // Key q0 + r lies past the prompt: its V row may hold anything; zero it.
-                uint8_t *vrow = smem + PL::kRing + (t % ST) * PL::kStageBytes + PL::kTileBytes;
+                const int idx = 2 * t + 1;
+                wait(bar_full + 8 * (idx % R), idx / R);
+                uint8_t *vrow = smem + PL::kRing + (idx % R) * PL::kTileBytes;
 #pragma unroll
                 for (int c = 0; c < 8 * PL::kSub; ++c)
                     *reinterpret_cast<uint4 *>(vrow + (c >> 3) * 16384 + r * 128 +
                                                (((c & 7) ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                fence_proxy_async_smem();
             }
-            fence_proxy_async_smem();
+            tmem_fence_before();
             __syncwarp();
             if (lane == 0)
-                mbar_arrive(bar_p_ready + 8 * (t & 1));
+                mbar_arrive(p_ready);
         }
-        // ---------------- the block's output: o = O / l ----------------
-        if (!flags[0] && !mbar_wait(bar_o_ready, 0)) {
-            flags[0] = 1;
-            atomicOr(p.err, kErrWaitFull);
-        }
-        tmem_fence_after();
-        const float inv = fast_rcp(l_run);
-        const bool valid = q0 + r < S;
-        __nv_bfloat16 *orow =
-            p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
+        // ---------------- the tile's output: o = O / l ----------------
+        if (n_g > 0) {
+            wait(pv_done, n_g - 1);
+            tmem_fence_after();
+            const float inv = fast_rcp(l_run);
+            const bool valid = q0 + r < S;
+            __nv_bfloat16 *orow =
+                p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-            float ov[32];
-            tmem_ld32_nowait(tmem + lane_base + PL::kColO + c * 32, ov);
-            tmem_wait_ld();
-            if (valid && !flags[0]) {
+            for (int c = 0; c < D / 32; ++c) {
+                float ov[32];
+                tmem_ld32_nowait(col_o + c * 32, ov);
+                tmem_wait_ld();
+                if (valid && !flags[0]) {
 #pragma unroll
-                for (int k = 0; k < 32; k += 8)
-                    *reinterpret_cast<uint4 *>(orow + c * 32 + k) = make_uint4(
-                        pack_bf16x2(ov[k] * inv, ov[k + 1] * inv),
-                        pack_bf16x2(ov[k + 2] * inv, ov[k + 3] * inv),
-                        pack_bf16x2(ov[k + 4] * inv, ov[k + 5] * inv),
-                        pack_bf16x2(ov[k + 6] * inv, ov[k + 7] * inv));
+                    for (int k = 0; k < 32; k += 8)
+                        *reinterpret_cast<uint4 *>(orow + c * 32 + k) = make_uint4(
+                            pack_bf16x2(ov[k] * inv, ov[k + 1] * inv),
+                            pack_bf16x2(ov[k + 2] * inv, ov[k + 3] * inv),
+                            pack_bf16x2(ov[k + 4] * inv, ov[k + 5] * inv),
+                            pack_bf16x2(ov[k + 6] * inv, ov[k + 7] * inv));
+                }
             }
+            tmem_fence_before();
         }
-        tmem_fence_before();
+    } else {
+        setmaxnreg_dec<PL::kRegsLow>();   // warps 10-11: no role
     }
 
     __syncthreads();
@@ -405,7 +474,7 @@ cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtens
                            const PrefillParams &p, cudaStream_t stream)
 {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(p.n_items * p.h));
+    cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
     cfg.blockDim = dim3(static_cast<unsigned>(head_dim == 64 ? PrefillPlan<64>::kThreads
                                                              : PrefillPlan<128>::kThreads));
     cfg.dynamicSmemBytes = prefill_smem_bytes(head_dim);
