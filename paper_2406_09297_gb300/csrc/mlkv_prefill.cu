@@ -34,8 +34,8 @@
 // Warp roles (384 threads): warps 0-3 query tile A, 4-7 query tile B (softmax and output), warp 8
 // TMA producer (both query tiles, then K_0, V_0, K_1, V_1, ... through a ring), warp 9 MMA issuer,
 // warps 10-11 idle.  The block launches with 168 registers a thread (three warps per SM
-// sub-partition); the last warpgroup gives registers back (64) and the softmax warpgroups take
-// them (216): 128 * 64 + 256 * 216 <= 384 * 168.
+// sub-partition); the last warpgroup gives registers back (72 or 88) and the softmax warpgroups
+// take them (216 or 208, head_dim 64 or 128): 128 * low + 256 * high <= 384 * 168.
 // Every wait is bounded; on expiry the kernel records an error bit, stops, lets its copies and MMAs
 // land and frees its TMEM.
 #include "mlkv_device.cuh"
@@ -47,7 +47,8 @@ namespace {
 template <int D>
 struct PrefillPlan {
     static constexpr int kThreads = 12 * 32;
-    static constexpr int kRegsLaunch = 168, kRegsLow = 64, kRegsHigh = 216;
+    static constexpr int kRegsLaunch = 168;
+    static constexpr int kRegsLow = D == 64 ? 72 : 88, kRegsHigh = D == 64 ? 216 : 208;
     static constexpr int kProducer = 8, kMma = 9;
     static constexpr int kSub = D / 64;                      // 64-channel blocks of a row
     static constexpr int kTileBytes = 128 * D * 2;           // 128 rows of Q, K or V
@@ -208,72 +209,81 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         if (lane == 0) {
             constexpr uint32_t kIdS = umma_idesc(128, 128, 0, 0);
             constexpr uint32_t kIdPV = umma_idesc(128, D, 0, 1);
-            const int n[2] = {n_a, n_b};
+            constexpr uint32_t kSlot = PL::kTileBytes >> 4;   // one ring slot in descriptor units
+            // Descriptors of query tile A and of ring slot 0.  A tile, a slot, a K step or a
+            // 64-channel block only moves the start-address field (shared addresses < 256 KB), so
+            // each MMA's descriptors are one add away; the tensor core queues little, and any
+            // latency between two MMAs of this thread leaves it idle.
+            const uint64_t dq = umma_desc(sbase + PL::kQ, 16, 1024, kLayoutSw128);
+            const uint64_t dk = umma_desc(sbase + PL::kRing, 16, 1024, kLayoutSw128);
+            const uint64_t dv = umma_desc(sbase + PL::kRing, 16384, 1024, kLayoutSw128);
             bool ok = true;
             auto wait = [&](uint32_t bar, int parity) {
-                if (ok && (flags[0] || !mbar_wait(bar, static_cast<uint32_t>(parity) & 1u)))
+                const uint32_t par = static_cast<uint32_t>(parity) & 1u;
+                if (ok && !mbar_test_wait(bar, par) && !mbar_wait(bar, par))
                     ok = false;
                 return ok;
             };
-            auto ring = [&](int idx) { return sbase + PL::kRing + (idx % R) * PL::kTileBytes; };
             auto tile_full = [&](int idx) { return wait(bar_full + 8 * (idx % R), idx / R); };
             auto issue_s = [&](int g, int t) {
-                const uint32_t qt = sbase + PL::kQ + g * PL::kTileBytes;
-                const uint32_t kt = ring(2 * t);
+                const uint64_t qa = dq + g * kSlot;
+                const uint64_t kb = dk + ((2 * t) % R) * kSlot;
 #pragma unroll
-                for (int k = 0; k < D / 16; ++k)
-                    umma_f16(tmem + PL::kColS + 128 * g,
-                             umma_desc(qt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
-                                       kLayoutSw128),
-                             umma_desc(kt + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024,
-                                       kLayoutSw128),
-                             kIdS, k > 0 ? 1 : 0);
+                for (int k = 0; k < D / 16; ++k) {
+                    const uint32_t off = (k >> 2) * 1024 + (k & 3) * 2;   // 16384 B, 32 B
+                    umma_f16(tmem + PL::kColS + 128 * g, qa + off, kb + off, kIdS, k > 0 ? 1 : 0);
+                }
                 umma_commit(bar_s_ready + 8 * g);
             };
-            auto issue_pv = [&](int g, int t) {
-                const uint32_t vt = ring(2 * t + 1);
+            auto issue_pv = [&](int g, int t, bool last) {
+                const uint64_t vb = dv + ((2 * t + 1) % R) * kSlot;
                 const uint32_t pc = tmem + (PL::kPSep ? PL::kColP + 64 * g : PL::kColS + 128 * g);
 #pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    umma_f16_ts(tmem + PL::kColO + D * g, pc + 8 * k,
-                                umma_desc(vt + k * 2048, 16384, 1024, kLayoutSw128), kIdPV,
+                for (int k = 0; k < 8; ++k)   // 16 keys = 2048 B of V, 8 TMEM columns of P
+                    umma_f16_ts(tmem + PL::kColO + D * g, pc + 8 * k, vb + k * 128, kIdPV,
                                 (t > 0 || k > 0) ? 1 : 0);
-                umma_commit(bar_pv_done + 8 * g);
+                // With P over S, the next S's completion already implies this product's.
+                if (PL::kPSep || last)
+                    umma_commit(bar_pv_done + 8 * g);
             };
             if (wait(bar_q, 0) && tile_full(0)) {
                 tmem_fence_after();
-                for (int g = 0; g < 2; ++g)
-                    if (n[g] > 0)
-                        issue_s(g, 0);
-                umma_commit(bar_empty);   // K_0 (ring slot 0)
+                if (n_a > 0)
+                    issue_s(0, 0);
+                issue_s(1, 0);
             }
+            // Ring slots are released by tile B's softmax warps (they see every MMA that read them
+            // complete), not by commits: a commit costs the tensor pipe about as much as a short MMA.
             for (int t = 0; ok && t < n_b; ++t) {
-                for (int g = 0; g < 2 && ok; ++g) {
-                    if (t >= n[g])
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    const int ng = g ? n_b : n_a;
+                    if (!ok || t >= ng)
                         continue;
-                    const bool next = t + 1 < n[g];
-                    if (PL::kPSep && next) {
+                    const bool next = t + 1 < ng;
+                    if (PL::kPSep) {
                         // S of the next tile as soon as this one's S has been read.
-                        if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
+                        if (next) {
+                            if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
+                                break;
+                            tmem_fence_after();
+                            issue_s(g, t + 1);
+                        }
+                        if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
                             break;
                         tmem_fence_after();
-                        issue_s(g, t + 1);
-                    }
-                    if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
-                        break;
-                    tmem_fence_after();
-                    issue_pv(g, t);
-                    if (!PL::kPSep && next) {
-                        if (!tile_full(2 * t + 2))
+                        issue_pv(g, t, !next);
+                    } else {
+                        // Everything first, then P V and the next S back to back.
+                        if (!tile_full(2 * t + 1) || (next && !tile_full(2 * t + 2)) ||
+                            !wait(bar_p_ready + 8 * g, t))
                             break;
-                        issue_s(g, t + 1);
+                        tmem_fence_after();
+                        issue_pv(g, t, !next);
+                        if (next)
+                            issue_s(g, t + 1);
                     }
                 }
-                if (!ok)
-                    break;
-                umma_commit(bar_empty + 8 * ((2 * t + 1) % R));       // V_t, read by both
-                if (t + 1 < n_b)
-                    umma_commit(bar_empty + 8 * ((2 * t + 2) % R));   // K_{t+1}, read by both
             }
             if (!ok) {
                 flags[0] = 1;
@@ -312,6 +322,15 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         float m_run = NEG_INF, l_run = 0.f;
         for (int t = 0; t < n_g; ++t) {
             wait(s_ready, t);
+            // Tile B's first warp frees ring slots whose readers have all completed: K_0 once S_B(0)
+            // is done; V_{t-1} and K_t once S_B(t) (P over S) or P_B V_{t-1} (own P) is done.
+            const bool releaser = grp == 1 && warp == 4 && lane == 0;
+            if (releaser && t == 0)
+                mbar_arrive(bar_empty);
+            if (releaser && t > 0 && !PL::kPSep) {
+                mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
+                mbar_arrive(bar_empty + 8 * ((2 * t) % R));
+            }
             tmem_fence_after();
             float sv[4][32];
 #pragma unroll
@@ -370,8 +389,13 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 m_run = m_new;
             }
             // The P buffer of the previous tile must have been read by its P V.
-            if (PL::kPSep && t > 0)
+            if (PL::kPSep && t > 0) {
                 wait(pv_done, t - 1);
+                if (releaser) {
+                    mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
+                    mbar_arrive(bar_empty + 8 * ((2 * t) % R));
+                }
+            }
             tmem_fence_after();
             const float2 sc2 = make_float2(scale, scale);
             const float2 nm2 = make_float2(-m_run, -m_run);
@@ -414,7 +438,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         }
         // ---------------- the tile's output: o = O / l ----------------
         if (n_g > 0) {
-            wait(pv_done, n_g - 1);
+            wait(pv_done, PL::kPSep ? n_g - 1 : 0);   // with P over S only the last P V commits
             tmem_fence_after();
             const float inv = fast_rcp(l_run);
             const bool valid = q0 + r < S;
