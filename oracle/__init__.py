@@ -46,6 +46,11 @@ def load(path):
     L.oracle_append.argtypes = [
         ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, ctypes.c_int, _ip,
         ctypes.c_int, _dp, _dp, ctypes.POINTER(_dp), ctypes.POINTER(_dp)]
+    L.oracle_merge_kv.argtypes = [ctypes.c_int, _ip, ctypes.c_int, ctypes.c_int, ctypes.c_longlong,
+                                  _dp, _dp]
+    L.oracle_bf16_rne.argtypes = [ctypes.c_double]
+    L.oracle_bf16_rne.restype = ctypes.c_uint
+    L.oracle_bf16_rne_array.argtypes = [_dp, ctypes.c_longlong, ctypes.POINTER(ctypes.c_uint16)]
     return L
 
 
@@ -203,4 +208,28 @@ def decode_layer(layer, owner, h, g, d, seq_lens, Q, K_owner, V_owner, nthreads=
                                    qp, karr, varr, out.ctypes.data_as(_dp), nthreads)
     if rc != ORACLE_OK:
         raise ValueError(f"oracle_decode_layer failed ({rc})")
+    return out
+
+
+def merge_kv(owner, h, g, W):
+    """Sec. 4.2 KV-weight merge: W [l][h][row] float64 -> [m][g][row] float64 means (owner order)."""
+    owner, op = _ints(owner)
+    W, wp = _f64(W)
+    l, h_, row = W.shape
+    assert h_ == h and l == len(owner)
+    m, _ = slots(owner)
+    if m < 1:
+        raise ValueError(f"invalid owner map ({m})")
+    out = np.zeros((m, g, row), dtype=np.float64)
+    rc = lib().oracle_merge_kv(l, op, h, g, row, wp, out.ctypes.data_as(_dp))
+    if rc != ORACLE_OK:
+        raise ValueError(f"oracle_merge_kv failed ({rc})")
+    return out
+
+
+def bf16_rne(x):
+    """Round-to-nearest-even of float64 values to bfloat16; returns the uint16 bit patterns."""
+    x, xp = _f64(x)
+    out = np.zeros(x.shape, dtype=np.uint16)
+    lib().oracle_bf16_rne_array(xp, x.size, out.ctypes.data_as(ctypes.POINTER(ctypes.c_uint16)))
     return out

@@ -1,5 +1,5 @@
 /*
- * MLKV decode- and prefill-attention oracle.
+ * MLKV decode- and prefill-attention oracle, and the KV-weight merge of the model conversion.
  *
  * TEST INFRASTRUCTURE ONLY.  This file states, in plain double-precision C, what the MLKV decode
  * path computes, so that the CUDA library can be checked against it.  Only the test suite,
@@ -380,4 +380,84 @@ int oracle_append(int layer, int l, const int *owner, int g, int d, int b, const
         }
     }
     return 1;
+}
+
+/* ------------------------------------------------------------------------------------------- */
+/* KV-weight merging (Sec. 4.2)                                                                  */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Sec. 4.2: the variants are converted from the MHA baseline by merging KV-head weights by
+ * averaging (the method the GQA paper found best): the heads of one group of a layer, and the
+ * heads of the later layers of a block, which have no KV heads of their own, become one KV head.
+ * Merged head j of owner layer o = the mean, over every layer n with owner[n] == o and every head
+ * i of group j (Eq. 12: i / (h/g) == j, 0-based), of W[n][i][:].
+ * W: [l][h][row] (per head, one projection's rows: head_dim x d_model, or head_dim for a bias);
+ * out: [m][g][row], owners in increasing layer order (the slots of oracle_slots).  The sum is
+ * taken in double precision in member order, then divided by the member count. */
+int oracle_merge_kv(int l, const int *owner, int h, int g, long long row, const double *W,
+                    double *out)
+{
+    if (row <= 0 || W == NULL || out == NULL)
+        return ORACLE_ERR_ARG;
+    int rc = oracle_validate(l, owner, h, g, 1);
+    if (rc != ORACLE_OK)
+        return rc;
+    const int G = h / g;
+    int s = 0;   /* slot of the current owner */
+    for (int o = 0; o < l; ++o) {
+        if (owner[o] != o)
+            continue;
+        for (int j = 0; j < g; ++j) {
+            double *dst = out + ((size_t)s * g + j) * (size_t)row;
+            for (long long r = 0; r < row; ++r) {
+                double sum = 0.0;
+                long long count = 0;
+                for (int n = 0; n < l; ++n) {
+                    if (owner[n] != o)
+                        continue;
+                    for (int i = j * G; i < (j + 1) * G; ++i) {
+                        sum += W[((size_t)n * h + i) * (size_t)row + (size_t)r];
+                        ++count;
+                    }
+                }
+                dst[r] = sum / (double)count;
+            }
+        }
+        ++s;
+    }
+    return ORACLE_OK;
+}
+
+/* bfloat16 (1 sign, 8 exponent, 7 stored significand bits) nearest to x, ties to the even
+ * significand; beyond the largest finite value by half a unit in the last place or more,
+ * infinity.  Written from the definition: scale |x| by its quantum (2^(e-7) for |x| in [2^e,
+ * 2^(e+1)), at least 2^-133, the subnormal quantum), round to an integer half-to-even (rint in the
+ * default rounding mode), scale back.  Returns the 16-bit pattern. */
+unsigned oracle_bf16_rne(double x)
+{
+    const unsigned sign = signbit(x) ? 0x8000u : 0u;
+    if (isnan(x))
+        return sign | 0x7FC0u;
+    const double a = fabs(x);
+    if (a == 0.0)
+        return sign;
+    int e;
+    (void)frexp(a, &e);            /* a = f 2^e, f in [0.5, 1): a in [2^(e-1), 2^e) */
+    int q = (e - 1) - 7;           /* 8 significant bits */
+    if (q < -133)
+        q = -133;
+    const double k = rint(ldexp(a, -q));   /* exact scaling, then half-to-even */
+    const double v = ldexp(k, q);
+    if (v > 0x1.FEp127)            /* largest finite bfloat16: (2 - 2^-7) 2^127 */
+        return sign | 0x7F80u;
+    const float f = (float)v;      /* exact: at most 8 significant bits, inside float's range */
+    uint32_t bits;
+    memcpy(&bits, &f, sizeof bits);
+    return sign | ((bits >> 16) & 0x7FFFu);
+}
+
+void oracle_bf16_rne_array(const double *x, long long n, uint16_t *out)
+{
+    for (long long k = 0; k < n; ++k)
+        out[k] = (uint16_t)oracle_bf16_rne(x[k]);
 }

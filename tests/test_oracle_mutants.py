@@ -2,7 +2,9 @@
 test_oracle_pins.py rejects every one of them: a dropped scale, a wrong group map, a block map
 that picks the wrong layer, an off-by-one visible length, a missing normalisation, a flipped sign,
 a wrong query row, a dropped factor in the cache size, a mis-numbered slot, a misplaced append,
-a prefill row that does not see its own position and prefill queries read head-major.
+a prefill row that does not see its own position, prefill queries read head-major, a merge that
+drops the block's later layers, picks heads by a modulo group, sums without dividing, and a
+bfloat16 rounding that truncates or rounds ties away from zero.
 """
 import os
 import subprocess
@@ -30,6 +32,12 @@ MUTANTS = [
      "int L = t > 0 ? t : 1;"),
     ("prefill-head-major-rows", "const double *q = jb->Q + (((size_t)beta * jb->s_max + t) * h + i) * d;",
      "const double *q = jb->Q + (((size_t)beta * h + i) * jb->s_max + t) * d;"),
+    ("merge-owner-only", "                    if (owner[n] != o)\n                        continue;\n                    for (int i = j * G;",
+     "                    if (n != o)\n                        continue;\n                    for (int i = j * G;"),
+    ("merge-group-modulo", "for (int i = j * G; i < (j + 1) * G; ++i) {", "for (int i = j; i < h; i += g) {"),
+    ("merge-sum-not-mean", "dst[r] = sum / (double)count;", "dst[r] = sum;"),
+    ("bf16-truncates", "const double k = rint(ldexp(a, -q));", "const double k = trunc(ldexp(a, -q));"),
+    ("bf16-ties-away", "const double k = rint(ldexp(a, -q));", "const double k = round(ldexp(a, -q));"),
 ]
 
 PIN_TESTS = [
@@ -47,6 +55,14 @@ PIN_TESTS = [
     pins.test_append_only_for_owner_layers,
     lambda: [pins.test_prefill_matches_causal_sdpa(*m) for m in pins.MAPS],
     pins.test_prefill_first_position_returns_value_row,
+    pins.test_merge_identity_map_returns_input,
+    lambda: [pins.test_merge_linear_closed_form(*c) for c in
+             [([0, 0, 0, 3, 3, 3], 12, 4), ([0, 0, 2, 2, 4, 4, 6, 6], 8, 1),
+              ([0, 0, 0, 0, 4, 5, 5], 6, 3)]],
+    pins.test_merge_permutation_invariance_and_locality,
+    pins.test_bf16_rne_matches_torch_on_float32_values,
+    pins.test_bf16_rne_brute_force_on_float64_values,
+    pins.test_bf16_rne_worked_cases,
 ]
 
 

@@ -10,6 +10,12 @@
 * Brute force on tiny inputs in 50-digit decimal arithmetic, without max subtraction.
 * Prefill: torch's scaled_dot_product_attention with its causal mask, in float64, per prompt; the
   first prompt position returns its value row; MLKV prefill equals MHA prefill on duplicated K/V.
+* KV-weight merge (Sec. 4.2): the identity map returns its input; a weight linear in (layer,
+  head, element) merges to the closed form at the block's and group's mean layer and head;
+  members permuted inside a block or group change nothing; blocks do not see each other.
+* bfloat16 rounding: torch's float32 -> bfloat16 conversion (round to nearest even) on float32
+  values, a brute-force nearest value over all 65,536 patterns on float64 values, and worked ties,
+  subnormals and overflow.
 """
 import decimal
 import os
@@ -363,3 +369,111 @@ def test_prefill_mlkv_equals_mha_on_duplicated_kv():
             mha.V[n][:, i] = c.V[owner[n]][:, i // G]
     for n in range(4):
         assert np.array_equal(c.prefill(n, Q[n], prompt_lens), mha.prefill(n, Q[n], prompt_lens))
+
+
+# ----------------------------------------------------------------------------------------------
+# KV-weight merge (Sec. 4.2) and bfloat16 rounding
+# ----------------------------------------------------------------------------------------------
+
+def test_merge_identity_map_returns_input():
+    # Every layer its own owner and g = h: every merged head has one member, itself.
+    rng = np.random.default_rng(31)
+    W = rng.standard_normal((5, 6, 40))
+    np.testing.assert_array_equal(oracle.merge_kv(list(range(5)), 6, 6, W), W)
+
+
+def _linear_weights(l, h, row):
+    n = np.arange(l, dtype=np.float64)[:, None, None]
+    i = np.arange(h, dtype=np.float64)[None, :, None]
+    r = np.arange(row, dtype=np.float64)[None, None, :]
+    return 1000.0 * n + 10.0 * i + 0.25 * r
+
+
+@pytest.mark.parametrize("owner,h,g", [
+    ([0, 0, 0, 3, 3, 3], 12, 4),          # Eq. 18 blocks of 3, GQA-4 inside
+    ([0, 0, 2, 2, 4, 4, 6, 6], 8, 1),     # blocks of 2, one KV head
+    ([0, 0, 0, 0, 4, 5, 5], 6, 3),        # blocks of 4, 1 and 2
+])
+def test_merge_linear_closed_form(owner, h, g):
+    # W = 1000 n + 10 i + r/4 is linear, so its mean over a block B and a group J is
+    # 1000 mean(B) + 10 mean(J) + r/4, with mean(J) = jG + (G-1)/2 for the contiguous group of Eq. 12.
+    l, row, G = len(owner), 7, h // g
+    out = oracle.merge_kv(owner, h, g, _linear_weights(l, h, row))
+    owners = sorted(set(owner))
+    for s_, o in enumerate(owners):
+        block = [n for n in range(l) if owner[n] == o]
+        for j in range(g):
+            expect = 1000.0 * (sum(block) / len(block)) + 10.0 * (j * G + (G - 1) / 2) + \
+                0.25 * np.arange(row)
+            np.testing.assert_allclose(out[s_, j], expect, rtol=0, atol=1e-9)
+
+
+def test_merge_permutation_invariance_and_locality():
+    owner, h, g = [0, 0, 0, 3, 3], 8, 2
+    rng = np.random.default_rng(32)
+    W = rng.standard_normal((5, 8, 16))
+    base = oracle.merge_kv(owner, h, g, W)
+    P = W.copy()
+    P[[0, 1, 2]] = W[[2, 0, 1]]                 # layers permuted inside block 0
+    P[:, [4, 5, 6, 7]] = W[:, [7, 5, 4, 6]]     # heads permuted inside group 1
+    np.testing.assert_allclose(oracle.merge_kv(owner, h, g, P), base, rtol=0, atol=1e-12)
+    Q = W.copy()
+    Q[3:] += 5.0                                # block 1 changes, block 0 does not see it
+    out = oracle.merge_kv(owner, h, g, Q)
+    np.testing.assert_array_equal(out[0], base[0])
+    np.testing.assert_allclose(out[1], base[1] + 5.0, rtol=0, atol=1e-12)
+
+
+def test_bf16_rne_matches_torch_on_float32_values():
+    rng = np.random.default_rng(33)
+    x = np.concatenate([
+        rng.standard_normal(20000).astype(np.float32),
+        (rng.standard_normal(5000) * 1e-39).astype(np.float32),      # float32 / bf16 subnormals
+        (rng.standard_normal(5000) * 3e38).astype(np.float32),       # near overflow
+        np.array([0.0, -0.0, 1.0, -1.0, 3.3895314e38, 3.4e38], dtype=np.float32),
+    ])
+    x = x[np.isfinite(x)]
+    ref = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(oracle.bf16_rne(x.astype(np.float64)), ref)
+
+
+def _all_bf16_values():
+    bits = np.arange(65536, dtype=np.uint32)
+    f = (bits << 16).astype(np.uint32).view(np.float32).astype(np.float64)
+    ok = np.isfinite(f)
+    return bits[ok].astype(np.uint16), f[ok]
+
+
+def test_bf16_rne_brute_force_on_float64_values():
+    bits, vals = _all_bf16_values()
+    order = np.argsort(vals, kind="stable")
+    bits, vals = bits[order], vals[order]
+    rng = np.random.default_rng(34)
+    x = np.concatenate([rng.standard_normal(300) * 10.0 ** rng.integers(-40, 38, 300),
+                        rng.uniform(-3.0, 3.0, 300)])
+    got = oracle.bf16_rne(x)
+    for xv, gb in zip(x, got):
+        d = np.abs(vals - xv)
+        best = np.flatnonzero(d == d.min())
+        cands = [int(bits[k]) for k in best if not (vals[k] == 0.0 and bits[k] == 0x8000)]
+        if len(cands) > 1:     # a tie: the even significand
+            cands = [c for c in cands if c % 2 == 0]
+        if xv < 0 and vals[best[0]] == 0.0:
+            cands = [0x8000]
+        assert int(gb) == cands[0], (xv, hex(int(gb)), [hex(c) for c in cands])
+
+
+def test_bf16_rne_worked_cases():
+    cases = [
+        (1.0, 0x3F80), (1.0 + 2.0 ** -8, 0x3F80),           # tie, even stays
+        (1.0 + 3 * 2.0 ** -8, 0x3F82),                       # tie, rounds up to even
+        (1.0 + 2.0 ** -8 + 2.0 ** -40, 0x3F81),              # just above the tie
+        (-0.0, 0x8000), (0.0, 0x0000),
+        (2.0 ** -133, 0x0001), (2.0 ** -134, 0x0000),        # smallest subnormal; tie to 0
+        (3 * 2.0 ** -134, 0x0002), (-(2.0 ** -126), 0x8080),
+        ((2 - 2.0 ** -7) * 2.0 ** 127, 0x7F7F),              # largest finite
+        ((2 - 2.0 ** -8) * 2.0 ** 127, 0x7F80),              # tie at the top: overflows
+        (1e300, 0x7F80), (-1e300, 0xFF80),
+    ]
+    for x, want in cases:
+        assert int(oracle.bf16_rne(np.array([x]))[0]) == want, (x, want)
