@@ -556,6 +556,71 @@ def run_prefill(args, w):
     print(json.dumps(line), flush=True)
 
 
+def _hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def run_merge(args, w):
+    """Sec. 4.2 conversion of the workload's model: its MHA K and V projections (l x h heads, each
+    head_dim x d_model, d_model = h * head_dim, seeded bf16) merged by averaging into the owner
+    map's m x g KV heads, one mlkv_merge_kv_weights per projection; L2 flushed before each
+    repetition.  HBM-bound: algorithmic bytes = inputs read once + outputs written once."""
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device, gen
+
+    torch.cuda.set_device(0)
+    row = w.d * w.h * w.d
+    m = len(w.owners())
+    Ws, outs = [], []
+    for kv in range(2):
+        W = torch.empty((w.l, w.h, row), dtype=torch.bfloat16, device="cuda")
+        for n in range(w.l):
+            device.fill_(W[n], w.seed + 7, gen.TID_W + 64 * kv + n, 0.02)
+        Ws.append(W)
+        outs.append(torch.empty((m, w.g, row), dtype=torch.bfloat16, device="cuda"))
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for kv in range(2):
+            mlkv.mlkv_merge_kv_weights(w.owner, w.h, w.g, Ws[kv], outs[kv], stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    times = []
+    with Clocks(0) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    nbytes = 2 * 2 * (w.l * w.h + m * w.g) * row
+    gbs = nbytes / (ms / 1e3) / 1e9
+    peak, kind = _hbm_peak()
+    line = {"metric": "KV-weight merge GB/s (K and V projections)", "value": gbs, "unit": "GB/s",
+            "higher_is_better": True, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "layers": w.l, "q_heads": w.h, "head_dim": w.d,
+                       "d_model": w.h * w.d, "layer_owner": list(w.owner), "kv_heads_per_owner": w.g,
+                       "l2": "flushed before every timed repetition"},
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s",
+                         "frac": gbs / peak, "peak_source": kind, "kernel": "merge_kernel",
+                         "alg_bytes_per_step": nbytes, "launches_per_step": 2},
+            "clocks": clocks.summary()}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -578,6 +643,8 @@ def main():
                     help="prefill throughput of the --config model (prompt of --prefill-len)")
     ap.add_argument("--prefill-batch", type=int, default=8)
     ap.add_argument("--prefill-len", type=int, default=2048)
+    ap.add_argument("--merge", action="store_true",
+                    help="Sec. 4.2 KV-weight merge of the --config model's K and V projections")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.loop:
@@ -586,6 +653,10 @@ def main():
     if args.prefill:
         from mlkv_synth import workloads
         run_prefill(args, workloads.by_name(args.config))
+        return
+    if args.merge:
+        from mlkv_synth import workloads
+        run_merge(args, workloads.by_name(args.config))
         return
 
     from mlkv_synth import workloads

@@ -257,6 +257,33 @@ int mlkv_decode_attention_static(const void *kv_slot, int batch, int n_q_heads, 
                                  int head_dim, int max_seq, const void *Q, void *out,
                                  const int *seq_lens, void *cuda_stream);
 
+/*
+ * mlkv_merge_kv_weights - converts one MHA projection (K or V) to MLKV by averaging (Sec. 4.2:
+ * "KV heads in the same group of the same layer, as well as the heads from subsequent layers which
+ * do not have KV heads of their own, are merged by averaging"): merged KV head j of owner layer o
+ * is the mean, over every layer n with layer_owner[n] == o and every query head i of group j
+ * (Eq. 12: i / (n_q_heads / n_kv_heads) == j), of W[n][i][:], rounded to bf16 (nearest, ties to
+ * even).  The sums are carried as pairs of floats with exact per-addition errors, so the result
+ * is the bf16 nearest to the exact mean unless that mean lies within about count^2 * 2^-48
+ * (relative) of a rounding boundary (count = members of the head), provided each column's sum
+ * of magnitudes stays below FLT_MAX (about 3.4e38).  Needs no cache.
+ *
+ *   layer_owner  host int32[n_layers]: owner[n] <= n and owner[owner[n]] == owner[n] (Eq. 18 or
+ *                any such map; the identity map with n_kv_heads < n_q_heads is the GQA conversion)
+ *   n_q_heads    heads per layer of the MHA model (h); n_kv_heads (g) must divide it
+ *   row_elems    elements of one head's rows: head_dim * d_model for a weight, head_dim for a bias;
+ *                a positive multiple of 8
+ *   W            device bf16 [n_layers][n_q_heads][row_elems], 16-byte aligned, read only
+ *   W_merged     device bf16 [m][n_kv_heads][row_elems], m = owner layers, in increasing layer
+ *                order (the slot order of mlkv_owner_slot); 16-byte aligned; must not overlap W
+ *   cuda_stream  the stream the kernel is queued on (asynchronous; nothing is allocated)
+ * Errors: MLKV_ERR_INVALID_ARG (null or unaligned pointers, sizes, overlap), MLKV_ERR_MAP (owner
+ * map, g not dividing h), MLKV_ERR_UNSUPPORTED (more than 1024 layers or 65535 merged heads),
+ * MLKV_ERR_CUDA.
+ */
+int mlkv_merge_kv_weights(const int *layer_owner, int n_layers, int n_q_heads, int n_kv_heads,
+                          int64_t row_elems, const void *W, void *W_merged, void *cuda_stream);
+
 /* Library version, major*10000 + minor*100 + patch. */
 int mlkv_version(void);
 

@@ -40,6 +40,7 @@ TID_Q = 0x100      # + layer          rows: beta,          cols: i*d + e
 TID_K = 0x200      # + owner layer    rows: beta*g + j,    cols: t*d + e
 TID_V = 0x300      # + owner layer    rows: beta*g + j,    cols: t*d + e
 TID_LEN = 0x400    #                  output n = beta: sequence length draw
+TID_W = 0x500      # + layer          rows: head i,        cols: element of the head's rows
 
 
 def mix64_int(z):

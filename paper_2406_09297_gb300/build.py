@@ -19,8 +19,8 @@ NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc" if os.path.exists(
     "/usr/local/cuda/bin/nvcc") else "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
-SOURCES = ["mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_prefill.cu", "mlkv_host.cpp",
-           "mlkv_noalloc.cu"]
+SOURCES = ["mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_prefill.cu", "mlkv_merge.cu",
+           "mlkv_host.cpp", "mlkv_noalloc.cu"]
 
 
 def _sources():

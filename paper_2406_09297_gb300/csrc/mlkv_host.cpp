@@ -872,6 +872,64 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
     return MLKV_OK;
 }
 
+int mlkv_merge_kv_weights(const int *layer_owner, int n_layers, int n_q_heads, int n_kv_heads,
+                          int64_t row_elems, const void *W, void *W_merged, void *cuda_stream)
+{
+    if (layer_owner == nullptr || W == nullptr || W_merged == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "layer_owner, W and W_merged must be non-NULL");
+    if (n_layers < 1 || n_q_heads < 1 || n_kv_heads < 1)
+        return fail(MLKV_ERR_INVALID_ARG, "sizes must be positive (l=%d h=%d g=%d)", n_layers,
+                    n_q_heads, n_kv_heads);
+    if (n_layers > mlkv::kMergeMaxLayers)
+        return fail(MLKV_ERR_UNSUPPORTED, "%d layers exceed %d", n_layers, mlkv::kMergeMaxLayers);
+    if (row_elems < 8 || row_elems % 8 != 0 || !aligned16(W) || !aligned16(W_merged))
+        return fail(MLKV_ERR_INVALID_ARG,
+                    "row_elems (%lld) must be a positive multiple of 8 and W, W_merged 16-byte "
+                    "aligned", static_cast<long long>(row_elems));
+    if (n_kv_heads > n_q_heads || n_q_heads % n_kv_heads != 0)
+        return fail(MLKV_ERR_MAP, "n_kv_heads %d must divide n_q_heads %d", n_kv_heads, n_q_heads);
+    static thread_local mlkv::MergeParams p;
+    int m = 0;
+    for (int n = 0; n < n_layers; ++n) {
+        const int o = layer_owner[n];
+        if (o < 0 || o > n || layer_owner[o] != o)
+            return fail(MLKV_ERR_MAP, "layer_owner[%d] = %d is not a layer <= %d that owns itself",
+                        n, o, n);
+        if (o == n)
+            ++m;
+    }
+    if (static_cast<long long>(m) * n_kv_heads > 65535)
+        return fail(MLKV_ERR_UNSUPPORTED, "%d owners x %d KV heads exceed 65535 merged heads", m,
+                    n_kv_heads);
+    // Sec. 4.2: the members of owner o are the layers of its block, in layer order.
+    int k = 0, sidx = 0;
+    for (int o = 0; o < n_layers; ++o) {
+        if (layer_owner[o] != o)
+            continue;
+        p.slot_begin[sidx++] = k;
+        for (int n = o; n < n_layers; ++n)
+            if (layer_owner[n] == o)
+                p.member[k++] = n;
+    }
+    p.slot_begin[sidx] = k;
+    const size_t in_bytes = static_cast<size_t>(n_layers) * n_q_heads * row_elems * 2;
+    const size_t out_bytes = static_cast<size_t>(m) * n_kv_heads * row_elems * 2;
+    const char *wi = static_cast<const char *>(W);
+    const char *wo = static_cast<const char *>(W_merged);
+    if (wo < wi + in_bytes && wi < wo + out_bytes)
+        return fail(MLKV_ERR_INVALID_ARG, "W_merged overlaps W");
+    p.W = static_cast<const __nv_bfloat16 *>(W);
+    p.out = static_cast<__nv_bfloat16 *>(W_merged);
+    p.row = row_elems;
+    p.h = n_q_heads;
+    p.g = n_kv_heads;
+    p.G = n_q_heads / n_kv_heads;
+    cudaError_t e = mlkv::launch_merge(p, m, static_cast<cudaStream_t>(cuda_stream));
+    if (e != cudaSuccess)
+        return fail_cuda(e, "merge launch");
+    return MLKV_OK;
+}
+
 int64_t mlkv_cache_bytes(mlkv_cache_t c)
 {
     if (c == nullptr)

@@ -72,6 +72,18 @@ cudaError_t prepare_prefill(int head_dim);
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream);
 
+// KV-weight merge (mlkv_merge.cu).  Passed by value.
+constexpr int kMergeMaxLayers = 1024;
+struct MergeParams {
+    const __nv_bfloat16 *W;   // [l][h][row]
+    __nv_bfloat16 *out;       // [m][g][row], owners in increasing layer order
+    long long row;            // elements per head row block, a multiple of 8
+    int h, g, G;
+    int slot_begin[kMergeMaxLayers + 1];   // members of slot s: member[slot_begin[s] .. [s+1])
+    int member[kMergeMaxLayers];           // layers grouped by slot
+};
+cudaError_t launch_merge(const MergeParams &p, int n_slots, cudaStream_t stream);
+
 struct AppendParams {
     const __nv_bfloat16 *K;   // [b][g][D]
     const __nv_bfloat16 *V;

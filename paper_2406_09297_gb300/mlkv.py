@@ -30,6 +30,7 @@ EXPORTED = [
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
+    "mlkv_merge_kv_weights",
 ]
 
 
@@ -68,6 +69,7 @@ def _load():
     L.mlkv_version.argtypes = []
     L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
     L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
+    L.mlkv_merge_kv_weights.argtypes = [ip, ci, ci, ci, i64, vp, vp, vp]
     return L
 
 
@@ -211,6 +213,15 @@ def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, 
     return _check(lib.mlkv_decode_attention_static(
         ctypes.c_void_p(kv_slot), batch, n_q_heads, kv_heads, head_dim, max_seq, _ptr(Q),
         _ptr(out), p, _stream(stream)))
+
+
+def mlkv_merge_kv_weights(layer_owner, n_q_heads, n_kv_heads, W, out, stream=None):
+    """Sec. 4.2 merge of one projection: W bf16 [l][h][row] -> out bf16 [m][g][row] (device)."""
+    owner = np.ascontiguousarray(np.asarray(layer_owner, dtype=np.int32))
+    row = W.numel() // (len(owner) * n_q_heads) if W is not None else 0
+    return _check(lib.mlkv_merge_kv_weights(
+        owner.ctypes.data_as(ctypes.POINTER(ctypes.c_int)), len(owner), n_q_heads, n_kv_heads,
+        row, _ptr(W), _ptr(out), _stream(stream)))
 
 
 class MLKVCache:
