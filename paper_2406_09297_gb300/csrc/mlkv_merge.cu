@@ -111,20 +111,35 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
 #pragma unroll
         for (int c = 0; c < 4; ++c)
             hi[c] = lo[c] = make_float2(0.f, 0.f);
-        if (v < nvec) {
-            auto src = [&](int mi) {
-                const int layer = p.member[b0 + mi / p.G];
-                const int head = j * p.G + mi % p.G;
-                return reinterpret_cast<const uint4 *>(
-                    p.W + (static_cast<size_t>(layer) * p.h + head) * head_stride +
-                    static_cast<size_t>(v) * 8);
+        if (v < nvec && m0 < m1) {
+            // Members in order: heads j*G .. j*G+G-1 of each layer of the block.  Walk them with a
+            // pointer and a head counter (no division per load).
+            const size_t col = static_cast<size_t>(v) * 8;
+            int lk = m0 / p.G;                   // member layer index
+            int hk = m0 - lk * p.G;              // head within the group
+            auto layer_ptr = [&](int k) {
+                return p.W + (static_cast<size_t>(p.member[b0 + k]) * p.h +
+                              static_cast<size_t>(j) * p.G) * head_stride + col;
+            };
+            const __nv_bfloat16 *ptr = layer_ptr(lk) + hk * head_stride;
+            auto next = [&]() {
+                const __nv_bfloat16 *cur = ptr;
+                if (++hk == p.G) {
+                    hk = 0;
+                    ++lk;
+                    if (b0 + lk < p.slot_begin[s + 1])
+                        ptr = layer_ptr(lk);
+                } else {
+                    ptr += head_stride;
+                }
+                return reinterpret_cast<const uint4 *>(cur);
             };
             int mi = m0;
             for (; mi + 4 <= m1; mi += 4) {
                 uint4 w[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u)   // four loads in flight before any addition
-                    w[u] = __ldcs(src(mi + u));
+                    w[u] = __ldcs(next());
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     acc_add2(hi[0], lo[0], unpack_bf16x2(w[u].x));
@@ -134,7 +149,7 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
                 }
             }
             for (; mi < m1; ++mi) {
-                const uint4 w = __ldcs(src(mi));
+                const uint4 w = __ldcs(next());
                 acc_add2(hi[0], lo[0], unpack_bf16x2(w.x));
                 acc_add2(hi[1], lo[1], unpack_bf16x2(w.y));
                 acc_add2(hi[2], lo[2], unpack_bf16x2(w.z));
