@@ -621,6 +621,68 @@ def run_merge(args, w):
     print(json.dumps(line), flush=True)
 
 
+def run_fused(args, w):
+    """Cross-layer fused decode (benchmark only: a model never has every layer's queries at once):
+    one step = for every owner, its new token appended and all its block's layers decoded in one
+    mlkv_decode_block_fused launch, which reads each K/V tile of the slot once.  Same inputs and
+    tokens/s as the decode step of run(); L2 flushed before every step."""
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device
+
+    torch.cuda.set_device(0)
+    owners = w.owners()
+    cache = mlkv.MLKVCache(w.l, w.h, w.d, w.owner, w.g, w.b, w.max_seq)
+    seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
+    blocks = {o: [n for n in range(w.l) if w.owner[n] == o] for o in owners}
+    Qb = {o: torch.stack([Q[n] for n in blocks[o]]) for o in owners}
+    outs = {o: torch.empty_like(Qb[o]) for o in owners}
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for o in owners:
+            cache.append(o, Kn[o], Vn[o], seq_lens, stream)
+            cache.decode_block_fused(o, Qb[o], outs[o], seq_lens, stream)
+
+    for _ in range(args.warmup):
+        step()
+    cache.sync_status()
+    times = []
+    with Clocks(0) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+    cache.sync_status()
+    ms = statistics.median(times)
+    tot_len = int(np.sum(seq_lens))
+    kv_bytes = 2 * len(owners) * w.g * tot_len * w.d * 2          # every slot read once
+    qo_bytes = 2 * w.l * w.b * w.h * w.d * 2
+    gbs = (kv_bytes + qo_bytes) / (ms / 1e3) / 1e9
+    flops = 4.0 * w.h * w.d * tot_len * w.l
+    peak, kind = _hbm_peak()
+    line = {"metric": "decode-attn tokens/s per step (all layers), cross-layer fused",
+            "value": w.b / (ms / 1e3), "unit": "tokens/s", "higher_is_better": True,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "dtype": "bf16",
+            "data": "synthetic", "benchmark_only": "needs every layer's queries at once",
+            "config": {"workload": w.name, "layers": w.l, "q_heads": w.h, "head_dim": w.d,
+                       "layer_owner": list(w.owner), "kv_heads_per_owner": w.g, "batch": w.b,
+                       "context": w.L, "l2": "flushed before every timed step"},
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s",
+                         "frac": gbs / peak, "peak_source": kind, "kernel": "prefill_kernel (fused)",
+                         "alg_bytes_per_step": kv_bytes + qo_bytes,
+                         "tensor_tflops_useful": flops / (ms / 1e3) / 1e12},
+            "gpu_launches": 2 * len(owners), "clocks": clocks.summary()}
+    print(json.dumps(line), flush=True)
+    cache.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -643,6 +705,8 @@ def main():
                     help="prefill throughput of the --config model (prompt of --prefill-len)")
     ap.add_argument("--prefill-batch", type=int, default=8)
     ap.add_argument("--prefill-len", type=int, default=2048)
+    ap.add_argument("--fused", action="store_true",
+                    help="cross-layer fused decode of the --config workload (benchmark only)")
     ap.add_argument("--merge", action="store_true",
                     help="Sec. 4.2 KV-weight merge of the --config model's K and V projections")
     args = ap.parse_args()
@@ -657,6 +721,10 @@ def main():
     if args.merge:
         from mlkv_synth import workloads
         run_merge(args, workloads.by_name(args.config))
+        return
+    if args.fused:
+        from mlkv_synth import workloads
+        run_fused(args, workloads.by_name(args.config))
         return
 
     from mlkv_synth import workloads

@@ -258,6 +258,27 @@ int mlkv_decode_attention_static(const void *kv_slot, int batch, int n_q_heads, 
                                  const int *seq_lens, void *cuda_stream);
 
 /*
+ * mlkv_decode_block_fused - decode attention of every layer of one owner block in one launch:
+ * each K/V tile of the owner's slot is read once for the query heads of all the block's layers.
+ * NOT a step of sequential decoding: layer n+1's queries depend on layer n's output, so a model
+ * never has them all at once; this call measures what the shared cache (Sec. 3) would allow if it
+ * did.  The result equals mlkv_decode_attention for each layer of the block (Eqs. 2-3, 15, 18).
+ *
+ *   owner_layer  an owner layer o; the block is every layer n with layer_owner[n] == o, in order
+ *   Q            device bf16 [L][batch][n_q_heads][head_dim], L = the block's layer count, layer-
+ *                major in block order; 16-byte aligned
+ *   out          device bf16 [L][batch][n_q_heads][head_dim]; must not overlap Q
+ *   seq_lens     host int32[batch]: positions [0, L_beta) of the owner's slot are visible (append
+ *                the new token first, e.g. with mlkv_append)
+ * Needs L <= 2 * floor(128 / G), G = n_q_heads / kv_heads (the L * G query rows of one KV head
+ * fill at most two 128-row tiles of whole layers), else MLKV_ERR_UNSUPPORTED.
+ * Errors: MLKV_ERR_INVALID_ARG (not an owner layer, null or unaligned pointers, overlap),
+ * MLKV_ERR_RANGE (lengths), MLKV_ERR_UNSUPPORTED, MLKV_ERR_CUDA.
+ */
+int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void *out,
+                            const int *seq_lens, void *cuda_stream);
+
+/*
  * mlkv_merge_kv_weights - converts one MHA projection (K or V) to MLKV by averaging (Sec. 4.2:
  * "KV heads in the same group of the same layer, as well as the heads from subsequent layers which
  * do not have KV heads of their own, are merged by averaging"): merged KV head j of owner layer o

@@ -117,6 +117,7 @@ struct mlkv_cache {
     int pdl = 1;                // programmatic dependent launch
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
+    int fused_ready = 0;        // the same for the fused-decode instance
     // mlkv_decode_step's recorded graph and the arguments it was recorded for
     int step_graph = 1;
     cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
@@ -838,6 +839,7 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
     p.G = c->G;
     p.s_max = s_max;
     p.slot = c->slot[layer];
+    p.fused_L = p.fused_L1 = 0;
     for (int beta = 0; beta < c->b; ++beta)
         p.prompt_len[beta] = prompt_lens[beta];
     // Work units, those that see the most keys first: two heads of a group at the same block when
@@ -868,6 +870,115 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
         p.n_units = n;
         if ((e = mlkv::launch_prefill(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
             return fail_cuda(e, "prefill launch");
+    }
+    return MLKV_OK;
+}
+
+int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void *out,
+                            const int *seq_lens, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (owner_layer < 0 || owner_layer >= c->l || c->owner[owner_layer] != owner_layer)
+        return fail(MLKV_ERR_INVALID_ARG, "layer %d is not an owner layer", owner_layer);
+    if (Q == nullptr || out == nullptr || !aligned16(Q) || !aligned16(out))
+        return fail(MLKV_ERR_INVALID_ARG, "Q and out must be non-NULL and 16-byte aligned");
+    if (seq_lens == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "seq_lens must be non-NULL");
+    int L = 0;
+    for (int n = 0; n < c->l; ++n)
+        L += c->owner[n] == owner_layer;
+    // Rows of one KV head: G heads in each of the block's L layers, in at most two 128-row tiles
+    // of whole layers.
+    const int L1 = 128 / c->G;
+    if (L > 2 * L1)
+        return fail(MLKV_ERR_UNSUPPORTED,
+                    "%d layers x %d heads per KV head exceed two tiles of 128 query rows", L, c->G);
+    if (c->h > mlkv::kPrefillMaxHeads || c->g > 255)
+        return fail(MLKV_ERR_UNSUPPORTED, "fused decode handles at most 255 KV heads");
+    for (int beta = 0; beta < c->b; ++beta)
+        if (seq_lens[beta] < 1 || seq_lens[beta] > c->max_seq)
+            return fail(MLKV_ERR_RANGE, "sequence length %d of sequence %d outside [1, %d]",
+                        seq_lens[beta], beta, c->max_seq);
+    const size_t qbytes = static_cast<size_t>(L) * c->b * c->h * c->d * 2;
+    const char *qs = static_cast<const char *>(Q);
+    const char *os = static_cast<const char *>(out);
+    if (os < qs + qbytes && qs < os + qbytes)
+        return fail(MLKV_ERR_INVALID_ARG, "out overlaps Q");
+    DeviceGuard guard(c->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    cudaError_t e;
+    if (!c->fused_ready) {
+        if ((e = mlkv::prepare_fused(c->d)) != cudaSuccess)
+            return fail_cuda(e, "cudaFuncSetAttribute(fused decode)");
+        c->fused_ready = 1;
+    }
+    static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
+    if (encode == nullptr)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+    // Q [L][b][h][d] as (channel, head in group, group, sequence, layer); a box of 64 channels x
+    // G heads x min(L1, L) layers is one tile's rows, layer-major.
+    CUtensorMap tmap_q;
+    const cuuint64_t dims[5] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->G),
+                                static_cast<cuuint64_t>(c->g), static_cast<cuuint64_t>(c->b),
+                                static_cast<cuuint64_t>(L)};
+    const cuuint64_t strides[4] = {static_cast<cuuint64_t>(c->d) * 2,
+                                   static_cast<cuuint64_t>(c->G) * c->d * 2,
+                                   static_cast<cuuint64_t>(c->h) * c->d * 2,
+                                   static_cast<cuuint64_t>(c->b) * c->h * c->d * 2};
+    const cuuint32_t box[5] = {64u, static_cast<cuuint32_t>(c->G), 1u, 1u,
+                               static_cast<cuuint32_t>(L < L1 ? L : L1)};
+    const cuuint32_t estr[5] = {1u, 1u, 1u, 1u, 1u};
+    CUresult r = encode(&tmap_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(Q), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled(fused Q) failed (CUresult %d)",
+                    static_cast<int>(r));
+    const CUtensorMap *tmap_kv = nullptr;
+    for (auto &v : c->variants)
+        if (v.v->tile_tokens == 128)
+            tmap_kv = &v.tmap;
+    if (tmap_kv == nullptr)
+        return fail(MLKV_ERR_UNSUPPORTED, "no 128-position cache map for d=%d", c->d);
+
+    static thread_local mlkv::PrefillParams p;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.err = c->err;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
+    p.b = c->b;
+    p.h = c->h;
+    p.g = c->g;
+    p.G = c->G;
+    p.s_max = c->max_seq;
+    p.slot = c->slot[owner_layer];
+    p.head_pairs = 0;
+    p.fused_L = L;
+    p.fused_L1 = L1;
+    for (int beta = 0; beta < c->b; ++beta)
+        p.prompt_len[beta] = seq_lens[beta];
+    // One unit per (sequence, KV head), the longest sequences first.
+    std::vector<int> order(c->b);
+    for (int beta = 0; beta < c->b; ++beta)
+        order[beta] = beta;
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
+    int n = 0;
+    for (int beta : order)
+        for (int j = 0; j < c->g; ++j) {
+            p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(j) << 24);
+            if (++n == mlkv::kPrefillMaxUnits) {
+                p.n_units = n;
+                if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+                    return fail_cuda(e, "fused decode launch");
+                n = 0;
+            }
+        }
+    if (n > 0) {
+        p.n_units = n;
+        if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+            return fail_cuda(e, "fused decode launch");
     }
     return MLKV_OK;
 }

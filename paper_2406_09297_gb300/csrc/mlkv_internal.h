@@ -61,6 +61,9 @@ struct PrefillParams {
     int *err;                 // device error word
     float scale_log2;         // log2(e) / sqrt(D)
     int b, h, g, G, s_max, slot, n_units, head_pairs;
+    // Cross-layer fused decode (mlkv_decode_block_fused): the block's L layers, L1 of them in tile
+    // B (the rest in tile A); prompt_len holds the sequence lengths.  Both 0 for prefill.
+    int fused_L, fused_L1;
     int prompt_len[MLKV_MAX_BATCH];
     uint32_t units[kPrefillMaxUnits];
 };
@@ -71,6 +74,9 @@ size_t prefill_smem_bytes(int head_dim);
 cudaError_t prepare_prefill(int head_dim);
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream);
+cudaError_t prepare_fused(int head_dim);
+cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
+                         const PrefillParams &p, cudaStream_t stream);
 
 // KV-weight merge (mlkv_merge.cu).  Passed by value.
 constexpr int kMergeMaxLayers = 1024;

@@ -91,7 +91,7 @@ __device__ __forceinline__ float max3f(float a, float b, float c)
     return d;
 }
 
-template <int D>
+template <int D, bool kFused>
 __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_q,
                    const __grid_constant__ CUtensorMap tmap_kv,
@@ -116,16 +116,19 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     // The unit: sequence, last query block of B, head pair or head (see PrefillParams::units).
+    // Fused decode: sequence and KV head j; S is then the sequence length, every query row sees
+    // positions [0, S), and the tiles hold the block's layers [0, L1) (B) and [L1, L) (A).
     const uint32_t u = p.units[blockIdx.x];
     const int beta = static_cast<int>(u & 0x3FFu);
-    const int qb_b = static_cast<int>((u >> 10) & 0x3FFFu);
     const int sel = static_cast<int>(u >> 24);
+    const int S = p.prompt_len[beta];
+    const int qb_b = kFused ? (S - 1) / 128 : static_cast<int>((u >> 10) & 0x3FFFu);
     const int head_a = p.head_pairs ? 2 * sel : sel;
     const int head_b = p.head_pairs ? 2 * sel + 1 : sel;
     const int n_b = qb_b + 1;                                   // key tiles 0 .. qb_b
-    const int n_a = p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0);   // 0: no tile A
-    const int S = p.prompt_len[beta];
-    const int j = head_b / p.G;                                 // Eq. 15
+    const int n_a = kFused ? (p.fused_L > p.fused_L1 ? n_b : 0)
+                           : (p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0));   // 0: no tile A
+    const int j = kFused ? sel : head_b / p.G;                  // Eq. 15
     const int zk = ((p.slot * 2 + 0) * p.b + beta) * p.g + j;
     const int zv = zk + p.b * p.g;
 
@@ -156,6 +159,20 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
+    if (kFused && warp < 8) {
+        // The tiles' rows past the TMA box (box_rows = G x min(L1, L)) are never loaded; zero them
+        // so that their (discarded) scores stay finite.  TMA writes only rows below box_rows.
+        const int grp = warp >> 2, r = threadIdx.x & 127;
+        const int box_rows = (p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1) * p.G;
+        if (r >= box_rows) {
+            uint8_t *qrow = smem + PL::kQ + grp * PL::kTileBytes;
+#pragma unroll
+            for (int c = 0; c < 8 * PL::kSub; ++c)
+                *reinterpret_cast<uint4 *>(qrow + (c >> 3) * 16384 + r * 128 +
+                                           (((c & 7) ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+            fence_proxy_async_smem();
+        }
+    }
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
@@ -167,14 +184,29 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         // ------------------------------------ producer ------------------------------------------
         setmaxnreg_dec<PL::kRegsLow>();
         if (lane == 0) {
-            mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kTileBytes);
+            if (kFused) {
+                // Q [L][b][h][D] as (channel, head in group, group, sequence, layer): a box of
+                // min(L1, L) layers x G heads = the tile's rows, layer-major (row = layer*G + i).
+                const int box_rows = (p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1) * p.G;
+                mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kSub * box_rows * 128);
 #pragma unroll
-            for (int sub = 0; sub < PL::kSub; ++sub) {
-                if (n_a > 0)
-                    tma_load_4d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64, head_a,
-                                (n_a - 1) * 128, beta);
-                tma_load_4d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
-                            sub * 64, head_b, qb_b * 128, beta);
+                for (int sub = 0; sub < PL::kSub; ++sub) {
+                    if (n_a > 0)
+                        tma_load_5d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64, 0, j,
+                                    beta, p.fused_L1);
+                    tma_load_5d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
+                                sub * 64, 0, j, beta, 0);
+                }
+            } else {
+                mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kTileBytes);
+#pragma unroll
+                for (int sub = 0; sub < PL::kSub; ++sub) {
+                    if (n_a > 0)
+                        tma_load_4d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64,
+                                    head_a, (n_a - 1) * 128, beta);
+                    tma_load_4d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
+                                sub * 64, head_b, qb_b * 128, beta);
+                }
             }
             const int n_idx = 2 * n_b;   // K_0, V_0, K_1, V_1, ...
             int idx = 0;
@@ -310,7 +342,8 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         const uint32_t s_ready = bar_s_ready + 8 * grp, s_free = bar_s_free + 8 * grp;
         const uint32_t p_ready = bar_p_ready + 8 * grp, pv_done = bar_pv_done + 8 * grp;
         // The prompt's last block holds keys past its end; the first tile to reach it zeroes them.
-        const bool zero_v = n_g > 0 && n_g == (S + 127) / 128 && (grp == 0 || n_a != n_b);
+        const bool zero_v =
+            n_g > 0 && (kFused || n_g == (S + 127) / 128) && (grp == 0 || n_a != n_b);
         const float scale = p.scale_log2;
         const float NEG_INF = -__int_as_float(0x7f800000);
         auto wait = [&](uint32_t bar, int parity) {
@@ -349,8 +382,9 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int k = 0; k < 32; ++k)
-                        if (c * 32 + k > r)
-                            sv[c][k] = NEG_INF;   // a later position: causal mask
+                        if (kFused ? q0 + c * 32 + k >= S   // past the sequence
+                                   : c * 32 + k > r)        // a later position: causal mask
+                            sv[c][k] = NEG_INF;
             }
             float mx[4];
 #pragma unroll
@@ -441,9 +475,19 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             wait(pv_done, PL::kPSep ? n_g - 1 : 0);   // with P over S only the last P V commits
             tmem_fence_after();
             const float inv = fast_rcp(l_run);
-            const bool valid = q0 + r < S;
-            __nv_bfloat16 *orow =
-                p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
+            bool valid;
+            __nv_bfloat16 *orow;
+            if (kFused) {
+                // Row r: layer (grp ? 0 : L1) + r / G of the block, head j*G + r % G; out [L][b][h][D].
+                const int L1 = p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1;
+                valid = r < (grp ? L1 : p.fused_L - p.fused_L1) * p.G;
+                const int layer = (grp ? 0 : p.fused_L1) + r / p.G;
+                orow = p.out + ((static_cast<size_t>(layer) * p.b + beta) * p.h + j * p.G +
+                                r % p.G) * D;
+            } else {
+                valid = q0 + r < S;
+                orow = p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
+            }
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 float ov[32];
@@ -474,10 +518,36 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     }
 }
 
-template <int D>
+template <int D, bool kFused = false>
 const void *prefill_fn()
 {
-    return reinterpret_cast<const void *>(&prefill_kernel<D>);
+    return reinterpret_cast<const void *>(&prefill_kernel<D, kFused>);
+}
+
+const void *kernel_fn(int head_dim, bool fused)
+{
+    if (fused)
+        return head_dim == 64 ? prefill_fn<64, true>() : prefill_fn<128, true>();
+    return head_dim == 64 ? prefill_fn<64>() : prefill_fn<128>();
+}
+
+cudaError_t launch(int head_dim, bool fused, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
+                   const PrefillParams &p, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
+    cfg.blockDim = dim3(static_cast<unsigned>(head_dim == 64 ? PrefillPlan<64>::kThreads
+                                                             : PrefillPlan<128>::kThreads));
+    cfg.dynamicSmemBytes = head_dim == 64 ? PrefillPlan<64>::kAlloc : PrefillPlan<128>::kAlloc;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void *args[] = {const_cast<CUtensorMap *>(tmap_q), const_cast<CUtensorMap *>(tmap_kv),
+                    const_cast<PrefillParams *>(&p)};
+    return cudaLaunchKernelExC(&cfg, kernel_fn(head_dim, fused), args);
 }
 
 }  // namespace
@@ -489,7 +559,14 @@ size_t prefill_smem_bytes(int head_dim)
 
 cudaError_t prepare_prefill(int head_dim)
 {
-    return cudaFuncSetAttribute(head_dim == 64 ? prefill_fn<64>() : prefill_fn<128>(),
+    return cudaFuncSetAttribute(kernel_fn(head_dim, false),
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(prefill_smem_bytes(head_dim)));
+}
+
+cudaError_t prepare_fused(int head_dim)
+{
+    return cudaFuncSetAttribute(kernel_fn(head_dim, true),
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(prefill_smem_bytes(head_dim)));
 }
@@ -497,21 +574,13 @@ cudaError_t prepare_prefill(int head_dim)
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream)
 {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
-    cfg.blockDim = dim3(static_cast<unsigned>(head_dim == 64 ? PrefillPlan<64>::kThreads
-                                                             : PrefillPlan<128>::kThreads));
-    cfg.dynamicSmemBytes = prefill_smem_bytes(head_dim);
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    void *args[] = {const_cast<CUtensorMap *>(tmap_q), const_cast<CUtensorMap *>(tmap_kv),
-                    const_cast<PrefillParams *>(&p)};
-    return cudaLaunchKernelExC(&cfg, head_dim == 64 ? prefill_fn<64>() : prefill_fn<128>(),
-                               args);
+    return launch(head_dim, false, tmap_q, tmap_kv, p, stream);
+}
+
+cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
+                         const PrefillParams &p, cudaStream_t stream)
+{
+    return launch(head_dim, true, tmap_q, tmap_kv, p, stream);
 }
 
 }  // namespace mlkv

@@ -30,7 +30,7 @@ EXPORTED = [
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
-    "mlkv_merge_kv_weights",
+    "mlkv_merge_kv_weights", "mlkv_decode_block_fused",
 ]
 
 
@@ -70,6 +70,7 @@ def _load():
     L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
     L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
     L.mlkv_merge_kv_weights.argtypes = [ip, ci, ci, ci, i64, vp, vp, vp]
+    L.mlkv_decode_block_fused.argtypes = [vp, ci, vp, vp, ip, vp]
     return L
 
 
@@ -215,6 +216,13 @@ def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, 
         _ptr(out), p, _stream(stream)))
 
 
+def mlkv_decode_block_fused(handle, owner_layer, Q, out, seq_lens, stream=None):
+    """Every layer of one owner block in one launch (benchmark only; Q, out [L][b][h][d])."""
+    a, p = _lens_ptr(seq_lens)
+    return _check(lib.mlkv_decode_block_fused(handle, owner_layer, _ptr(Q), _ptr(out), p,
+                                              _stream(stream)))
+
+
 def mlkv_merge_kv_weights(layer_owner, n_q_heads, n_kv_heads, W, out, stream=None):
     """Sec. 4.2 merge of one projection: W bf16 [l][h][row] -> out bf16 [m][g][row] (device)."""
     owner = np.ascontiguousarray(np.asarray(layer_owner, dtype=np.int32))
@@ -267,6 +275,9 @@ class MLKVCache:
     def prefill(self, layer, Q, K, V, out, prompt_lens, stream=None):
         """Causal prefill of one layer; Q / out [b][s_max][h][d], K / V [b][g][s_max][d]."""
         return mlkv_prefill(self.handle, layer, Q, K, V, out, prompt_lens, int(Q.shape[1]), stream)
+
+    def decode_block_fused(self, owner_layer, Q, out, seq_lens, stream=None):
+        return mlkv_decode_block_fused(self.handle, owner_layer, Q, out, seq_lens, stream)
 
     def load_prefix(self, layer, K, V, length, stream=None):
         return mlkv_load_prefix(self.handle, layer, K, V, length, stream)
