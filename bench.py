@@ -10,8 +10,11 @@ value   decode tokens/s of the whole job = batch * world / step time; device tim
         mlkv_decode_step call (the library replays the step's launches from a CUDA graph), CUDA
         events on the launching stream, L2 flushed (a 512 MiB write) before every step outside
         the timed events.
-e2e     the same metric end to end: the step's Q and new K/V copied from pinned host memory, one
-        mlkv_decode_step call, every layer's output copied back, all inside the timed region.
+e2e     the same metric end to end through the C ABI with host buffers: one
+        mlkv_decode_step_host call per step (the step's Q and new K/V copied from pinned host
+        memory, every layer's decode, every layer's output copied back), inside the timed region;
+        queued behind the L2 flush like the device-timed steps, the host waiting for each step's
+        outputs before the next.
 roofline  the decode kernel: logical K/V bytes per launch / mean launch duration (CUDA events
         around each launch) against the measured HBM copy bandwidth.
 cpu_baseline  the fp64 oracle (test infrastructure) on the host cores, on a bounded sample.
@@ -341,21 +344,13 @@ def run(args, w):
     host_k = Ks.cpu().pin_memory()
     host_v = Vs.cpu().pin_memory()
     host_out = torch.empty((w.l, w.b, w.h, w.d), dtype=torch.bfloat16).pin_memory()
-    dq = torch.empty_like(host_q, device="cuda")
-    dk = torch.empty_like(host_k, device="cuda")
-    dv = torch.empty_like(host_v, device="cuda")
-    dout = torch.empty_like(host_out, device="cuda")
     h2d = (host_q.numel() + host_k.numel() + host_v.numel()) * 2
     d2h = host_out.numel() * 2
 
     def e2e_step():
         # the user's view: this step's inputs from pinned host memory, one library call for the
         # step, every layer's output back to pinned host memory
-        dq.copy_(host_q, non_blocking=True)
-        dk.copy_(host_k, non_blocking=True)
-        dv.copy_(host_v, non_blocking=True)
-        mlkv.mlkv_decode_step(cache.handle, dq, dk, dv, dout, seq_lens)
-        host_out.copy_(dout, non_blocking=True)
+        mlkv.mlkv_decode_step_host(cache.handle, host_q, host_k, host_v, host_out, seq_lens)
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -363,8 +358,10 @@ def run(args, w):
     torch.cuda.synchronize()
     e_times = []
     for _ in range(args.steps):
+        # As for the device-timed steps, the L2 flush keeps the GPU busy while the host queues the
+        # call (a user loop queues step k+1 while step k runs); the host then waits for this step's
+        # outputs in host memory before the next.
         flush.zero_()
-        torch.cuda.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()

@@ -141,6 +141,22 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
                      const int *seq_lens, void *cuda_stream);
 
 /*
+ * mlkv_decode_step_host - mlkv_decode_step with the step's tensors in host memory (the user's end
+ * of a step): Q, K and V are copied to device staging buffers held by the cache, the step runs on
+ * them and every layer's output is copied back to out, all queued on cuda_stream with one
+ * cudaMemcpyAsync per tensor.  Layouts as for mlkv_decode_step, in host memory.
+ * With page-locked buffers (cudaHostAlloc, cudaHostRegister) and option "step_graph" = 1 the copies
+ * and the launches of a step are recorded into one CUDA graph the second time the same arguments
+ * come and replayed after (as for mlkv_decode_step); pageable buffers run directly, and their
+ * copies synchronise with the host as CUDA's pageable copies do.  out holds the step's outputs
+ * once the stream has reached the end of the call's work.  The staging buffers, 2 * (l*b*h*d +
+ * m*b*g*d) bf16, are allocated on the first call and kept until mlkv_cache_destroy.
+ * Errors: as mlkv_decode_step, and MLKV_ERR_OOM for the staging buffers.
+ */
+int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
+                          const int *seq_lens, void *cuda_stream);
+
+/*
  * mlkv_prefill - the prompt of every sequence through one layer at once (prefill): owner layers
  * first store the prompt's K/V at positions [0, s_max) of their slot (Sec. 3: only a layer with KV
  * heads of its own stores them); then prompt position t of query head i attends, causally, to

@@ -135,6 +135,12 @@ struct mlkv_cache {
         }
     } step_key, pending_key;   // recorded arguments; arguments seen once, not yet recorded
     int step_graph_replays = 0;
+    // mlkv_decode_step_host: device staging of the step's inputs and outputs, its own graph
+    void *stage = nullptr;     // Q [l][b][h][d], K, V [m][b][g][d], out [l][b][h][d]
+    cudaGraphExec_t host_exec = nullptr;
+    cudaStream_t side = nullptr;   // the copies that overlap the step's layers
+    cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};   // fork, inputs in, mid, outputs out
+    StepKey host_key, host_pending;
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0, last_tc = 0;
     // per-variant launch state
@@ -400,6 +406,15 @@ int mlkv_cache_destroy(mlkv_cache_t c)
     cudaDeviceSynchronize();
     if (c->step_exec)
         cudaGraphExecDestroy(c->step_exec);
+    if (c->host_exec)
+        cudaGraphExecDestroy(c->host_exec);
+    for (cudaEvent_t ev : c->ev)
+        if (ev)
+            cudaEventDestroy(ev);
+    if (c->side)
+        cudaStreamDestroy(c->side);
+    if (c->stage)
+        cudaFree(c->stage);
     if (c->record_stream)
         cudaStreamDestroy(c->record_stream);
     free_all(c);
@@ -615,13 +630,23 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
 }
 
 // The layer calls of one decode step, issued on `stream`.
+// With in_ready, layer 1 onwards waits for it (the later layers' queries still arriving); with
+// before_last, it is recorded once every layer but the last has been issued.
 static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
-                      const int *seq_lens, void *stream)
+                      const int *seq_lens, void *stream, cudaEvent_t in_ready = nullptr,
+                      cudaEvent_t before_last = nullptr)
 {
     const size_t qo = static_cast<size_t>(c->b) * c->h * c->d * 2;   // bytes of one layer's Q
     const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
     for (int n = 0; n < c->l; ++n) {
         int rc;
+        cudaError_t e = cudaSuccess;
+        if (n == 1 && in_ready != nullptr)
+            e = cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), in_ready, 0);
+        if (e == cudaSuccess && n == c->l - 1 && before_last != nullptr)
+            e = cudaEventRecord(before_last, static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess)
+            return fail_cuda(e, "step event");
         // Layers after the first follow this library's own launch of the preceding layer.
         const int early = (n > 0 && c->pdl) ? 1 : 0;
         const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
@@ -636,6 +661,92 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
     }
     return MLKV_OK;
 }
+
+}  // extern "C"
+
+namespace {
+
+mlkv_cache::StepKey step_key_of(const mlkv_cache *c, const void *Q, const void *K, const void *V,
+                                void *out, const int *seq_lens)
+{
+    mlkv_cache::StepKey key;
+    key.Q = Q;
+    key.K = K;
+    key.V = V;
+    key.out = out;
+    key.lens.assign(seq_lens, seq_lens + c->b);
+    key.tile = c->tile_tokens;
+    key.grid = c->grid;
+    key.cluster = c->cluster;
+    key.pdl = c->pdl;
+    key.tc = c->tc;
+    key.l2 = c->l2_persist;
+    return key;
+}
+
+// Runs a step's work: replayed from `exec` when `key` is what it was recorded with; issued directly
+// when these arguments were not seen on the previous call (about half the host time of recording,
+// and in a decode loop lengths change every step); recorded when they come back.  Recording runs
+// on a private stream (the caller's may be the legacy default stream, which cannot be captured);
+// the replay goes to the caller's stream.
+template <class Issue>
+int record_or_replay(mlkv_cache *c, const mlkv_cache::StepKey &key, mlkv_cache::StepKey &recorded,
+                     mlkv_cache::StepKey &pending, cudaGraphExec_t &exec, cudaStream_t stream,
+                     Issue issue)
+{
+    cudaError_t e;
+    if (exec == nullptr || !(key == recorded)) {
+        if (!(key == pending)) {
+            pending = key;
+            return issue(stream);
+        }
+        if (c->record_stream == nullptr &&
+            (e = cudaStreamCreateWithFlags(&c->record_stream, cudaStreamNonBlocking)) != cudaSuccess)
+            return fail_cuda(e, "cudaStreamCreateWithFlags");
+        e = cudaStreamBeginCapture(c->record_stream, cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess)
+            return fail_cuda(e, "cudaStreamBeginCapture");
+        int rc = issue(c->record_stream);
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamEndCapture(c->record_stream, &graph);
+        if (rc != MLKV_OK) {
+            if (graph)
+                cudaGraphDestroy(graph);
+            return rc;
+        }
+        if (e != cudaSuccess)
+            return fail_cuda(e, "cudaStreamEndCapture");
+        bool updated = false;
+        if (exec != nullptr) {
+            cudaGraphExecUpdateResultInfo info;
+            updated = cudaGraphExecUpdate(exec, graph, &info) == cudaSuccess;
+            if (!updated) {
+                cudaGetLastError();
+                cudaGraphExecDestroy(exec);
+                exec = nullptr;
+            }
+        }
+        if (!updated) {
+            e = cudaGraphInstantiate(&exec, graph, 0);
+            if (e != cudaSuccess) {
+                cudaGraphDestroy(graph);
+                exec = nullptr;
+                return fail_cuda(e, "cudaGraphInstantiate");
+            }
+        }
+        cudaGraphDestroy(graph);
+        recorded = key;
+    }
+    e = cudaGraphLaunch(exec, stream);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "cudaGraphLaunch");
+    ++c->step_graph_replays;
+    return MLKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
 
 int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
                      const int *seq_lens, void *cuda_stream)
@@ -660,70 +771,162 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
     if (!c->step_graph || cap != cudaStreamCaptureStatusNone)
         return issue_step(c, q, k, v, o, seq_lens, cuda_stream);   // the caller records us
 
-    mlkv_cache::StepKey key;
-    key.Q = Q;
-    key.K = K;
-    key.V = V;
-    key.out = out;
-    key.lens.assign(seq_lens, seq_lens + c->b);
-    key.tile = c->tile_tokens;
-    key.grid = c->grid;
-    key.cluster = c->cluster;
-    key.pdl = c->pdl;
-    key.tc = c->tc;
-    key.l2 = c->l2_persist;
-    if (c->step_exec == nullptr || !(key == c->step_key)) {
-        if (!(key == c->pending_key)) {
-            // Arguments not seen on the previous call: issue the launches directly (about half the
-            // host time of recording them), since in a decode loop lengths change every step.
-            // Arguments that come back on the next call are recorded then.
-            c->pending_key = key;
-            return issue_step(c, q, k, v, o, seq_lens, cuda_stream);
+    mlkv_cache::StepKey key = step_key_of(c, Q, K, V, out, seq_lens);
+    return record_or_replay(c, key, c->step_key, c->pending_key, c->step_exec, stream,
+                            [&](cudaStream_t s) { return issue_step(c, q, k, v, o, seq_lens, s); });
+}
+
+int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
+                          const int *seq_lens, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
+    if (Q == nullptr || K == nullptr || V == nullptr || out == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "Q, K, V and out must be non-NULL");
+    int rc = check_seq_lens(c, seq_lens);
+    if (rc != MLKV_OK)
+        return rc;
+    DeviceGuard guard(c->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    cudaError_t e;
+    mlkv_cache::StepKey key = step_key_of(c, Q, K, V, out, seq_lens);
+    if (c->host_exec != nullptr && c->step_graph && key == c->host_key) {
+        // The arguments this step was recorded with (their buffers were checked then).
+        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+        if ((e = cudaStreamIsCapturing(stream, &cap)) != cudaSuccess)
+            return fail_cuda(e, "cudaStreamIsCapturing");
+        if (cap == cudaStreamCaptureStatusNone) {
+            if ((e = cudaGraphLaunch(c->host_exec, stream)) != cudaSuccess)
+                return fail_cuda(e, "cudaGraphLaunch");
+            ++c->step_graph_replays;
+            return MLKV_OK;
         }
-        // Record the step once for these arguments (on a private stream: the caller's may be the
-        // legacy default stream, which cannot be captured), then replay it on the caller's.
-        if (c->record_stream == nullptr &&
-            (e = cudaStreamCreateWithFlags(&c->record_stream, cudaStreamNonBlocking)) != cudaSuccess)
-            return fail_cuda(e, "cudaStreamCreateWithFlags");
-        e = cudaStreamBeginCapture(c->record_stream, cudaStreamCaptureModeThreadLocal);
-        if (e != cudaSuccess)
-            return fail_cuda(e, "cudaStreamBeginCapture");
-        rc = issue_step(c, q, k, v, o, seq_lens, c->record_stream);
-        cudaGraph_t graph = nullptr;
-        e = cudaStreamEndCapture(c->record_stream, &graph);
-        if (rc != MLKV_OK) {
-            if (graph)
-                cudaGraphDestroy(graph);
-            return rc;
-        }
-        if (e != cudaSuccess)
-            return fail_cuda(e, "cudaStreamEndCapture");
-        bool updated = false;
-        if (c->step_exec != nullptr) {
-            cudaGraphExecUpdateResultInfo info;
-            updated = cudaGraphExecUpdate(c->step_exec, graph, &info) == cudaSuccess;
-            if (!updated) {
-                cudaGetLastError();
-                cudaGraphExecDestroy(c->step_exec);
-                c->step_exec = nullptr;
-            }
-        }
-        if (!updated) {
-            e = cudaGraphInstantiate(&c->step_exec, graph, 0);
-            if (e != cudaSuccess) {
-                cudaGraphDestroy(graph);
-                c->step_exec = nullptr;
-                return fail_cuda(e, "cudaGraphInstantiate");
-            }
-        }
-        cudaGraphDestroy(graph);
-        c->step_key = key;
     }
-    e = cudaGraphLaunch(c->step_exec, stream);
-    if (e != cudaSuccess)
-        return fail_cuda(e, "cudaGraphLaunch");
-    ++c->step_graph_replays;
-    return MLKV_OK;
+    const size_t qo_bytes = static_cast<size_t>(c->l) * c->b * c->h * c->d * 2;
+    const size_t kv_bytes = static_cast<size_t>(c->m) * c->b * c->g * c->d * 2;
+    if (c->stage == nullptr && (e = cudaMalloc(&c->stage, 2 * qo_bytes + 2 * kv_bytes)) != cudaSuccess) {
+        c->stage = nullptr;
+        return fail(MLKV_ERR_OOM, "staging buffers (%zu bytes): %s", 2 * qo_bytes + 2 * kv_bytes,
+                    cudaGetErrorString(e));
+    }
+    char *dq = static_cast<char *>(c->stage);
+    char *dk = dq + qo_bytes;
+    char *dv = dk + kv_bytes;
+    char *dout = dv + kv_bytes;
+    // Page-locked, 16-byte-aligned buffers are read and written by copy kernels through their
+    // device-mapped addresses (one launch in, one out); anything else takes one cudaMemcpyAsync
+    // per tensor (a copy-engine transfer has ~12 us of fixed latency).
+    const void *dev[4] = {nullptr, nullptr, nullptr, nullptr};
+    bool mapped = true;
+    {
+        const void *hp[4] = {Q, K, V, out};
+        for (int k = 0; k < 4; ++k) {
+            cudaPointerAttributes at;
+            if (cudaPointerGetAttributes(&at, hp[k]) != cudaSuccess ||
+                at.type != cudaMemoryTypeHost || at.devicePointer == nullptr ||
+                !aligned16(at.devicePointer)) {
+                cudaGetLastError();
+                mapped = false;
+                break;
+            }
+            dev[k] = at.devicePointer;
+        }
+    }
+    if (mapped && c->side == nullptr) {
+        if ((e = cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking)) != cudaSuccess)
+            return fail_cuda(e, "cudaStreamCreateWithFlags");
+        for (cudaEvent_t &ev : c->ev)
+            if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess)
+                return fail_cuda(e, "cudaEventCreateWithFlags");
+    }
+    auto issue = [&](cudaStream_t s) {
+        if (mapped) {
+            // Layer 0's queries and the new tokens first; the other layers' queries on a side
+            // branch while layer 0 runs; the outputs of all layers but the last on the side branch
+            // while the last runs; the last layer's outputs at the end.
+            const size_t q1 = qo_bytes / c->l;   // one layer
+            const bool split = c->l > 1;
+            mlkv::StageParams a{};
+            a.n = 3;
+            a.src[0] = dev[0]; a.dst[0] = dq; a.bytes[0] = split ? q1 : qo_bytes;
+            a.src[1] = dev[1]; a.dst[1] = dk; a.bytes[1] = kv_bytes;
+            a.src[2] = dev[2]; a.dst[2] = dv; a.bytes[2] = kv_bytes;
+            cudaError_t err = cudaSuccess;
+            if (split) {
+                err = cudaEventRecord(c->ev[0], s);
+                if (err == cudaSuccess)
+                    err = cudaStreamWaitEvent(c->side, c->ev[0], 0);
+                mlkv::StageParams b{};
+                b.n = 1;
+                b.src[0] = static_cast<const char *>(dev[0]) + q1; b.dst[0] = dq + q1;
+                b.bytes[0] = qo_bytes - q1;
+                if (err == cudaSuccess)
+                    err = mlkv::launch_stage_copy(b, c->side);
+                if (err == cudaSuccess)
+                    err = cudaEventRecord(c->ev[1], c->side);
+            }
+            if (err == cudaSuccess)
+                err = mlkv::launch_stage_copy(a, s);
+            if (err != cudaSuccess)
+                return fail_cuda(err, "copy-in of the step's inputs");
+            int r = issue_step(c, dq, dk, dv, dout, seq_lens, s, split ? c->ev[1] : nullptr,
+                               split ? c->ev[2] : nullptr);
+            if (r != MLKV_OK)
+                return r;
+            char *hout = static_cast<char *>(const_cast<void *>(dev[3]));
+            if (split) {
+                mlkv::StageParams o{};
+                o.n = 1;
+                o.src[0] = dout; o.dst[0] = hout; o.bytes[0] = qo_bytes - q1;
+                err = cudaStreamWaitEvent(c->side, c->ev[2], 0);
+                if (err == cudaSuccess)
+                    err = mlkv::launch_stage_copy(o, c->side);
+                if (err == cudaSuccess)
+                    err = cudaEventRecord(c->ev[3], c->side);
+            }
+            mlkv::StageParams last{};
+            last.n = 1;
+            last.src[0] = dout + (split ? qo_bytes - q1 : 0);
+            last.dst[0] = hout + (split ? qo_bytes - q1 : 0);
+            last.bytes[0] = split ? q1 : qo_bytes;
+            if (err == cudaSuccess)
+                err = mlkv::launch_stage_copy(last, s);
+            if (err == cudaSuccess && split)
+                err = cudaStreamWaitEvent(s, c->ev[3], 0);   // the side branch rejoins
+            if (err != cudaSuccess)
+                return fail_cuda(err, "copy-out of the step's outputs");
+            return MLKV_OK;
+        }
+        cudaError_t err = cudaMemcpyAsync(dq, Q, qo_bytes, cudaMemcpyHostToDevice, s);
+        if (err == cudaSuccess)
+            err = cudaMemcpyAsync(dk, K, kv_bytes, cudaMemcpyHostToDevice, s);
+        if (err == cudaSuccess)
+            err = cudaMemcpyAsync(dv, V, kv_bytes, cudaMemcpyHostToDevice, s);
+        if (err != cudaSuccess)
+            return fail_cuda(err, "host-to-device copy of the step's inputs");
+        int r = issue_step(c, dq, dk, dv, dout, seq_lens, s);
+        if (r != MLKV_OK)
+            return r;
+        err = cudaMemcpyAsync(out, dout, qo_bytes, cudaMemcpyDeviceToHost, s);
+        if (err != cudaSuccess)
+            return fail_cuda(err, "device-to-host copy of the step's outputs");
+        return MLKV_OK;
+    };
+    // Only page-locked host memory can be recorded into a graph; anything else runs directly.
+    bool pinned = c->step_graph != 0;
+    for (const void *ptr : {Q, K, V, static_cast<const void *>(out)}) {
+        cudaPointerAttributes at;
+        if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess || at.type != cudaMemoryTypeHost) {
+            cudaGetLastError();
+            pinned = false;
+        }
+    }
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if ((e = cudaStreamIsCapturing(stream, &cap)) != cudaSuccess)
+        return fail_cuda(e, "cudaStreamIsCapturing");
+    if (!pinned || cap != cudaStreamCaptureStatusNone)
+        return issue(stream);
+    return record_or_replay(c, key, c->host_key, c->host_pending, c->host_exec, stream, issue);
 }
 
 int mlkv_load_prefix(mlkv_cache_t c, int layer, const void *K, const void *V, int len,

@@ -78,6 +78,16 @@ cudaError_t prepare_fused(int head_dim);
 cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                          const PrefillParams &p, cudaStream_t stream);
 
+// Copies through device-mapped page-locked host memory (mlkv_stage.cu): up to 4 segments, each a
+// multiple of 16 bytes with 16-byte-aligned ends.
+struct StageParams {
+    const void *src[4];
+    void *dst[4];
+    size_t bytes[4];
+    int n;
+};
+cudaError_t launch_stage_copy(const StageParams &p, cudaStream_t stream);
+
 // KV-weight merge (mlkv_merge.cu).  Passed by value.
 constexpr int kMergeMaxLayers = 1024;
 struct MergeParams {

@@ -30,7 +30,7 @@ EXPORTED = [
     "mlkv_load_prefix", "mlkv_cache_bytes", "mlkv_num_slots", "mlkv_owner_slot", "mlkv_kv_ptr",
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
-    "mlkv_merge_kv_weights", "mlkv_decode_block_fused",
+    "mlkv_merge_kv_weights", "mlkv_decode_block_fused", "mlkv_decode_step_host",
 ]
 
 
@@ -53,6 +53,7 @@ def _load():
     L.mlkv_decode_attention.argtypes = [vp, ci, vp, vp, ip, vp]
     L.mlkv_append_decode_attention.argtypes = [vp, ci, vp, vp, vp, vp, ip, vp]
     L.mlkv_decode_step.argtypes = [vp, vp, vp, vp, vp, ip, vp]
+    L.mlkv_decode_step_host.argtypes = [vp, vp, vp, vp, vp, ip, vp]
     L.mlkv_load_prefix.argtypes = [vp, ci, vp, vp, ci, vp]
     L.mlkv_cache_bytes.argtypes = [vp]
     L.mlkv_cache_bytes.restype = i64
@@ -145,6 +146,13 @@ def mlkv_decode_step(handle, Q, K, V, out, seq_lens, stream=None):
     a, p = _lens_ptr(seq_lens)
     return _check(lib.mlkv_decode_step(handle, _ptr(Q), _ptr(K), _ptr(V), _ptr(out), p,
                                        _stream(stream)))
+
+
+def mlkv_decode_step_host(handle, Q, K, V, out, seq_lens, stream=None):
+    """mlkv_decode_step with Q, K, V and out in host memory (page-locked for the graph replay)."""
+    a, p = _lens_ptr(seq_lens)
+    return _check(lib.mlkv_decode_step_host(handle, _ptr(Q), _ptr(K), _ptr(V), _ptr(out), p,
+                                            _stream(stream)))
 
 
 def mlkv_prefill(handle, layer, Q, K, V, out, prompt_lens, s_max, stream=None):
@@ -275,6 +283,9 @@ class MLKVCache:
     def prefill(self, layer, Q, K, V, out, prompt_lens, stream=None):
         """Causal prefill of one layer; Q / out [b][s_max][h][d], K / V [b][g][s_max][d]."""
         return mlkv_prefill(self.handle, layer, Q, K, V, out, prompt_lens, int(Q.shape[1]), stream)
+
+    def decode_step_host(self, Q, K, V, out, seq_lens, stream=None):
+        return mlkv_decode_step_host(self.handle, Q, K, V, out, seq_lens, stream)
 
     def decode_block_fused(self, owner_layer, Q, out, seq_lens, stream=None):
         return mlkv_decode_block_fused(self.handle, owner_layer, Q, out, seq_lens, stream)

@@ -167,3 +167,37 @@ def test_decode_loop_growing_lengths(owner, h, g, d, b, prefix):
                 mx, mean = errors(from_dev(out[n]), expect)
                 assert mx <= MAX_ABS and mean <= MEAN_ABS, (s, n, mx, mean)
         cache.sync_status()
+
+
+def test_step_host_buffers_match_device_step():
+    # mlkv_decode_step_host: the same step with Q, K, V and out in host memory; pinned buffers are
+    # replayed from a graph from the second call on (recorded then), pageable ones run directly.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    from mlkv_synth import device, workloads
+    w = workloads.config(1)
+    with mlkv.MLKVCache(w.l, w.h, w.d, w.owner, w.g, w.b, w.max_seq) as cache:
+        seq_lens, Q, Kn, Vn = device.workload_inputs(w, cache)
+        owners = w.owners()
+        Qs = torch.stack(Q)
+        Ks = torch.stack([Kn[n] for n in owners])
+        Vs = torch.stack([Vn[n] for n in owners])
+        ref = torch.empty((w.l, w.b, w.h, w.d), dtype=torch.bfloat16, device="cuda")
+        cache.decode_step(Qs, Ks, Vs, ref, seq_lens)
+        torch.cuda.synchronize()
+        want = ref.cpu()
+        for pinned in (True, False):
+            hq, hk, hv = Qs.cpu(), Ks.cpu(), Vs.cpu()
+            out = torch.full((w.l, w.b, w.h, w.d), float("nan"), dtype=torch.bfloat16)
+            if pinned:
+                hq, hk, hv, out = hq.pin_memory(), hk.pin_memory(), hv.pin_memory(), out.pin_memory()
+            before = cache.get_option("step_graph_replays")
+            for _ in range(4):
+                out.fill_(float("nan"))
+                cache.decode_step_host(hq, hk, hv, out, seq_lens)
+                torch.cuda.synchronize()
+                assert torch.equal(out.view(torch.int16), want.view(torch.int16))
+            replays = cache.get_option("step_graph_replays") - before
+            assert replays == (3 if pinned else 0), (pinned, replays)
+        cache.sync_status()
