@@ -287,25 +287,39 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             // Ring slots are released by tile B's softmax warps (they see every MMA that read them
             // complete), not by commits: a commit costs the tensor pipe about as much as a short MMA.
             for (int t = 0; ok && t < n_b; ++t) {
+                if (PL::kPSep) {
+                    // Both tiles' next S as soon as each tile's S has been read (early in its
+                    // softmax), then both P V as their P arrive: neither softmax waits for the
+                    // other tile's P before its next scores are computed.
+#pragma unroll
+                    for (int g = 0; g < 2; ++g) {
+                        const int ng = g ? n_b : n_a;
+                        if (!ok || t + 1 >= ng)
+                            continue;
+                        if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
+                            break;
+                        tmem_fence_after();
+                        issue_s(g, t + 1);
+                    }
+#pragma unroll
+                    for (int g = 0; g < 2; ++g) {
+                        const int ng = g ? n_b : n_a;
+                        if (!ok || t >= ng)
+                            continue;
+                        if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
+                            break;
+                        tmem_fence_after();
+                        issue_pv(g, t, t + 1 >= ng);
+                    }
+                    continue;
+                }
 #pragma unroll
                 for (int g = 0; g < 2; ++g) {
                     const int ng = g ? n_b : n_a;
                     if (!ok || t >= ng)
                         continue;
                     const bool next = t + 1 < ng;
-                    if (PL::kPSep) {
-                        // S of the next tile as soon as this one's S has been read.
-                        if (next) {
-                            if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
-                                break;
-                            tmem_fence_after();
-                            issue_s(g, t + 1);
-                        }
-                        if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
-                            break;
-                        tmem_fence_after();
-                        issue_pv(g, t, !next);
-                    } else {
+                    {
                         // Everything first, then P V and the next S back to back.
                         if (!tile_full(2 * t + 1) || (next && !tile_full(2 * t + 2)) ||
                             !wait(bar_p_ready + 8 * g, t))
