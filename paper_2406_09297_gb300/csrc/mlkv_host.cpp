@@ -118,6 +118,8 @@ struct mlkv_cache {
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
     int fused_ready = 0;        // the same for the fused-decode instance
+    float *fused_part = nullptr;   // context-chunk partials of mlkv_decode_block_fused
+    size_t fused_part_floats = 0;
     // mlkv_decode_step's recorded graph and the arguments it was recorded for
     int step_graph = 1;
     cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
@@ -415,6 +417,8 @@ int mlkv_cache_destroy(mlkv_cache_t c)
         cudaStreamDestroy(c->side);
     if (c->stage)
         cudaFree(c->stage);
+    if (c->fused_part)
+        cudaFree(c->fused_part);
     if (c->record_stream)
         cudaStreamDestroy(c->record_stream);
     free_all(c);
@@ -1159,9 +1163,40 @@ int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void
     p.head_pairs = 0;
     p.fused_L = L;
     p.fused_L1 = L1;
-    for (int beta = 0; beta < c->b; ++beta)
+    int max_len = 0;
+    for (int beta = 0; beta < c->b; ++beta) {
         p.prompt_len[beta] = seq_lens[beta];
-    // One unit per (sequence, KV head), the longest sequences first.
+        max_len = std::max(max_len, seq_lens[beta]);
+    }
+    // Units (sequence, KV head, chunk of the context): about one per SM when there are fewer
+    // (sequence, KV head) pairs than SMs, the chunks' partial results then merged.
+    const int n_kt_max = (max_len + 127) / 128;
+    const int want = std::max(1, 152 / (c->b * c->g));
+    int kc = (n_kt_max + want - 1) / want;
+    kc = std::max(kc, (n_kt_max + mlkv::kPrefillMaxBlocks - 1) / mlkv::kPrefillMaxBlocks);
+    const int cmax = (n_kt_max + kc - 1) / kc;
+    p.fused_kc = kc;
+    p.fused_cmax = cmax;
+    p.part = p.part_lse = nullptr;
+    if (cmax > 1) {
+        const size_t rows = static_cast<size_t>(c->b) * c->g * cmax * L * c->G;
+        const size_t floats = rows * (c->d + 1);
+        if (floats > c->fused_part_floats) {
+            if (c->fused_part)
+                cudaFree(c->fused_part);
+            c->fused_part = nullptr;
+            c->fused_part_floats = 0;
+            if ((e = cudaMalloc(&c->fused_part, floats * sizeof(float))) != cudaSuccess) {
+                c->fused_part = nullptr;
+                return fail(MLKV_ERR_OOM, "fused-decode partials (%zu bytes): %s",
+                            floats * sizeof(float), cudaGetErrorString(e));
+            }
+            c->fused_part_floats = floats;
+        }
+        p.part = c->fused_part;
+        p.part_lse = c->fused_part + rows * c->d;
+    }
+    // The longest sequences first.
     std::vector<int> order(c->b);
     for (int beta = 0; beta < c->b; ++beta)
         order[beta] = beta;
@@ -1169,20 +1204,25 @@ int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void
                      [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
     int n = 0;
     for (int beta : order)
-        for (int j = 0; j < c->g; ++j) {
-            p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(j) << 24);
-            if (++n == mlkv::kPrefillMaxUnits) {
-                p.n_units = n;
-                if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
-                    return fail_cuda(e, "fused decode launch");
-                n = 0;
+        for (int j = 0; j < c->g; ++j)
+            for (int ch = 0; ch * kc < (seq_lens[beta] + 127) / 128; ++ch) {
+                p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(ch) << 10) |
+                             (static_cast<uint32_t>(j) << 24);
+                if (++n == mlkv::kPrefillMaxUnits) {
+                    p.n_units = n;
+                    if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) !=
+                        cudaSuccess)
+                        return fail_cuda(e, "fused decode launch");
+                    n = 0;
+                }
             }
-        }
     if (n > 0) {
         p.n_units = n;
         if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
             return fail_cuda(e, "fused decode launch");
     }
+    if (cmax > 1 && (e = mlkv::launch_fused_combine(c->d, p, stream)) != cudaSuccess)
+        return fail_cuda(e, "fused decode merge launch");
     return MLKV_OK;
 }
 

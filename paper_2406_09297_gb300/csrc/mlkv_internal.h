@@ -64,6 +64,11 @@ struct PrefillParams {
     // Cross-layer fused decode (mlkv_decode_block_fused): the block's L layers, L1 of them in tile
     // B (the rest in tile A); prompt_len holds the sequence lengths.  Both 0 for prefill.
     int fused_L, fused_L1;
+    // Split over the context: a unit holds key tiles [chunk*kc, chunk*kc + kc) of its sequence;
+    // with more than one chunk (cmax > 1) it writes o = O/l (f32) and lse = m + log2(l) to part /
+    // part_lse [b][g][cmax][L*G rows] and combine_fused merges the chunks.
+    int fused_kc, fused_cmax;
+    float *part, *part_lse;
     int prompt_len[MLKV_MAX_BATCH];
     uint32_t units[kPrefillMaxUnits];
 };
@@ -77,6 +82,7 @@ cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtens
 cudaError_t prepare_fused(int head_dim);
 cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                          const PrefillParams &p, cudaStream_t stream);
+cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream);
 
 // Copies through device-mapped page-locked host memory (mlkv_stage.cu): up to 4 segments, each a
 // multiple of 16 bytes with 16-byte-aligned ends.

@@ -122,7 +122,13 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     const int beta = static_cast<int>(u & 0x3FFu);
     const int sel = static_cast<int>(u >> 24);
     const int S = p.prompt_len[beta];
-    const int qb_b = kFused ? (S - 1) / 128 : static_cast<int>((u >> 10) & 0x3FFFu);
+    // Fused decode: key tiles [kt0, kt0 + n_b) of the sequence (a chunk of p.fused_kc tiles).
+    const int chunk = static_cast<int>((u >> 10) & 0x3FFFu);
+    const int n_kt = (S + 127) / 128;
+    const int kt0 = kFused ? chunk * p.fused_kc : 0;
+    const int kt1 = kFused ? min(kt0 + p.fused_kc, n_kt) : 0;
+    const bool has_end = !kFused || kt1 == n_kt;   // the unit holds the sequence's last tile
+    const int qb_b = kFused ? kt1 - kt0 - 1 : chunk;
     const int head_a = p.head_pairs ? 2 * sel : sel;
     const int head_b = p.head_pairs ? 2 * sel + 1 : sel;
     const int n_b = qb_b + 1;                                   // key tiles 0 .. qb_b
@@ -225,7 +231,8 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 const int z = (idx & 1) ? zv : zk;
 #pragma unroll
                 for (int sub = 0; sub < PL::kSub; ++sub)
-                    tma_load_3d(dst + sub * 16384, &tmap_kv, fb, sub * 64, (idx >> 1) * 128, z);
+                    tma_load_3d(dst + sub * 16384, &tmap_kv, fb, sub * 64,
+                                ((idx >> 1) + kt0) * 128, z);
             }
             // No copy may still be in flight when the CTA exits.
             if (!mbar_wait(bar_q, 0))
@@ -348,7 +355,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
         const int n_g = grp ? n_b : n_a;
         const int head = grp ? head_b : head_a;
-        const int q0 = (n_g - 1) * 128;
+        const int q0 = (kt0 + n_g - 1) * 128;       // first position of the unit's last tile
         const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * grp;
         const uint32_t col_o = tmem + lane_off + PL::kColO + D * grp;
         const uint32_t col_p =
@@ -356,8 +363,8 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
         const uint32_t s_ready = bar_s_ready + 8 * grp, s_free = bar_s_free + 8 * grp;
         const uint32_t p_ready = bar_p_ready + 8 * grp, pv_done = bar_pv_done + 8 * grp;
         // The prompt's last block holds keys past its end; the first tile to reach it zeroes them.
-        const bool zero_v =
-            n_g > 0 && (kFused || n_g == (S + 127) / 128) && (grp == 0 || n_a != n_b);
+        const bool zero_v = n_g > 0 && (kFused ? has_end : n_g == (S + 127) / 128) &&
+                            (grp == 0 || n_a != n_b);
         const float scale = p.scale_log2;
         const float NEG_INF = -__int_as_float(0x7f800000);
         auto wait = [&](uint32_t bar, int parity) {
@@ -390,7 +397,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 if (lane == 0)
                     mbar_arrive(s_free);
             }
-            const bool diag = t == n_g - 1;
+            const bool diag = t == n_g - 1 && has_end;
             if (diag) {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -498,6 +505,29 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 const int layer = (grp ? 0 : p.fused_L1) + r / p.G;
                 orow = p.out + ((static_cast<size_t>(layer) * p.b + beta) * p.h + j * p.G +
                                 r % p.G) * D;
+                if (p.fused_cmax > 1) {
+                    // One chunk of the context: o = O / l and lse = m + log2(l) for the merge.
+                    const size_t row = ((static_cast<size_t>(beta) * p.g + j) * p.fused_cmax +
+                                        chunk) * (p.fused_L * p.G) +
+                                       layer * p.G + r % p.G;
+                    float *prow = p.part + row * D;
+                    if (valid && !flags[0])
+                        p.part_lse[row] = m_run + log2f(l_run);
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        float ov[32];
+                        tmem_ld32_nowait(col_o + c * 32, ov);
+                        tmem_wait_ld();
+                        if (valid && !flags[0]) {
+#pragma unroll
+                            for (int k = 0; k < 32; k += 4)
+                                *reinterpret_cast<float4 *>(prow + c * 32 + k) =
+                                    make_float4(ov[k] * inv, ov[k + 1] * inv, ov[k + 2] * inv,
+                                                ov[k + 3] * inv);
+                        }
+                    }
+                    valid = false;   // nothing more to store for this row
+                }
             } else {
                 valid = q0 + r < S;
                 orow = p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
@@ -530,6 +560,45 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                      "n"(PL::kTmemCols)
                      : "memory");
     }
+}
+
+// Merges the context chunks of the fused decode: per output row (sequence, KV head, block layer,
+// group head), weights 2^(lse_c - max) over the sequence's chunks.  One warp per row.
+template <int D>
+__global__ void __launch_bounds__(256) combine_fused_kernel(const __grid_constant__ PrefillParams p)
+{
+    const int rows_per_head = p.fused_L * p.G;
+    const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= static_cast<long long>(p.b) * p.g * rows_per_head)
+        return;
+    const int rr = static_cast<int>(row % rows_per_head);
+    const int bj = static_cast<int>(row / rows_per_head);
+    const int beta = bj / p.g, j = bj - beta * p.g;
+    const int n_kt = (p.prompt_len[beta] + 127) / 128;
+    const int chunks = (n_kt + p.fused_kc - 1) / p.fused_kc;
+    const size_t base = static_cast<size_t>(bj) * p.fused_cmax * rows_per_head + rr;
+    float mx = -__int_as_float(0x7f800000);
+    for (int c = 0; c < chunks; ++c)
+        mx = fmaxf(mx, p.part_lse[base + static_cast<size_t>(c) * rows_per_head]);
+    constexpr int E = D / 32;   // columns per lane
+    float acc[E] = {};
+    float wsum = 0.f;
+    for (int c = 0; c < chunks; ++c) {
+        const size_t r = base + static_cast<size_t>(c) * rows_per_head;
+        const float w = exp2f(p.part_lse[r] - mx);
+        wsum += w;
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            acc[e] += w * p.part[r * D + lane * E + e];
+    }
+    const float inv = 1.f / wsum;
+    const int layer = rr / p.G, i = rr - layer * p.G;
+    __nv_bfloat16 *orow = p.out + ((static_cast<size_t>(layer) * p.b + beta) * p.h + j * p.G + i) * D;
+#pragma unroll
+    for (int e = 0; e < E; e += 2)
+        *reinterpret_cast<uint32_t *>(orow + lane * E + e) =
+            pack_bf16x2(acc[e] * inv, acc[e + 1] * inv);
 }
 
 template <int D, bool kFused = false>
@@ -595,6 +664,17 @@ cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensor
                          const PrefillParams &p, cudaStream_t stream)
 {
     return launch(head_dim, true, tmap_q, tmap_kv, p, stream);
+}
+
+cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream)
+{
+    const long long rows = static_cast<long long>(p.b) * p.g * p.fused_L * p.G;
+    const unsigned blocks = static_cast<unsigned>((rows + 7) / 8);
+    if (head_dim == 64)
+        combine_fused_kernel<64><<<blocks, 256, 0, stream>>>(p);
+    else
+        combine_fused_kernel<128><<<blocks, 256, 0, stream>>>(p);
+    return cudaGetLastError();
 }
 
 }  // namespace mlkv

@@ -89,3 +89,10 @@ def test_fused_rejects_bad_arguments():
         with pytest.raises(mlkv.MLKVError) as e:
             cache.decode_block_fused(0, q, out, [5])
         assert e.value.code == mlkv.MLKV_ERR_UNSUPPORTED
+
+
+def test_fused_unsplit_context():
+    # b * g >= 152 (SMs): one unit per (sequence, KV head), no merge of context chunks.
+    rng = np.random.default_rng(73)
+    lens = list(rng.integers(1, 600, 40))
+    _run([0, 0, 0], 8, 4, 64, lens, 600, 73)
