@@ -56,6 +56,7 @@ LENS = [1, 127, 128, 129, 700, 1000]
     ("mha identity (one row a tile)", [0, 1], 4, 4, 64),
     ("llama-shaped (d 128, G 4, blocks of 4)", [0, 0, 0, 0, 4, 4, 4, 4], 32, 8, 128),
     ("non-uniform blocks", [0, 0, 2, 2, 2, 5], 8, 2, 128),
+    ("d 128, two tiles (G 16: 8 + 4 layers)", [0] * 12, 16, 1, 128),
 ])
 def test_fused_equals_per_layer_decode(name, owner, h, g, d):
     _run(owner, h, g, d, LENS, 1000, 71)

@@ -75,6 +75,15 @@ def test_prefill_long_prompts(d):
         _prefill_model(owner, h, g, d, b, [2048, 1500], s_max, s_max, 52, cache, ref, nthreads=2)
 
 
+def test_prefill_long_prompt_every_row():
+    # A 6000-position prompt: 47 key tiles per query block, units of very different lengths.
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, g, d = [0], 4, 1, 64
+    with mlkv.MLKVCache(1, h, d, owner, g, 1, 6000) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, 1, 6000)
+        _prefill_model(owner, h, g, d, 1, [6000], 6000, 6000, 54, cache, ref, nthreads=8)
+
+
 def test_prefill_then_decode_continues():
     # The cache a prefill leaves is the cache decoding continues from (Sec. 4.5: a prompt, then
     # tokens one by one): one decode step at length prompt + 1 in every layer.
