@@ -51,6 +51,21 @@ def _peaks():
         return 6800.0, "fallback"
 
 
+def max_over_ranks(ms, dist, device):
+    """The job's step time: the slowest rank's (every rank runs a whole replica, weak scaling)."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(batch, world, ms):
+    """Whole-job tokens per second: every rank's batch over the slowest rank's step time."""
+    return batch * world / (ms / 1e3)
+
+
 def _dist():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -299,12 +314,8 @@ def run(args, w):
             ev[k][1].record()
         barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    ms = sum(step_ms) / len(step_ms)
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = w.b * world / (ms / 1e3)
+    ms = max_over_ranks(sum(step_ms) / len(step_ms), dist, "cuda")
+    value = job_value(w.b, world, ms)
 
     # ---- decode kernel durations ---------------------------------------------------------------
     # The graph-timed step is nothing but the l decode launches back to back, so its device time
@@ -369,12 +380,8 @@ def run(args, w):
         e1.record()
         e1.synchronize()
         e_times.append(e0.elapsed_time(e1))
-    e_ms = sum(e_times) / len(e_times)
-    if dist is not None:
-        t = torch.tensor([e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
-    e2e_val = w.b * world / (e_ms / 1e3)
+    e_ms = max_over_ranks(sum(e_times) / len(e_times), dist, "cuda")
+    e2e_val = job_value(w.b, world, e_ms)
     cache.sync_status()
 
     result = None
