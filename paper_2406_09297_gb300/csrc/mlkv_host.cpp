@@ -141,7 +141,7 @@ struct mlkv_cache {
     void *stage = nullptr;     // Q [l][b][h][d], K, V [m][b][g][d], out [l][b][h][d]
     cudaGraphExec_t host_exec = nullptr;
     cudaStream_t side = nullptr;   // the copies that overlap the step's layers
-    cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};   // fork, inputs in, mid, outputs out
+    cudaEvent_t ev[2] = {nullptr, nullptr};   // fork, the later layers' queries in
     StepKey host_key, host_pending;
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0, last_tc = 0;
@@ -817,8 +817,8 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
     char *dk = dq + qo_bytes;
     char *dv = dk + kv_bytes;
     char *dout = dv + kv_bytes;
-    // Page-locked, 16-byte-aligned buffers are read and written by copy kernels through their
-    // device-mapped addresses (one launch in, one out); anything else takes one cudaMemcpyAsync
+    // Page-locked, 16-byte-aligned buffers are read by copy kernels and written by the layers
+    // themselves through their device-mapped addresses; anything else takes one cudaMemcpyAsync
     // per tensor (a copy-engine transfer has ~12 us of fixed latency).
     const void *dev[4] = {nullptr, nullptr, nullptr, nullptr};
     bool mapped = true;
@@ -846,8 +846,7 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
     auto issue = [&](cudaStream_t s) {
         if (mapped) {
             // Layer 0's queries and the new tokens first; the other layers' queries on a side
-            // branch while layer 0 runs; the outputs of all layers but the last on the side branch
-            // while the last runs; the last layer's outputs at the end.
+            // branch while layer 0 runs (joined before layer 1).
             const size_t q1 = qo_bytes / c->l;   // one layer
             const bool split = c->l > 1;
             mlkv::StageParams a{};
@@ -873,33 +872,11 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
                 err = mlkv::launch_stage_copy(a, s);
             if (err != cudaSuccess)
                 return fail_cuda(err, "copy-in of the step's inputs");
-            int r = issue_step(c, dq, dk, dv, dout, seq_lens, s, split ? c->ev[1] : nullptr,
-                               split ? c->ev[2] : nullptr);
-            if (r != MLKV_OK)
-                return r;
-            char *hout = static_cast<char *>(const_cast<void *>(dev[3]));
-            if (split) {
-                mlkv::StageParams o{};
-                o.n = 1;
-                o.src[0] = dout; o.dst[0] = hout; o.bytes[0] = qo_bytes - q1;
-                err = cudaStreamWaitEvent(c->side, c->ev[2], 0);
-                if (err == cudaSuccess)
-                    err = mlkv::launch_stage_copy(o, c->side);
-                if (err == cudaSuccess)
-                    err = cudaEventRecord(c->ev[3], c->side);
-            }
-            mlkv::StageParams last{};
-            last.n = 1;
-            last.src[0] = dout + (split ? qo_bytes - q1 : 0);
-            last.dst[0] = hout + (split ? qo_bytes - q1 : 0);
-            last.bytes[0] = split ? q1 : qo_bytes;
-            if (err == cudaSuccess)
-                err = mlkv::launch_stage_copy(last, s);
-            if (err == cudaSuccess && split)
-                err = cudaStreamWaitEvent(s, c->ev[3], 0);   // the side branch rejoins
-            if (err != cudaSuccess)
-                return fail_cuda(err, "copy-out of the step's outputs");
-            return MLKV_OK;
+            // The layers write their outputs straight into the page-locked buffer: every store of a
+            // decode output is a plain global store, which reaches host memory through its mapped
+            // address as well as device memory.
+            return issue_step(c, dq, dk, dv, static_cast<char *>(const_cast<void *>(dev[3])),
+                              seq_lens, s, split ? c->ev[1] : nullptr, nullptr);
         }
         cudaError_t err = cudaMemcpyAsync(dq, Q, qo_bytes, cudaMemcpyHostToDevice, s);
         if (err == cudaSuccess)
