@@ -204,7 +204,8 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
 /*
  * mlkv_set_option / mlkv_get_option - tuning knobs (host only, take effect on the next call):
  *   "tile_tokens"  positions per pipeline stage: 64, 128 or 256 (d=64) / 64 or 128 (d=128);
- *                  0 (default) picks per call: the longer tile when the mean length is >= 512
+ *                  0 (default) picks per call: the longer tile when the mean length is >= 512,
+ *                  except 128 for d=64 when batch x kv_heads >= 32 and the mean length <= 4096
  *   "grid"         persistent CTA count; 0 = one wave of resident CTAs (default)
  *   "l2_persist"   1 = give each decode launch an L2 access-policy window over its owner's slot
  *                  (default 0)

@@ -174,17 +174,25 @@ int check_seq_lens(const mlkv_cache *c, const int *seq_lens)
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Longer tiles move more bytes per TMA request and per barrier round trip; shorter ones waste less
-// on short sequences.  mean_len < 0 means "unknown" (reports the long-sequence choice).
-int default_tile_tokens(int d, double mean_len)
+// on short sequences.  For d = 64 the 128-position variant is small enough for two CTAs per SM,
+// so the next layer's CTAs start (and fetch) while this layer's last ones finish: measured faster
+// for many segments of moderate length (64 x 2048: 85 vs 89 us a step; 512 x ~2048: 527 vs 560),
+// slower for few long segments or HBM-bound layers (1 x 131072, 256 x 8192).  mean_len < 0 means
+// "unknown" (reports the long-sequence choice).
+int default_tile_tokens(int d, double mean_len, int segments)
 {
-    if (d == 64)
-        return (mean_len < 0 || mean_len >= 512) ? 256 : 128;
+    if (d == 64) {
+        if (mean_len >= 0 && (mean_len < 512 || (segments >= 32 && mean_len <= 4096)))
+            return 128;
+        return 256;
+    }
     return (mean_len < 0 || mean_len >= 512) ? 128 : 64;
 }
 
 mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0)
 {
-    const int T = c->tile_tokens > 0 ? c->tile_tokens : default_tile_tokens(c->d, mean_len);
+    const int T = c->tile_tokens > 0 ? c->tile_tokens
+                                     : default_tile_tokens(c->d, mean_len, c->b * c->g);
     mlkv_cache::Variant *plain = nullptr;
     for (auto &v : c->variants) {
         if (v.v->tile_tokens != T)
@@ -459,7 +467,8 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
 
 static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
                        const void *Q, void *out, const int *seq_lens, void *cuda_stream,
-                       int early_fetch = 0, const void *Q_next = nullptr)
+                       int early_fetch = 0, const void *Q_next = nullptr,
+                       int newest_ready = 0)
 {
     if (c == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
@@ -575,6 +584,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.early_fetch = early_fetch;
+    p.newest_ready = newest_ready;
     p.Q_next = static_cast<const __nv_bfloat16 *>(Q_next);
     // Segments split over many CTAs are merged by a separate parallel kernel: one warp merging
     // dozens of partials would serialise on its loads.
@@ -642,6 +652,7 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
 {
     const size_t qo = static_cast<size_t>(c->b) * c->h * c->d * 2;   // bytes of one layer's Q
     const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
+    int prev_combine = 0;
     for (int n = 0; n < c->l; ++n) {
         int rc;
         cudaError_t e = cudaSuccess;
@@ -654,14 +665,23 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         // Layers after the first follow this library's own launch of the preceding layer.
         const int early = (n > 0 && c->pdl) ? 1 : 0;
         const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
+        // A segment's newest row: an owner layer appends it itself (fused); a later layer of the
+        // block finds it complete when the owner's launch is not the previous one (each decode
+        // and combine grid triggers its dependents only after its own wait, so a grid starts
+        // with every grid two or more launches back complete).  The tcgen05 kernel keeps its
+        // early trigger: no such guarantee through it.
+        const int newest_ready =
+            (early && c->tc == 0 &&
+             (c->owner[n] == n || c->owner[n] != n - 1 || prev_combine)) ? 1 : 0;
         if (c->owner[n] == n)
             rc = decode_impl(c, n, K + kv * c->slot[n], V + kv * c->slot[n], Q + qo * n,
-                             out + qo * n, seq_lens, stream, early, q_next);
+                             out + qo * n, seq_lens, stream, early, q_next, newest_ready);
         else
             rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream,
-                             early, q_next);
+                             early, q_next, newest_ready);
         if (rc != MLKV_OK)
             return rc;
+        prev_combine = c->last_deferred;   // a combine launch followed this layer's decode
     }
     return MLKV_OK;
 }

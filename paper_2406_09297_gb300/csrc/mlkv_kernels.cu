@@ -224,16 +224,18 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     uint32_t qa[KS][4];
     if (early && warp < NCW && tile_lo < tile_hi)
         load_q_frag<D>(qa, p, wk.beta, wk.j, lane);
-    if (warp != PL::kProducer) {
-        if (!early)
-            grid_dependency_wait();
+    if (warp != PL::kProducer && !early)
+        grid_dependency_wait();
+    // The CTA's trigger (its first launch_dependents) comes only after the wait for the previous
+    // grid: so when a grid starts, every grid two or more launches back has completed, and a row
+    // such a grid wrote needs no wait (p.newest_ready).
+    if (warp == PL::kEpilogue && lane == 0) {
+        grid_dependency_wait();
         grid_dependents_launch();
     }
 
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
-        if (lane != 0)
-            grid_dependents_launch();   // only lane 0 touches global memory
         if (lane == 0) {
         int issued = 0;
         int tile = tile_lo;
@@ -253,7 +255,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                                  static_cast<uint32_t>(hi - lo));
         }
         for (; tile < tile_hi; ++tile) {
-            if (!waited && wk.tt == wk.nt - 1) {
+            if (!waited && wk.tt == wk.nt - 1 && !p.newest_ready) {
                 grid_dependency_wait();   // this tile holds the newest row
                 waited = true;
             }
@@ -306,12 +308,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 }
             }
             ++issued;
-            if (issued == STAGES)
-                grid_dependents_launch();   // the first loads are in flight
             wk.next(p, s_len, s_start);
         }
-        if (issued < STAGES)
-            grid_dependents_launch();
         // No copy may still be in flight when the CTA exits.
         const int first = issued > STAGES ? issued - STAGES : 0;
         for (int k = first; k < issued; ++k)
@@ -985,9 +983,9 @@ constexpr DecodeVariant make_variant()
 }
 
 // (head_dim, positions per tile, ring stages, consumer warps); the first match of a
-// (head_dim, tile) pair is used.
+// (head_dim, tile) pair is used.  <64, 128, 2, 4> fits twice on an SM (90 KB, 167 registers).
 const DecodeVariant kVariants[] = {
-    make_variant<64, 128, 5, 8>(),
+    make_variant<64, 128, 2, 4>(),
     make_variant<64, 256, 3, 4>(),
     make_variant<64, 64, 4, 4>(),
     make_variant<128, 64, 5, 4>(),
