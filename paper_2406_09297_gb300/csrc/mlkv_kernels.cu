@@ -168,14 +168,74 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     const int P = gridDim.x;
     const int cta = blockIdx.x;
     const int N = p.num_tiles;
-    const int tile_lo = static_cast<int>(static_cast<long long>(cta) * N / P);
-    const int tile_hi = static_cast<int>(static_cast<long long>(cta + 1) * N / P);
+    // floor(c N / P) in 32 bits when c N fits (a 64-bit division costs ~0.1 us at CTA start).
+    const bool narrow = static_cast<long long>(P) * N < (1ll << 32);
+    const int tile_lo = narrow ? static_cast<int>(static_cast<uint32_t>(cta) * N / P)
+                               : static_cast<int>(static_cast<long long>(cta) * N / P);
+    const int tile_hi = narrow ? static_cast<int>(static_cast<uint32_t>(cta + 1) * N / P)
+                               : static_cast<int>(static_cast<long long>(cta + 1) * N / P);
 
-    if (threadIdx.x == 0) {
+    const bool early = p.early_fetch != 0;
+    // The producer's copy of one tile into stage `s` (query rows too when a later piece starts).
+    auto issue_tile = [&](const TileWalk<T> &w, int s, bool with_q) {
+        const uint32_t fb = bar_full + 8 * s;
+        const uint32_t qbytes = static_cast<uint32_t>(p.G) * D * 2;
+        // A segment's last tile may be partly visible: only its boxes of 64 positions that
+        // hold visible rows are fetched (the rest of the stage keeps stale rows, which the
+        // consumers mask in S and zero in V).
+        const int vis = w.L - w.tt * T;
+        const int nbox = vis < T ? (vis + 63) / 64 : 0;
+        const uint32_t kv_bytes =
+            nbox > 0 ? static_cast<uint32_t>(nbox) * 64u * D * 2u * 2u : PL::kStageBytes;
+        mbar_arrive_expect_tx(fb, kv_bytes + (with_q ? qbytes : 0u));
+        if (with_q) {
+            const __nv_bfloat16 *q0 = p.Q + (static_cast<size_t>(w.beta) * p.h +
+                                             static_cast<size_t>(w.j) * p.G) * D;
+            for (int r = 0; r < p.G; ++r)
+                bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2, fb);
+        }
+        const int zk = ((p.slot * 2 + 0) * p.b + w.beta) * p.g + w.j;
+        const int zv = zk + p.b * p.g;
+        const int y = w.tt * T;
+        const uint32_t kdst = sbase + s * PL::kStageBytes;
+        const uint32_t vdst = kdst + PL::kTileBytes;
+        if (nbox == 0) {
+#pragma unroll
+            for (int sub = 0; sub < PL::kSub; ++sub) {
+                tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
+                tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
+            }
+        } else {
+            for (int bx = 0; bx < nbox; ++bx) {
+#pragma unroll
+                for (int sub = 0; sub < PL::kSub; ++sub) {
+                    const uint32_t off = sub * T * 128 + bx * 64 * 128;
+                    tma_load_3d(kdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zk);
+                    tma_load_3d(vdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zv);
+                }
+            }
+        }
+    };
+    // The ring's barriers belong to the producer lane.  With early fetch and one length for every
+    // sequence it also sends its first tile before the CTA barrier: a CTA that got its SM late
+    // (the last ones of a layer decide the layer's end) then has data on the way at once.
+    bool pre_issued = false;
+    if (threadIdx.x == PL::kProducer * 32) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(bar_full + 8 * s, 1);
             mbar_init(bar_empty + 8 * s, NCW);
         }
+        fence_barrier_init();
+        if (early && p.uniform_len > 0 && tile_lo < tile_hi) {
+            TileWalk<T> w0;
+            w0.init(p, s_len, s_start, tile_lo);
+            if (w0.tt != w0.nt - 1 || p.newest_ready) {   // not a newest row still to wait for
+                issue_tile(w0, 0, false);
+                pre_issued = true;
+            }
+        }
+    }
+    if (threadIdx.x == 0) {
         for (int r = 0; r < 2; ++r) {
             mbar_init(bar_res_full + 8 * r, 1);
             mbar_init(bar_res_empty + 8 * r, 1);
@@ -218,7 +278,6 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // write the last piece (scratch) or, at the latest, before they exit -- so this grid finishes
     // only after the previous one, as the next layer's wait expects.  The fused append writes
     // the newest row of this layer's own slot, which no earlier layer reads.
-    const bool early = p.early_fetch != 0;
     // The first piece's query fragments come straight from global memory, before the wait when
     // the queries cannot be the previous kernel's output; later pieces find theirs in a slot.
     uint32_t qa[KS][4];
@@ -237,8 +296,10 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
         if (lane == 0) {
-        int issued = 0;
-        int tile = tile_lo;
+        int issued = pre_issued ? 1 : 0;
+        int tile = tile_lo + issued;
+        if (pre_issued)
+            wk.next(p, s_len, s_start);
         bool waited = !early;
         if (!early)
             grid_dependency_wait();
@@ -267,46 +328,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             }
             if (flags[0])
                 break;
-            const uint32_t fb = bar_full + 8 * s;
             // A later piece starts here: its query rows come with the tile.
-            const bool with_q = (wk.tt == 0 && tile != tile_lo);
-            const uint32_t qbytes = static_cast<uint32_t>(p.G) * D * 2;
-            // A segment's last tile may be partly visible: only its boxes of 64 positions that
-            // hold visible rows are fetched (the rest of the stage keeps stale rows, which the
-            // consumers mask in S and zero in V).
-            const int vis = wk.L - wk.tt * T;
-            const int nbox = vis < T ? (vis + 63) / 64 : 0;
-            const uint32_t kv_bytes =
-                nbox > 0 ? static_cast<uint32_t>(nbox) * 64u * D * 2u * 2u : PL::kStageBytes;
-            mbar_arrive_expect_tx(fb, kv_bytes + (with_q ? qbytes : 0u));
-            if (with_q) {
-                const __nv_bfloat16 *q0 = p.Q + (static_cast<size_t>(wk.beta) * p.h +
-                                                 static_cast<size_t>(wk.j) * p.G) * D;
-                for (int r = 0; r < p.G; ++r)
-                    bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2,
-                              fb);
-            }
-            const int zk = ((p.slot * 2 + 0) * p.b + wk.beta) * p.g + wk.j;
-            const int zv = zk + p.b * p.g;
-            const int y = wk.tt * T;
-            const uint32_t kdst = sbase + s * PL::kStageBytes;
-            const uint32_t vdst = kdst + PL::kTileBytes;
-            if (nbox == 0) {
-#pragma unroll
-                for (int sub = 0; sub < PL::kSub; ++sub) {
-                    tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
-                    tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
-                }
-            } else {
-                for (int bx = 0; bx < nbox; ++bx) {
-#pragma unroll
-                    for (int sub = 0; sub < PL::kSub; ++sub) {
-                        const uint32_t off = sub * T * 128 + bx * 64 * 128;
-                        tma_load_3d(kdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zk);
-                        tma_load_3d(vdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zv);
-                    }
-                }
-            }
+            issue_tile(wk, s, wk.tt == 0 && tile != tile_lo);
             ++issued;
             wk.next(p, s_len, s_start);
         }
