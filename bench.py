@@ -281,6 +281,8 @@ def run(args, w):
         cache.set_option("tile_tokens", args.tile)
     if args.grid:
         cache.set_option("grid", args.grid)
+    if args.cluster >= 0:
+        cache.set_option("cluster", args.cluster)
     if args.l2_persist:
         cache.set_option("l2_persist", 1)
     if args.no_pdl:
@@ -455,6 +457,8 @@ def run_loop(args):
             cache.set_option("tc", args.tc)
             if args.grid:
                 cache.set_option("grid", args.grid)
+            if args.cluster >= 0:
+                cache.set_option("cluster", args.cluster)
             for n in owners:
                 kp, vp, strides = cache.kv_ptr(cache.owner_slot(n)[1])
                 device.fill_slot(kp, vp, strides, seed, n, b, g, d, max_seq)
@@ -706,6 +710,8 @@ def main():
     ap.add_argument("--config", default=DEFAULT_WORKLOAD)
     ap.add_argument("--tile", type=int, default=0)
     ap.add_argument("--grid", type=int, default=0)
+    ap.add_argument("--cluster", type=int, default=-1, choices=[-1, 0, 1, 2, 4],
+                    help="decode 'cluster' option (-1: the library default)")
     ap.add_argument("--l2-persist", action="store_true")
     ap.add_argument("--no-pdl", action="store_true")
     ap.add_argument("--tc", type=int, default=0, choices=[0, 1],

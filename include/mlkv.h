@@ -212,7 +212,9 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through
- *                  distributed shared memory; 0 = always the global-memory merge
+ *                  distributed shared memory (with two CTAs per SM, the largest size whose grid
+ *                  fits twice, so the next layer's CTAs are resident meanwhile); 0 = always the
+ *                  global-memory merge; 2 or 4 = that cluster size whenever it applies
  *   "pdl"          1 (default) = programmatic dependent launch: a decode launch's set-up overlaps
  *                  the previous kernel of the stream (it touches no global memory before that
  *                  kernel has completed); 0 = plain stream order

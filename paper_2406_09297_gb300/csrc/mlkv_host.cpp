@@ -550,8 +550,27 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                 grid = static_cast<int>(S);
             }
             if (c->cluster) {
+                // With two CTAs per SM, a grid that fits twice lets the next layer's CTAs all be
+                // resident, streaming their tiles, while this layer's finish; that hides the
+                // ramp of each layer, which the tile-unit model does not see.  So the largest
+                // cluster size whose grid fits twice wins while each CTA keeps >= 4 tiles
+                // (measured, 64 segments of 16 tiles of 128: 2-CTA clusters 80.5 us per
+                // 12-layer step against 84.7 us for 4-CTA clusters; with 32 segments 4-CTA
+                // clusters, 128 CTAs, stay the better).
+                if (c->cluster == 1 && var->ctas_per_sm >= 2) {
+                    for (int k : {4, 2}) {
+                        if (cluster_k == 0 && nt % k == 0 && nt / k >= 4 && 2 * S * k <= wave &&
+                            var->clusters[k] >= 2 * S)
+                            cluster_k = k;
+                    }
+                }
                 for (int k : {2, 4}) {
-                    if (nt % k == 0 && S * k <= wave && var->clusters[k] >= S && nt / k + 2 < best) {
+                    if (cluster_k > 1 && c->cluster == 1)
+                        break;      // chosen above
+                    if (c->cluster > 1 && k != c->cluster)
+                        continue;   // one cluster size asked for
+                    if (nt % k == 0 && S * k <= wave && var->clusters[k] >= S &&
+                        (c->cluster > 1 || nt / k + 2 < best)) {
                         best = nt / k + 2;
                         cluster_k = k;
                     }
@@ -1350,8 +1369,8 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         return MLKV_OK;
     }
     if (std::strcmp(key, "cluster") == 0) {
-        if (value != 0 && value != 1)
-            return fail(MLKV_ERR_INVALID_ARG, "cluster must be 0 or 1");
+        if (value != 0 && value != 1 && value != 2 && value != 4)
+            return fail(MLKV_ERR_INVALID_ARG, "cluster must be 0, 1, 2 or 4");
         c->cluster = static_cast<int>(value);
         return MLKV_OK;
     }
