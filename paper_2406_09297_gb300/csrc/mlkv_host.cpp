@@ -553,14 +553,15 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                 // With two CTAs per SM, a grid that fits twice lets the next layer's CTAs all be
                 // resident, streaming their tiles, while this layer's finish; that hides the
                 // ramp of each layer, which the tile-unit model does not see.  So the largest
-                // cluster size whose grid fits twice wins while each CTA keeps >= 4 tiles
-                // (measured, 64 segments of 16 tiles of 128: 2-CTA clusters 80.5 us per
+                // cluster size whose grid fits twice wins while each CTA keeps >= 4 tiles and the
+                // grid still holds a quarter of the resident CTAs, enough copies in flight to
+                // stream (measured, 64 segments of 16 tiles of 128: 2-CTA clusters 80.5 us per
                 // 12-layer step against 84.7 us for 4-CTA clusters; with 32 segments 4-CTA
                 // clusters, 128 CTAs, stay the better).
                 if (c->cluster == 1 && var->ctas_per_sm >= 2) {
                     for (int k : {4, 2}) {
                         if (cluster_k == 0 && nt % k == 0 && nt / k >= 4 && 2 * S * k <= wave &&
-                            var->clusters[k] >= 2 * S)
+                            4 * S * k >= wave && var->clusters[k] >= 2 * S)
                             cluster_k = k;
                     }
                 }

@@ -193,3 +193,10 @@ def test_cluster_size_forced(k):
     # the CTAs of the default shape), or 4-CTA clusters.
     run_small_case([0, 0, 2], 12, 1, 64, 64, [2048] * 64, 2048, seed=21,
                    options={"cluster": k}, expect={"last_cluster_k": k, "last_tile_tokens": 128})
+
+
+def test_cluster_rule_keeps_a_streaming_grid():
+    # One long segment on the two-CTA-per-SM tile: a cluster of its pieces would be a grid of a
+    # few CTAs, so the stream-K split over the SMs (and the separate merge) is kept.
+    run_small_case([0, 0], 8, 1, 64, 1, [8192], 8192, seed=22, options={"tile_tokens": 128},
+                   expect={"last_cluster_k": 0, "last_deferred_merge": 1})
