@@ -345,8 +345,9 @@ __global__ void __launch_bounds__(TcPlan<D, T, STAGES>::kThreads, 1)
                 const int vis = ws.L - ws.tt * T;
                 if (p.K_new != nullptr && vis <= T) {
                     // Fused append: the tile holds position L-1, the new token.  Its K/V replace
-                    // the tile row (the copy read the cache before the token was stored) and go
-                    // to the cache for the layers that read this slot later.
+                    // the tile row (the copy may have read the cache before the token was stored)
+                    // and, in the owner layer, go to the cache for the layers that read this slot
+                    // later.
                     const int r_new = vis - 1;
                     if (lane < 8 * PL::kSub) {
                         const size_t src =
@@ -356,12 +357,15 @@ __global__ void __launch_bounds__(TcPlan<D, T, STAGES>::kThreads, 1)
                         uint8_t *st = smem + s * PL::kStageBytes;
                         *reinterpret_cast<uint4 *>(st + swz<T>(r_new, lane)) = kn;
                         *reinterpret_cast<uint4 *>(st + PL::kTileBytes + swz<T>(r_new, lane)) = vn;
-                        const size_t dst =
-                            ((((static_cast<size_t>(p.slot) * 2) * p.b + ws.beta) * p.g + ws.j) *
-                                 static_cast<size_t>(p.max_seq) + (ws.L - 1)) * D + lane * 8;
-                        *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
-                        *reinterpret_cast<uint4 *>(
-                            p.cache + dst + static_cast<size_t>(p.b) * p.g * p.max_seq * D) = vn;
+                        if (p.store_new) {
+                            const size_t dst =
+                                ((((static_cast<size_t>(p.slot) * 2) * p.b + ws.beta) * p.g +
+                                  ws.j) * static_cast<size_t>(p.max_seq) + (ws.L - 1)) * D +
+                                lane * 8;
+                            *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
+                            *reinterpret_cast<uint4 *>(
+                                p.cache + dst + static_cast<size_t>(p.b) * p.g * p.max_seq * D) = vn;
+                        }
                     }
                     fence_proxy_async_smem();
                     __syncwarp();

@@ -468,7 +468,7 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
 static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
                        const void *Q, void *out, const int *seq_lens, void *cuda_stream,
                        int early_fetch = 0, const void *Q_next = nullptr,
-                       int newest_ready = 0)
+                       int newest_ready = 0, int store_new = 1)
 {
     if (c == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
@@ -605,6 +605,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     p.decode_grid = grid;
     p.early_fetch = early_fetch;
     p.newest_ready = newest_ready;
+    p.store_new = K_new != nullptr ? store_new : 0;
     p.Q_next = static_cast<const __nv_bfloat16 *>(Q_next);
     // Segments split over many CTAs are merged by a separate parallel kernel: one warp merging
     // dozens of partials would serialise on its loads.
@@ -672,7 +673,6 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
 {
     const size_t qo = static_cast<size_t>(c->b) * c->h * c->d * 2;   // bytes of one layer's Q
     const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
-    int prev_combine = 0;
     for (int n = 0; n < c->l; ++n) {
         int rc;
         cudaError_t e = cudaSuccess;
@@ -685,23 +685,24 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         // Layers after the first follow this library's own launch of the preceding layer.
         const int early = (n > 0 && c->pdl) ? 1 : 0;
         const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
-        // A segment's newest row: an owner layer appends it itself (fused); a later layer of the
-        // block finds it complete when the owner's launch is not the previous one (each decode
-        // and combine grid triggers its dependents only after its own wait, so a grid starts
-        // with every grid two or more launches back complete).  The tcgen05 kernel keeps its
-        // early trigger: no such guarantee through it.
-        const int newest_ready =
-            (early && c->tc == 0 &&
-             (c->owner[n] == n || c->owner[n] != n - 1 || prev_combine)) ? 1 : 0;
+        // A segment's newest row is the step's new token of the owner: the owner layer appends
+        // it itself (fused); a later layer of the block replaces that row of its tiles from the
+        // same input without storing it.  So no layer waits for another's launch to store it
+        // (newest_ready).  The tcgen05 kernel does neither and keeps the plain wait.
+        const int patch = (early && c->tc == 0) ? 1 : 0;
+        const int newest_ready = patch;
+        const size_t ks = kv * c->slot[c->owner[n]];
         if (c->owner[n] == n)
-            rc = decode_impl(c, n, K + kv * c->slot[n], V + kv * c->slot[n], Q + qo * n,
-                             out + qo * n, seq_lens, stream, early, q_next, newest_ready);
+            rc = decode_impl(c, n, K + ks, V + ks, Q + qo * n, out + qo * n, seq_lens, stream,
+                             early, q_next, newest_ready, 1);
+        else if (patch)
+            rc = decode_impl(c, n, K + ks, V + ks, Q + qo * n, out + qo * n, seq_lens, stream,
+                             early, q_next, newest_ready, 0);
         else
             rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream,
                              early, q_next, newest_ready);
         if (rc != MLKV_OK)
             return rc;
-        prev_combine = c->last_deferred;   // a combine launch followed this layer's decode
     }
     return MLKV_OK;
 }

@@ -44,9 +44,11 @@ struct DecodeParams {
                               // layer, which writes neither Q nor any cache row but a segment's
                               // newest: Q and the tiles without that row are read before the
                               // dependency wait
-    int newest_ready;         // 1: the segments' newest rows are complete when the grid starts
-                              // (written by a grid two or more launches back, or by this one's
-                              // fused append): no wait before a segment's last tile
+    int newest_ready;         // 1: the segments' newest rows are replaced from K_new/V_new by this
+                              // grid: no wait before a segment's last tile
+    int store_new;            // with K_new: 1 = also store the new token in the cache (the owner
+                              // layer's fused append); 0 = only replace the tiles' newest rows (a
+                              // later layer of the block, whose owner's launch stores the token)
     int seq_len[MLKV_MAX_BATCH];
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };

@@ -220,6 +220,11 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // sequence it also sends its first tile before the CTA barrier: a CTA that got its SM late
     // (the last ones of a layer decide the layer's end) then has data on the way at once.
     bool pre_issued = false;
+    // The trigger comes first: the next launch (inside a decode step, the next layer's decode)
+    // may start as soon as every CTA of this grid is resident.  What it reads before its own
+    // dependency wait is fixed by p.early_fetch, and it finishes only after this grid.
+    if (threadIdx.x == 0)
+        grid_dependents_launch();
     if (threadIdx.x == PL::kProducer * 32) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(bar_full + 8 * s, 1);
@@ -268,16 +273,16 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     TileWalk<T> wk;
     if (tile_lo < tile_hi)
         wk.init(p, s_len, s_start, tile_lo);
-    // Everything above overlaps the previous kernel's tail.  Normally global memory is touched only
-    // after the dependency wait.  When the previous kernel is this library's decode of the
-    // preceding layer (p.early_fetch, inside mlkv_decode_step), that kernel writes nothing this one
-    // reads except the newest row (position L-1) of the slot it appended to, which lies in the
-    // last tile of a segment, and the merge scratch (partials, counters).  So the queries and
-    // every other tile are fetched at once; the producer waits before it fetches a segment's last
-    // tile, the epilogue warp before it writes its first record, and the consumers before they
-    // write the last piece (scratch) or, at the latest, before they exit -- so this grid finishes
-    // only after the previous one, as the next layer's wait expects.  The fused append writes
-    // the newest row of this layer's own slot, which no earlier layer reads.
+    // Everything above overlaps the previous kernels' tails.  Normally global memory is touched
+    // only after the dependency wait.  When the previous kernels still running are this library's
+    // decodes of the preceding layers (p.early_fetch, inside mlkv_decode_step), they write nothing
+    // this one reads except the newest row (position L-1) of the slot an owner appended to, which
+    // lies in the last tile of a segment, and the merge scratch (partials, counters).  So the
+    // queries and every other tile are fetched at once, and a segment's last tile too when this
+    // grid replaces its newest row from K_new/V_new (p.newest_ready; else the producer waits
+    // before fetching it); the epilogue warp waits before it writes its first record, and the
+    // consumers before they write the last piece (scratch) or, at the latest, before they exit --
+    // so this grid finishes only after the previous one, as the next layer's wait expects.
     // The first piece's query fragments come straight from global memory, before the wait when
     // the queries cannot be the previous kernel's output; later pieces find theirs in a slot.
     uint32_t qa[KS][4];
@@ -285,13 +290,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         load_q_frag<D>(qa, p, wk.beta, wk.j, lane);
     if (warp != PL::kProducer && !early)
         grid_dependency_wait();
-    // The CTA's trigger (its first launch_dependents) comes only after the wait for the previous
-    // grid: so when a grid starts, every grid two or more launches back has completed, and a row
-    // such a grid wrote needs no wait (p.newest_ready).
-    if (warp == PL::kEpilogue && lane == 0) {
+    if (warp == PL::kEpilogue && lane == 0)
         grid_dependency_wait();
-        grid_dependents_launch();
-    }
 
     // -------------------------------- producer warp --------------------------------------------
     if (warp == PL::kProducer) {
@@ -437,8 +437,9 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 const uint32_t vt = kt + PL::kTileBytes;
                 if (p.K_new != nullptr && valid <= TW) {
                     // Fused append: this warp's slice holds position L-1, the new token.  Its K/V
-                    // replace the tile rows (the copy read the cache before the token was stored)
-                    // and are stored in the cache for the layers that read this slot later.
+                    // replace the tile rows (the copy may have read the cache before the token was
+                    // stored) and, in the owner layer, are stored in the cache for the layers that
+                    // read this slot later.
                     const int r_new = row0 + valid - 1;
                     if (lane < 8 * PL::kSub) {
                         const size_t src = (static_cast<size_t>(beta) * p.g + j) * D + lane * 8;
@@ -447,12 +448,14 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                         uint8_t *st = smem + s * PL::kStageBytes;
                         *reinterpret_cast<uint4 *>(st + swz<T>(r_new, lane)) = kn;
                         *reinterpret_cast<uint4 *>(st + PL::kTileBytes + swz<T>(r_new, lane)) = vn;
-                        const size_t dst =
-                            ((((static_cast<size_t>(p.slot) * 2) * p.b + beta) * p.g + j) *
-                                 static_cast<size_t>(p.max_seq) + (L - 1)) * D + lane * 8;
-                        *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
-                        *reinterpret_cast<uint4 *>(
-                            p.cache + dst + static_cast<size_t>(p.b) * p.g * p.max_seq * D) = vn;
+                        if (p.store_new) {
+                            const size_t dst =
+                                ((((static_cast<size_t>(p.slot) * 2) * p.b + beta) * p.g + j) *
+                                     static_cast<size_t>(p.max_seq) + (L - 1)) * D + lane * 8;
+                            *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
+                            *reinterpret_cast<uint4 *>(
+                                p.cache + dst + static_cast<size_t>(p.b) * p.g * p.max_seq * D) = vn;
+                        }
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
