@@ -29,7 +29,7 @@ def _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref):
 
 @pytest.mark.parametrize("owner,h,g,d,b,lens,max_seq", [
     ([0, 0, 2, 2, 2, 5], 12, 2, 64, 5, [1, 300, 1000, 77, 640], 1024),
-    ([0, 0, 0, 0], 12, 1, 64, 64, [2048] * 64, 2048),            # cluster mode
+    ([0, 0, 0, 0], 12, 1, 64, 64, [2048] * 64, 2048),            # whole segments per CTA
     ([0, 0, 2], 16, 4, 128, 3, [5000, 20, 4096], 5000),
 ])
 def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
@@ -61,14 +61,22 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
             else:
                 cache2.decode_attention(n, Q[n], out2[n], lens)
         torch.cuda.synchronize()
-        assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
+        uniform = bool((lens == lens[0]).all())
+        if uniform:
+            # With one length the step's later layers run whole segments per CTA (no merge),
+            # while the layer calls split segments into clusters: same results up to rounding.
+            assert cache.get_option("last_cluster_k") == 0
+            assert cache.get_option("last_grid") == b * g
+        else:
+            assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
         for n in range(l):
             if owner[n] == n:
                 s = owners.index(n)
                 ref.append(n, gen.bf16_bits_to_f64(kn[s]), gen.bf16_bits_to_f64(vn[s]), lens)
             expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens)
-            mx, mean = errors(from_dev(out[n]), expect)
-            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+            for o in (out, out2):
+                mx, mean = errors(from_dev(o[n]), expect)
+                assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
         cache.sync_status()
         cache2.sync_status()
 
