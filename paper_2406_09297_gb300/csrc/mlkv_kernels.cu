@@ -889,8 +889,10 @@ __global__ void __launch_bounds__(kCombineThreads)
 {
     __shared__ float s_w[kCombineMaxPieces];
     __shared__ float s_red[kCombineThreads];
-    grid_dependency_wait();
+    // The next layer's decode may start at once: it reads neither the partials nor `out`, and it
+    // writes partials only after its own dependency wait (after this grid).
     grid_dependents_launch();
+    grid_dependency_wait();
     const int seg = blockIdx.x;
     const int row = blockIdx.y;
     const int G = p.G;
