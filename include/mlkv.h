@@ -130,6 +130,11 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
  *   K, V     device bf16 [m][batch][g][d], every owner layer's new token, in slot order
  *   out      device bf16 [l][batch][h][d]
  *   seq_lens host int32[batch], as for mlkv_decode_attention
+ * The results equal those of the layer calls up to rounding: inside a step the layers' launches
+ * overlap and may split a layer's work differently (whole segments per CTA).  Every layer of an
+ * owner's block reads that owner's new token from K and V (the later layers take their newest
+ * row from there rather than from the cache), so K and V, like Q, must stay valid until the stream
+ * has run the whole step.
  * With option "step_graph" = 1 (default) a call whose pointers, lengths and options equal those of
  * the previous call replays a CUDA graph of the step's launches (recorded on the second such call;
  * new values in the same buffers are fine); a call with arguments different from the previous
