@@ -189,10 +189,11 @@ int default_tile_tokens(int d, double mean_len, int segments)
     return (mean_len < 0 || mean_len >= 512) ? 128 : 64;
 }
 
-mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0)
+mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0, int force_T = 0)
 {
-    const int T = c->tile_tokens > 0 ? c->tile_tokens
-                                     : default_tile_tokens(c->d, mean_len, c->b * c->g);
+    const int T = force_T > 0            ? force_T
+                  : c->tile_tokens > 0 ? c->tile_tokens
+                                       : default_tile_tokens(c->d, mean_len, c->b * c->g);
     mlkv_cache::Variant *plain = nullptr;
     for (auto &v : c->variants) {
         if (v.v->tile_tokens != T)
@@ -468,7 +469,7 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
 static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void *V_new,
                        const void *Q, void *out, const int *seq_lens, void *cuda_stream,
                        int early_fetch = 0, const void *Q_next = nullptr,
-                       int newest_ready = 0, int store_new = 1)
+                       int newest_ready = 0, int store_new = 1, int in_step = 0)
 {
     if (c == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
@@ -490,7 +491,13 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     for (int beta = 0; beta < c->b; ++beta)
         mean_len += seq_lens[beta];
     mean_len /= c->b;
-    mlkv_cache::Variant *var = pick_variant(c, mean_len);
+    // Inside a decode step, a layer that is one long segment (d = 64) runs on the 128-position
+    // tile (two CTAs per SM) over 64 CTAs, so the next layers' grids stream beside it (measured,
+    // batch 1, 131072 positions, 12 layers: MLKV-2 81.9 us against 96.3 us for the 256-position
+    // tile on the one-wave split, MQA 95.8 against 119.7; 48 or 76 CTAs were slower than 64).
+    const bool single_long = in_step && c->tile_tokens == 0 && c->grid <= 0 && c->d == 64 &&
+                             c->b * c->g == 1 && seq_lens[0] >= 16384;
+    mlkv_cache::Variant *var = pick_variant(c, mean_len, single_long ? 128 : 0);
     if (var == nullptr)
         return fail(MLKV_ERR_UNSUPPORTED, "no decode variant for d=%d tile_tokens=%d", c->d,
                     c->tile_tokens);
@@ -559,6 +566,8 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     }
     if (c->grid > 0) {
         grid = static_cast<int>(std::min<long long>(std::min(c->grid, c->max_ctas), tiles));
+    } else if (single_long && var->v->tile_tokens == 128) {
+        grid = static_cast<int>(std::min<long long>(64, tiles));
     } else if (whole > 0) {
         grid = static_cast<int>(whole);
     } else {
@@ -718,13 +727,13 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         const size_t ks = kv * c->slot[c->owner[n]];
         if (c->owner[n] == n)
             rc = decode_impl(c, n, K + ks, V + ks, Q + qo * n, out + qo * n, seq_lens, stream,
-                             early, q_next, newest_ready, 1);
+                             early, q_next, newest_ready, 1, 1);
         else if (patch)
             rc = decode_impl(c, n, K + ks, V + ks, Q + qo * n, out + qo * n, seq_lens, stream,
-                             early, q_next, newest_ready, 0);
+                             early, q_next, newest_ready, 0, 1);
         else
             rc = decode_impl(c, n, nullptr, nullptr, Q + qo * n, out + qo * n, seq_lens, stream,
-                             early, q_next, newest_ready);
+                             early, q_next, newest_ready, 1, 1);
         if (rc != MLKV_OK)
             return rc;
     }

@@ -209,3 +209,27 @@ def test_step_host_buffers_match_device_step():
             replays = cache.get_option("step_graph_replays") - before
             assert replays == (3 if pinned else 0), (pinned, replays)
         cache.sync_status()
+
+
+def test_step_single_long_segment():
+    # Batch 1, one KV head, 16384 positions: inside the step the later layers run the
+    # 128-position tile over 64 CTAs (the separate merge launch combines the pieces).
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, g, d, b, L = [0, 0, 0], 12, 1, 64, 1, 16384
+    lens = np.full(b, L, dtype=np.int32)
+    with mlkv.MLKVCache(len(owner), h, d, owner, g, b, L) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, L)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 61, cache, ref)
+        out = torch.full((len(owner), b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cache.decode_step(to_dev(qb), to_dev(kn), to_dev(vn), out, lens)
+        torch.cuda.synchronize()
+        assert cache.get_option("last_tile_tokens") == 128
+        assert cache.get_option("last_grid") == 64
+        ref.append(0, gen.bf16_bits_to_f64(kn[0]), gen.bf16_bits_to_f64(vn[0]), lens)
+        for n in range(len(owner)):
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens)
+            mx, mean = errors(from_dev(out[n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
