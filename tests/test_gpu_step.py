@@ -233,3 +233,32 @@ def test_step_single_long_segment():
             mx, mean = errors(from_dev(out[n]), expect)
             assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
         cache.sync_status()
+
+
+@pytest.mark.parametrize("b,g,L,grid,tile", [
+    (128, 2, 512, 128, 128),    # 256 segments of 4 tiles of 128: 128 CTAs of two segments
+    (64, 4, 4352, 64, 256),     # 256 segments of 17 tiles of 256: 64 CTAs of four segments
+])
+def test_step_whole_segments_per_cta(b, g, L, grid, tile):
+    # Inside a step the later layers run whole segments per CTA, several per CTA here: each later
+    # segment's queries arrive with its first tile.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, d = [0, 0, 0], 12, 64
+    lens = np.full(b, L, dtype=np.int32)
+    with mlkv.MLKVCache(len(owner), h, d, owner, g, b, L) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, L)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 71, cache, ref)
+        out = torch.full((len(owner), b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cache.decode_step(to_dev(qb), to_dev(kn), to_dev(vn), out, lens)
+        torch.cuda.synchronize()
+        assert cache.get_option("last_grid") == grid
+        assert cache.get_option("last_tile_tokens") == tile
+        assert cache.get_option("last_cluster_k") == 0
+        ref.append(0, gen.bf16_bits_to_f64(kn[0]), gen.bf16_bits_to_f64(vn[0]), lens)
+        for n in range(len(owner)):
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
+            mx, mean = errors(from_dev(out[n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
