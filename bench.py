@@ -285,6 +285,10 @@ def run(args, w):
         cache.set_option("cluster", args.cluster)
     if args.l2_persist:
         cache.set_option("l2_persist", 1)
+    if args.l2_prefetch >= 0:
+        cache.set_option("l2_prefetch", args.l2_prefetch)
+    if args.step_kernel >= 0:
+        cache.set_option("step_kernel", args.step_kernel)
     if args.no_pdl:
         cache.set_option("pdl", 0)
     cache.set_option("tc", args.tc)
@@ -305,7 +309,9 @@ def run(args, w):
 
     step()
     cache.sync_status()
-    launches_per_step = w.l * (2 if cache.get_option("last_deferred_merge") else 1)
+    step_kernel = bool(cache.get_option("last_step_kernel"))   # one launch for every layer
+    launches_per_step = 1 if step_kernel else (
+        w.l * (2 if cache.get_option("last_deferred_merge") else 1))
 
     def barrier():
         if dist is not None:
@@ -356,10 +362,20 @@ def run(args, w):
     alg_bytes = kv_layer + qo_layer
     peak, peak_kind = _peaks()
     achieved = alg_bytes / (mean_kernel_ms / 1e3) / 1e9
+    # per launch: one layer, or every layer when the step is one multi-layer launch (the ratio
+    # of bytes to time is the same)
+    launch_bytes = alg_bytes * (w.l if step_kernel else 1)
+    launch_ms = ms if step_kernel else mean_kernel_ms
+    # The step's floor in DRAM bytes: every owner slot's visible rows once (the later layers of a
+    # block could read them from L2), every layer's queries and outputs once.
+    unique_bytes = len(w.owners()) * kv_layer + w.l * qo_layer
+    unique_gbs = unique_bytes / (ms / 1e3) / 1e9
     cold = [layer_ms[n] for n in range(w.l) if w.owner[n] == n]
     cold_gbs = alg_bytes / (statistics.mean(cold) / 1e3) / 1e9
     del big_flush
     kernel_name = "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel"
+    options = {k: int(cache.get_option(k)) for k in ("l2_prefetch", "l2_persist", "tc",
+                                                      "step_kernel")}
     traffic = _recorded_traffic(w, kernel_name)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
@@ -408,9 +424,15 @@ def run(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind,
-                         "kernel": kernel_name, "alg_bytes_per_launch": alg_bytes,
-                         "mean_launch_ms": mean_kernel_ms,
+                         "frac_vs_8tbs": achieved / 8000.0,
+                         "kernel": kernel_name, "alg_bytes_per_launch": launch_bytes,
+                         "mean_launch_ms": launch_ms, "launches_per_step": launches_per_step,
+                         "step_ms_per_layer": mean_kernel_ms,
+                         "dram_unique_bytes_per_step": unique_bytes,
+                         "dram_unique_gbs": unique_gbs,
+                         "dram_frac_step": unique_gbs / peak,
                          "owner_launch_gbs": cold_gbs, "owner_launch_frac": cold_gbs / peak},
+            "options": options,
             "step_kv_gbs": kv_layer * w.l / (ms / 1e3) / 1e9,
             "layer_ms": layer_ms,
             "clocks": clocks.summary(),
@@ -713,6 +735,10 @@ def main():
     ap.add_argument("--cluster", type=int, default=-1, choices=[-1, 0, 1, 2, 4],
                     help="decode 'cluster' option (-1: the library default)")
     ap.add_argument("--l2-persist", action="store_true")
+    ap.add_argument("--l2-prefetch", type=int, default=-1, choices=[-1, 0, 1],
+                    help="option l2_prefetch (-1: the library's default)")
+    ap.add_argument("--step-kernel", type=int, default=-1, choices=[-1, 0, 1],
+                    help="option step_kernel (-1: the library's default)")
     ap.add_argument("--no-pdl", action="store_true")
     ap.add_argument("--tc", type=int, default=0, choices=[0, 1],
                     help="0: the mma.sync decode kernel (default); 1: the tcgen05 kernel")

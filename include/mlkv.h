@@ -212,8 +212,28 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  0 (default) picks per call: the longer tile when the mean length is >= 512,
  *                  except 128 for d=64 when batch x kv_heads >= 32 and the mean length <= 4096
  *   "grid"         persistent CTA count; 0 = one wave of resident CTAs (default)
- *   "l2_persist"   1 = give each decode launch an L2 access-policy window over its owner's slot
- *                  (default 0)
+ *   "l2_persist"   1 = keep part of each owner's slot in L2 for the later layers of its block:
+ *                  switching it on reserves the device's largest persisting-L2 set-aside for this
+ *                  process's CUDA context (cudaLimitPersistingL2CacheSize; the limit belongs to
+ *                  the context, so other work in the process sees the smaller normal L2 too), and
+ *                  every decode launch then reads its owner's slot through an access-policy
+ *                  window over the slot's first bytes (at most the device's window size) whose
+ *                  persisting share is set-aside / window; the last layer of a block marks its
+ *                  hits normal again.  Switching it off (or destroying the cache) resets the
+ *                  persisting lines and restores the earlier set-aside.  MLKV_ERR_UNSUPPORTED
+ *                  where the device has no set-aside.  Default 0 (see the design notes for the
+ *                  measurements behind the default).
+ *   "l2_prefetch"  1 = when mlkv_decode_step runs as one multi-layer launch (see "step_kernel")
+ *                  and the visible K/V rows of all owner slots fit in 5/8 of L2, every CTA first
+ *                  prefetches its share of them into L2 (cp.async.bulk.prefetch); 0 (default) = no
+ *                  prefetch, measured faster on GB300.  Results are identical.
+ *   "step_kernel"  1 (default) = mlkv_decode_step issues the whole step as one launch of the
+ *                  decode kernel over every (layer, sequence, KV head) item when every sequence
+ *                  has one length, the tcgen05 kernel, a fixed grid and l2_persist (whose windows
+ *                  are per layer) are off, the model has at
+ *                  most 128 layers and the estimated makespan is no longer than per-layer
+ *                  launches' (a few long segments, e.g. batch 1 at long context, keep per-layer
+ *                  launches); 0 = always one launch per layer.  Same results within the tolerance.
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through
@@ -231,7 +251,10 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  * Read-only (mlkv_get_option): "sm_count", "l2_bytes", "max_grid", "ctas_per_sm", and for the most
  * recent decode launch "last_grid", "last_tile_tokens", "last_cluster_k" (0 = global merge),
  * "last_deferred_merge", "last_tc" (1 if it ran the tcgen05 kernel), and "step_graph_replays"
- * (graph launches by mlkv_decode_step).
+ * (graph launches by mlkv_decode_step), "l2_persist_bytes" (the set-aside reserved while
+ * l2_persist is on, else 0), "l2_window_max" (the device's largest access-policy window),
+ * "last_step_kernel" (1 if the most recent mlkv_decode_step ran as one multi-layer launch) and
+ * "last_l2_prefetch" (1 if that launch prefetched the slots into L2).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.
  */
 int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);
@@ -280,6 +303,22 @@ int mlkv_block_owner_map(int n_layers, int n_owners, int *layer_owner);
 int mlkv_decode_attention_static(const void *kv_slot, int batch, int n_q_heads, int kv_heads,
                                  int head_dim, int max_seq, const void *Q, void *out,
                                  const int *seq_lens, void *cuda_stream);
+
+/*
+ * mlkv_static_status - the error record of mlkv_decode_attention_static on the current device.
+ * The paper has no counterpart (see mlkv_decode_attention_static).
+ *
+ * The kernels of mlkv_decode_attention_static report an expired bounded wait (see
+ * mlkv_sync_status) by setting bits of an error word inside the library's static scratch array;
+ * the word is cleared once when a device is set up and then keeps every bit set since.  This call
+ * waits for cuda_stream (a cudaStream_t, NULL = legacy default stream) to finish, reads the word,
+ * clears it if it is non-zero, and returns MLKV_ERR_DEVICE if it was (mlkv_last_error gives the
+ * bits), MLKV_ERR_CUDA if the stream reported a CUDA error, else MLKV_OK.  It allocates nothing.
+ * Call it after the static calls whose status matters have been queued on cuda_stream (with
+ * several streams, after all of them have finished); the first call on a device sets the device
+ * up as mlkv_decode_attention_static does, so make it outside any stream capture.
+ */
+int mlkv_static_status(void *cuda_stream);
 
 /*
  * mlkv_decode_block_fused - decode attention of every layer of one owner block in one launch:

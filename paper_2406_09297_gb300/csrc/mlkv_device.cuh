@@ -217,11 +217,35 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 // the per-sequence tables, which the kernel copies from its parameters into shared memory.
 template <int T>
 struct TileWalk {
-    int beta, j, tt, nt, L, seg_first;
+    int beta, j, tt, nt, L, seg_first, layer, item;
 
+    // Multi-layer launch: (layer, beta, j) of item `item`.
+    __device__ __forceinline__ void set_item(const DecodeParams &p)
+    {
+        const int S = p.b * p.g;
+        layer = item / S;
+        const int seg = item - layer * S;
+        beta = seg / p.g;
+        j = seg - beta * p.g;
+    }
+
+    // `tile`: the flattened tile of a single-layer launch, or the CTA's own tile count in a
+    // multi-layer launch (its k-th item is item blockIdx.x + k gridDim.x).
     __device__ __forceinline__ void init(const DecodeParams &p, const int *s_len,
                                          const int *s_start, int tile)
     {
+        if (p.ml_layers > 0) {
+            L = p.uniform_len;
+            nt = (L + T - 1) / T;
+            const int k = tile / nt;
+            tt = tile - k * nt;
+            item = static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x);
+            seg_first = k * nt;
+            set_item(p);
+            return;
+        }
+        layer = 0;
+        item = 0;
         if (p.uniform_len > 0) {
             L = p.uniform_len;
             nt = (L + T - 1) / T;
@@ -255,6 +279,12 @@ struct TileWalk {
         if (++tt < nt)
             return;
         tt = 0;
+        if (p.ml_layers > 0) {
+            item += static_cast<int>(gridDim.x);
+            seg_first += nt;
+            set_item(p);
+            return;
+        }
         if (p.uniform_len > 0) {
             seg_first += nt;
             if (++j == p.g) {
@@ -280,6 +310,34 @@ __device__ __forceinline__ int cta_of_tile(int tile, int N, int P)
     return static_cast<int>((static_cast<long long>(tile + 1) * P - 1) / N);
 }
 
+
+// Multi-layer launch with every sequence of one length: CTA `cta` of `P` prefetches into L2 its
+// 1/P share of the visible rows (positions [0, L)) of every (slot, K|V, beta, j) row of slots
+// 0 .. ml_slots - 1, slot by slot, so that the whole step's K/V streams from HBM at the copy
+// engines' rate while the CTAs work.  Shares are 128-byte aligned; chunks of at most 1 MiB.
+template <int D>
+__device__ __forceinline__ void prefetch_slots_share(const DecodeParams &p, int cta, int P)
+{
+    const size_t row_bytes = static_cast<size_t>(p.uniform_len) * D * 2;
+    const size_t rows = 2ull * p.b * p.g;                  // rows of one slot
+    const size_t slot_bytes = rows * row_bytes;
+    const size_t pitch = static_cast<size_t>(p.max_seq) * D * 2;
+    const uint8_t *base = reinterpret_cast<const uint8_t *>(p.cache);
+    for (int s = 0; s < p.ml_slots; ++s) {
+        size_t lo = (slot_bytes * cta / P) & ~static_cast<size_t>(127);
+        const size_t hi =
+            cta + 1 == P ? slot_bytes : (slot_bytes * (cta + 1) / P) & ~static_cast<size_t>(127);
+        while (lo < hi) {
+            const size_t r = lo / row_bytes;
+            const size_t off = lo - r * row_bytes;
+            size_t n = min(hi - lo, row_bytes - off);
+            n = min(n, static_cast<size_t>(1u << 20));
+            bulk_prefetch_l2(base + (static_cast<size_t>(s) * rows + r) * pitch + off,
+                             static_cast<uint32_t>(n));
+            lo += n;
+        }
+    }
+}
 
 // the TMA 128-byte swizzle: the chunk index within a 128-byte row is XORed with (row mod 8).
 template <int T>
@@ -373,7 +431,8 @@ __device__ __forceinline__ unsigned atomic_add_acq_rel_gpu(unsigned *addr, unsig
     return old;
 }
 
-enum : int { kMetaBeta = 0, kMetaJ, kMetaSeg, kMetaWhole, kMetaFirst, kMetaLast, kMetaStop };
+enum : int { kMetaBeta = 0, kMetaJ, kMetaSeg, kMetaWhole, kMetaFirst, kMetaLast, kMetaStop,
+             kMetaLayer };
 
 // ------------------------------------------------------------------------------------------------
 // epilogue warp: output, partials and the cross-CTA merge of finished pieces
@@ -390,7 +449,8 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
 {
     const int G = p.G;
     const int beta = meta[kMetaBeta], j = meta[kMetaJ], seg = meta[kMetaSeg];
-    __nv_bfloat16 *ob = p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+    __nv_bfloat16 *ob = p.out + static_cast<size_t>(meta[kMetaLayer]) * p.ml_q_stride +
+                        (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
     if (meta[kMetaWhole]) {
         for (int i = lane * 4; i < G * D; i += 128) {
             const float4 v = *reinterpret_cast<const float4 *>(ro + i);

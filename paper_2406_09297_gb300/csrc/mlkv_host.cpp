@@ -113,6 +113,11 @@ struct mlkv_cache {
     int tile_tokens = 0;
     int grid = 0;
     int l2_persist = 0;
+    size_t persist_bytes = 0;   // the context's persisting-L2 set-aside while l2_persist is on
+    size_t persist_prev = 0;    // the set-aside before l2_persist was switched on
+    int l2_prefetch = 0;        // multi-layer step: prefetch the step's slots into L2 when they fit
+    int step_kernel = 1;        // mlkv_decode_step: one multi-layer launch where it applies
+    int last_step_kernel = 0;   // 1 if the most recent step ran as one multi-layer launch
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
@@ -128,12 +133,12 @@ struct mlkv_cache {
         const void *Q = nullptr, *K = nullptr, *V = nullptr;
         void *out = nullptr;
         std::vector<int> lens;
-        int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1, tc = -1;
+        int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1, tc = -1, pf = -1, sk = -1;
         bool operator==(const StepKey &o) const
         {
             return Q == o.Q && K == o.K && V == o.V && out == o.out && lens == o.lens &&
                    tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
-                   l2 == o.l2 && tc == o.tc;
+                   l2 == o.l2 && tc == o.tc && pf == o.pf && sk == o.sk;
         }
     } step_key, pending_key;   // recorded arguments; arguments seen once, not yet recorded
     int step_graph_replays = 0;
@@ -145,6 +150,7 @@ struct mlkv_cache {
     StepKey host_key, host_pending;
     // the most recent decode launch (read-only options, for tests and tuning)
     int last_grid = 0, last_tile = 0, last_cluster_k = 0, last_deferred = 0, last_tc = 0;
+    int last_l2_prefetch = 0;
     // per-variant launch state
     struct Variant {
         const mlkv::DecodeVariant *v = nullptr;
@@ -173,27 +179,11 @@ int check_seq_lens(const mlkv_cache *c, const int *seq_lens)
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Longer tiles move more bytes per TMA request and per barrier round trip; shorter ones waste less
-// on short sequences.  For d = 64 the 128-position variant is small enough for two CTAs per SM,
-// so the next layer's CTAs start (and fetch) while this layer's last ones finish: measured faster
-// for many segments of moderate length (64 x 2048: 85 vs 89 us a step; 512 x ~2048: 527 vs 560),
-// slower for few long segments or HBM-bound layers (1 x 131072, 256 x 8192).  mean_len < 0 means
-// "unknown" (reports the long-sequence choice).
-int default_tile_tokens(int d, double mean_len, int segments)
-{
-    if (d == 64) {
-        if (mean_len >= 0 && (mean_len < 512 || (segments >= 32 && mean_len <= 4096)))
-            return 128;
-        return 256;
-    }
-    return (mean_len < 0 || mean_len >= 512) ? 128 : 64;
-}
-
 mlkv_cache::Variant *pick_variant(mlkv_cache *c, double mean_len = -1.0, int force_T = 0)
 {
     const int T = force_T > 0            ? force_T
                   : c->tile_tokens > 0 ? c->tile_tokens
-                                       : default_tile_tokens(c->d, mean_len, c->b * c->g);
+                                       : mlkv::default_tile_tokens(c->d, mean_len, c->b * c->g);
     mlkv_cache::Variant *plain = nullptr;
     for (auto &v : c->variants) {
         if (v.v->tile_tokens != T)
@@ -415,6 +405,11 @@ int mlkv_cache_destroy(mlkv_cache_t c)
         return MLKV_OK;
     DeviceGuard guard(c->device);
     cudaDeviceSynchronize();
+    if (c->l2_persist) {
+        cudaCtxResetPersistingL2Cache();
+        cudaDeviceSetLimit(cudaLimitPersistingL2CacheSize, c->persist_prev);
+        cudaGetLastError();
+    }
     if (c->step_exec)
         cudaGraphExecDestroy(c->step_exec);
     if (c->host_exec)
@@ -647,14 +642,29 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                            ? 1
                            : 0;
 
+    p.pf_own = 0;
+    p.ml_layers = 0;
+    p.ml_slots = 0;
+    p.ml_q_stride = 0;
+    p.ml_kv_stride = 0;
+
+    // L2 persistence (option l2_persist): every layer of an owner's block reads the slot through
+    // an access-policy window over the slot's first bytes (at most the device's window size),
+    // persisting as large a share of it as the set-aside holds (hitRatio = set-aside / window),
+    // so the lines the owner layer brings in stay for the block's later layers.  The block's last
+    // layer marks its hits normal again, which frees the set-aside for the next block's owner.
     cudaAccessPolicyWindow win = {};
     const cudaAccessPolicyWindow *winp = nullptr;
-    if (c->l2_persist && c->window_max > 0) {
+    if (c->l2_persist && c->window_max > 0 && c->persist_bytes > 0) {
         const size_t slot_bytes = c->cache_bytes / c->m;
         win.base_ptr = static_cast<char *>(c->cache) + slot_bytes * p.slot;
         win.num_bytes = std::min<size_t>(slot_bytes, static_cast<size_t>(c->window_max));
-        win.hitRatio = 1.0f;
-        win.hitProp = cudaAccessPropertyPersisting;
+        win.hitRatio = static_cast<float>(
+            std::min(1.0, static_cast<double>(c->persist_bytes) / win.num_bytes));
+        bool last_of_block = true;
+        for (int k = layer + 1; k < c->l; ++k)
+            last_of_block = last_of_block && c->owner[k] != c->owner[layer];
+        win.hitProp = last_of_block ? cudaAccessPropertyNormal : cudaAccessPropertyPersisting;
         win.missProp = cudaAccessPropertyStreaming;
         winp = &win;
     }
@@ -676,6 +686,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     c->last_cluster_k = cluster_k;
     c->last_tc = var->v->tc;
     c->last_deferred = p.deferred_merge;
+    c->last_l2_prefetch = 0;
     return MLKV_OK;
 }
 
@@ -697,13 +708,115 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
     return decode_impl(c, layer, nullptr, nullptr, Q, out, seq_lens, cuda_stream);
 }
 
-// The layer calls of one decode step, issued on `stream`.
+// The whole decode step as one launch of the decode kernel over every (layer, segment) item
+// (DecodeParams::ml_layers), where that applies: every sequence has one length, the mma.sync
+// kernel, default grid, no L2-persistence windows (they are per layer), at most kMaxStepLayers
+// layers, and a makespan no longer than the
+// per-layer launches' (below).  Items are whole segments, so nothing is merged and no
+// scratch is shared; every layer takes its segments' newest rows from the step's new tokens,
+// and owner layers store them.  *done tells whether it was issued.  With in_ready, the launch
+// waits for it (queries still arriving).
+static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
+                         const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done)
+{
+    *done = false;
+    c->last_step_kernel = 0;
+    if (!c->step_kernel || c->tc || c->grid > 0 || c->l2_persist || c->l > mlkv::kMaxStepLayers)
+        return MLKV_OK;
+    for (int beta = 1; beta < c->b; ++beta)
+        if (seq_lens[beta] != seq_lens[0])
+            return MLKV_OK;
+    const int L = seq_lens[0];
+    mlkv_cache::Variant *var = pick_variant(c, static_cast<double>(L));
+    if (var == nullptr || var->v->tc)
+        return MLKV_OK;
+    const int T = var->v->tile_tokens;
+    const long long nt = (L + T - 1) / T;
+    const long long S = static_cast<long long>(c->b) * c->g;
+    const long long items = c->l * S;
+    const long long slots = static_cast<long long>(var->ctas_per_sm) * c->sm_count;
+    // Makespans in tiles: one launch gives each CTA ceil(items / slots) whole segments; per-layer
+    // launches split every layer over the machine but pay a launch, a ramp and merges per layer
+    // (about 4 tiles' time each; they overlap only in part).  A few long segments (batch 1 at
+    // long context) stay with the per-layer split.
+    const long long per = (items + slots - 1) / slots;
+    if (per * nt > c->l * ((S * nt + slots - 1) / slots + 4) || items * nt > 0x7fffffffLL)
+        return MLKV_OK;
+    const int grid = static_cast<int>((items + per - 1) / per);
+
+    static thread_local mlkv::DecodeParams p;
+    p.Q = reinterpret_cast<const __nv_bfloat16 *>(Q);
+    p.out = reinterpret_cast<__nv_bfloat16 *>(out);
+    p.K_new = reinterpret_cast<const __nv_bfloat16 *>(K);
+    p.V_new = reinterpret_cast<const __nv_bfloat16 *>(V);
+    p.cache = static_cast<__nv_bfloat16 *>(c->cache);
+    p.max_seq = c->max_seq;
+    p.part_o = c->part_o;
+    p.part_lse = c->part_lse;
+    p.counters = c->counters;
+    p.err = c->err;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
+    p.b = c->b;
+    p.h = c->h;
+    p.g = c->g;
+    p.G = c->G;
+    p.slot = 0;
+    p.num_tiles = static_cast<int>(items * nt);
+    p.uniform_len = L;
+    p.cluster_k = 0;
+    p.deferred_merge = 0;
+    p.tile_tokens = T;
+    p.decode_grid = grid;
+    p.Q_next = nullptr;
+    p.early_fetch = 0;
+    p.newest_ready = 1;
+    p.store_new = 0;
+    // L2 prefetch of every slot's visible rows when they all fit with room to spare.
+    const long long all_kv = static_cast<long long>(c->m) * 2 * c->b * c->g * L * c->d * 2;
+    p.pf_own = (c->l2_prefetch && all_kv <= static_cast<long long>(c->l2_bytes) * 5 / 8) ? 1 : 0;
+    p.ml_slots = c->m;
+    p.ml_layers = c->l;
+    p.ml_q_stride = static_cast<long long>(c->b) * c->h * c->d;
+    p.ml_kv_stride = static_cast<long long>(c->b) * c->g * c->d;
+    for (int n = 0; n < c->l; ++n) {
+        p.ml_slot[n] = static_cast<unsigned char>(c->slot[n]);
+        p.ml_store[n] = c->owner[n] == n ? 1 : 0;
+    }
+    cudaError_t e = cudaSuccess;
+    if (in_ready != nullptr)
+        e = cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), in_ready, 0);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "step event");
+    DeviceGuard guard(c->device);
+    e = mlkv::launch_decode(*var->v, grid, var->v->smem_bytes, static_cast<cudaStream_t>(stream),
+                            &var->tmap, &var->tmap_rows, p, nullptr, c->pdl != 0);
+    if (e != cudaSuccess)
+        return fail_cuda(e, "decode launch (multi-layer step)");
+    c->last_grid = grid;
+    c->last_tile = T;
+    c->last_cluster_k = 0;
+    c->last_tc = 0;
+    c->last_deferred = 0;
+    c->last_l2_prefetch = p.pf_own;
+    c->last_step_kernel = 1;
+    *done = true;
+    return MLKV_OK;
+}
+
+// The layer calls of one decode step, issued on `stream` (one multi-layer launch where
+// issue_step_ml applies).
 // With in_ready, layer 1 onwards waits for it (the later layers' queries still arriving); with
 // before_last, it is recorded once every layer but the last has been issued.
 static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
                       const int *seq_lens, void *stream, cudaEvent_t in_ready = nullptr,
                       cudaEvent_t before_last = nullptr)
 {
+    if (before_last == nullptr) {
+        bool done = false;
+        const int rc = issue_step_ml(c, Q, K, V, out, seq_lens, stream, in_ready, &done);
+        if (rc != MLKV_OK || done)
+            return rc;
+    }
     const size_t qo = static_cast<size_t>(c->b) * c->h * c->d * 2;   // bytes of one layer's Q
     const size_t kv = static_cast<size_t>(c->b) * c->g * c->d * 2;   // one owner's new token
     for (int n = 0; n < c->l; ++n) {
@@ -759,6 +872,8 @@ mlkv_cache::StepKey step_key_of(const mlkv_cache *c, const void *Q, const void *
     key.pdl = c->pdl;
     key.tc = c->tc;
     key.l2 = c->l2_persist;
+    key.pf = c->l2_prefetch;
+    key.sk = c->step_kernel;
     return key;
 }
 
@@ -1400,7 +1515,48 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
     if (std::strcmp(key, "l2_persist") == 0) {
         if (value != 0 && value != 1)
             return fail(MLKV_ERR_INVALID_ARG, "l2_persist must be 0 or 1");
+        if (value == c->l2_persist)
+            return MLKV_OK;
+        DeviceGuard guard(c->device);
+        cudaError_t e;
+        if (value == 1) {
+            // Reserve the largest persisting-L2 set-aside the device allows for this process's
+            // context (a per-context limit that ends with the context; no device setting changes).
+            int max_persist = 0;
+            e = cudaDeviceGetAttribute(&max_persist, cudaDevAttrMaxPersistingL2CacheSize, c->device);
+            if (e != cudaSuccess)
+                return fail_cuda(e, "cudaDeviceGetAttribute(MaxPersistingL2CacheSize)");
+            if (max_persist <= 0 || c->window_max <= 0)
+                return fail(MLKV_ERR_UNSUPPORTED, "the device has no persisting L2 set-aside");
+            size_t prev = 0, now = 0;
+            if ((e = cudaDeviceGetLimit(&prev, cudaLimitPersistingL2CacheSize)) != cudaSuccess ||
+                (e = cudaDeviceSetLimit(cudaLimitPersistingL2CacheSize,
+                                        static_cast<size_t>(max_persist))) != cudaSuccess ||
+                (e = cudaDeviceGetLimit(&now, cudaLimitPersistingL2CacheSize)) != cudaSuccess)
+                return fail_cuda(e, "cudaLimitPersistingL2CacheSize");
+            c->persist_prev = prev;
+            c->persist_bytes = now;
+        } else {
+            // Lines still marked persisting go back to normal; the earlier set-aside returns.
+            if ((e = cudaCtxResetPersistingL2Cache()) != cudaSuccess ||
+                (e = cudaDeviceSetLimit(cudaLimitPersistingL2CacheSize, c->persist_prev)) !=
+                    cudaSuccess)
+                return fail_cuda(e, "restoring the persisting L2 set-aside");
+            c->persist_bytes = 0;
+        }
         c->l2_persist = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_prefetch") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "l2_prefetch must be 0 or 1");
+        c->l2_prefetch = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "step_kernel") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "step_kernel must be 0 or 1");
+        c->step_kernel = static_cast<int>(value);
         return MLKV_OK;
     }
     if (std::strcmp(key, "cluster") == 0) {
@@ -1444,6 +1600,30 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "l2_persist") == 0) {
         *value = c->l2_persist;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_persist_bytes") == 0) {
+        *value = static_cast<int64_t>(c->persist_bytes);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_window_max") == 0) {
+        *value = c->window_max;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "l2_prefetch") == 0) {
+        *value = c->l2_prefetch;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "step_kernel") == 0) {
+        *value = c->step_kernel;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_step_kernel") == 0) {
+        *value = c->last_step_kernel;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_l2_prefetch") == 0) {
+        *value = c->last_l2_prefetch;
         return MLKV_OK;
     }
     if (std::strcmp(key, "cluster") == 0) {

@@ -18,6 +18,9 @@ enum : int {
     kErrDrain = 4,      // the producer gave up waiting for its last copies at exit
 };
 
+// Layers one multi-layer decode launch can cover (DecodeParams::ml_layers).
+constexpr int kMaxStepLayers = 128;
+
 // Split-KV decode of one layer.  Passed by value (__grid_constant__), so a launch needs no
 // device-side metadata and is stream-ordered and graph-capturable by construction.
 struct DecodeParams {
@@ -49,6 +52,20 @@ struct DecodeParams {
     int store_new;            // with K_new: 1 = also store the new token in the cache (the owner
                               // layer's fused append); 0 = only replace the tiles' newest rows (a
                               // later layer of the block, whose owner's launch stores the token)
+    int pf_own;               // multi-layer launch: 1 = prefetch the step's slots into L2
+    // Multi-layer launch (ml_layers > 0, every sequence of one length): one grid covers every
+    // (layer, segment) item of a decode step, item i = layer * b g + beta g + j, each a whole
+    // segment, CTA c taking items c, c + P, c + 2P, ...  Q and out then hold every layer
+    // ([layer][b][h][D], ml_q_stride elements apart) and K_new / V_new every owner's new token
+    // ([slot][b][g][D], ml_kv_stride elements apart); layer n reads slot ml_slot[n], and stores
+    // its new token in the cache if ml_store[n] (an owner layer), else only replaces its tiles'
+    // newest rows with it.  slot, store_new and Q_next are unused; pf_own = 1 has every CTA
+    // prefetch its share of the visible rows of all ml_slots slots into L2 at the start.
+    int ml_layers;
+    int ml_slots;             // owner slots the step reads (with pf_own: all prefetched into L2)
+    long long ml_q_stride, ml_kv_stride;
+    unsigned char ml_slot[kMaxStepLayers];
+    unsigned char ml_store[kMaxStepLayers];
     int seq_len[MLKV_MAX_BATCH];
     int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
 };
@@ -154,6 +171,24 @@ cudaError_t launch_decode(const DecodeVariant &v, int grid, size_t smem, cudaStr
                           const CUtensorMap *tmap, const CUtensorMap *tmap_rows,
                           const DecodeParams &p, const cudaAccessPolicyWindow *window,
                           bool pdl = true);
+
+// Default positions per tile of the mma.sync decode kernel for a launch over `segments`
+// (sequence, KV head) pairs of mean length mean_len.  Longer tiles move more bytes per TMA
+// request and per barrier round trip; shorter ones waste less on short sequences.  For d = 64 the
+// 128-position variant is small enough for two CTAs per SM, so the next layer's CTAs start (and
+// fetch) while this layer's last ones finish: measured faster for many segments of moderate
+// length (64 x 2048: 85 vs 89 us a step; 512 x ~2048: 527 vs 560), slower for few long segments
+// or HBM-bound layers (1 x 131072, 256 x 8192).  mean_len < 0 means "unknown" (reports the
+// long-sequence choice).
+inline int default_tile_tokens(int d, double mean_len, int segments)
+{
+    if (d == 64) {
+        if (mean_len >= 0 && (mean_len < 512 || (segments >= 32 && mean_len <= 4096)))
+            return 128;
+        return 256;
+    }
+    return (mean_len < 0 || mean_len >= 512) ? 128 : 64;
+}
 
 // Sets the calling thread's mlkv_last_error() text.
 void set_last_error(const char *msg);

@@ -51,7 +51,7 @@ namespace {
 template <int D, int T, int STAGES, int NCW>
 struct Plan {
     static constexpr int kThreads = (NCW + 2) * 32;   // consumers, one producer, one epilogue warp
-    // Variants whose ring fits twice in an SM's shared memory ask for two resident CTAs.
+    // Variants whose ring fits twice in an SM's shared memory are sized for two resident CTAs.
     static constexpr int kMinBlocks = (STAGES * 2 * T * D * 2 <= 80 * 1024) ? 2 : 1;
     static constexpr int kProducer = NCW;             // warp indices
     static constexpr int kEpilogue = NCW + 1;
@@ -96,12 +96,12 @@ struct Plan {
 // S = Q K^T in the mma.m16n8k16 layout, rows >= G (the padding of the group to 16 rows) zero.
 template <int D>
 __device__ __forceinline__ void load_q_frag(uint32_t (&qa)[D / 16][4], const DecodeParams &p,
-                                            int beta, int j, int lane)
+                                            const __nv_bfloat16 *Q, int beta, int j, int lane)
 {
     const int G = p.G;
     const int qr = lane >> 2, qc = (lane & 3) * 2;
     const __nv_bfloat16 *qb =
-        p.Q + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+        Q + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
     const bool r0 = qr < G, r1 = qr + 8 < G;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
@@ -169,14 +169,36 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     const int cta = blockIdx.x;
     const int N = p.num_tiles;
     // floor(c N / P) in 32 bits when c N fits (a 64-bit division costs ~0.1 us at CTA start).
+    // A multi-layer launch numbers each CTA's own tiles from 0: its items c, c + P, ... (whole
+    // segments of nt tiles each).
+    const bool ml = p.ml_layers > 0;
     const bool narrow = static_cast<long long>(P) * N < (1ll << 32);
-    const int tile_lo = narrow ? static_cast<int>(static_cast<uint32_t>(cta) * N / P)
-                               : static_cast<int>(static_cast<long long>(cta) * N / P);
-    const int tile_hi = narrow ? static_cast<int>(static_cast<uint32_t>(cta + 1) * N / P)
-                               : static_cast<int>(static_cast<long long>(cta + 1) * N / P);
+    int tile_lo, tile_hi;
+    if (ml) {
+        const int items = p.ml_layers * p.b * p.g;
+        const int nt = (p.uniform_len + T - 1) / T;
+        tile_lo = 0;
+        tile_hi = (cta < items ? (items - 1 - cta) / P + 1 : 0) * nt;
+    } else {
+        tile_lo = narrow ? static_cast<int>(static_cast<uint32_t>(cta) * N / P)
+                         : static_cast<int>(static_cast<long long>(cta) * N / P);
+        tile_hi = narrow ? static_cast<int>(static_cast<uint32_t>(cta + 1) * N / P)
+                         : static_cast<int>(static_cast<long long>(cta + 1) * N / P);
+    }
+    // Per-layer pointers: a multi-layer launch reads layer `layer`'s queries, writes its outputs,
+    // reads its owner's slot and new token; a single-layer launch has one of each.
+    auto q_of = [&](int layer) {
+        return ml ? p.Q + static_cast<size_t>(layer) * p.ml_q_stride : p.Q;
+    };
+    auto slot_of = [&](int layer) { return ml ? static_cast<int>(p.ml_slot[layer]) : p.slot; };
 
     const bool early = p.early_fetch != 0;
-    // The producer's copy of one tile into stage `s` (query rows too when a later piece starts).
+    // The producer warp's copy of one tile into stage `s` (query rows too when a later piece
+    // starts); called by all 32 lanes with the same arguments.  On GB300 one issuing thread
+    // completes about one bulk copy per ~0.5 us whatever its size (measured: 8 to 64 KB, from L2
+    // or HBM, 2 to 8 copies outstanding), while copies from different lanes proceed side by side;
+    // so the copies of a tile -- K and V boxes, query rows -- go out from different lanes, and
+    // successive stages from different groups of lanes.  Lane 0 first announces the stage's bytes.
     auto issue_tile = [&](const TileWalk<T> &w, int s, bool with_q) {
         const uint32_t fb = bar_full + 8 * s;
         const uint32_t qbytes = static_cast<uint32_t>(p.G) * D * 2;
@@ -187,37 +209,38 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         const int nbox = vis < T ? (vis + 63) / 64 : 0;
         const uint32_t kv_bytes =
             nbox > 0 ? static_cast<uint32_t>(nbox) * 64u * D * 2u * 2u : PL::kStageBytes;
-        mbar_arrive_expect_tx(fb, kv_bytes + (with_q ? qbytes : 0u));
-        if (with_q) {
-            const __nv_bfloat16 *q0 = p.Q + (static_cast<size_t>(w.beta) * p.h +
-                                             static_cast<size_t>(w.j) * p.G) * D;
-            for (int r = 0; r < p.G; ++r)
-                bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2, fb);
-        }
-        const int zk = ((p.slot * 2 + 0) * p.b + w.beta) * p.g + w.j;
+        if (lane == 0)
+            mbar_arrive_expect_tx(fb, kv_bytes + (with_q ? qbytes : 0u));
+        __syncwarp();
+        // copy i of this tile goes out from lane (i + rot) mod 32
+        const int per_tile = 2 * PL::kSub * (nbox > 0 ? nbox : 1);
+        const int mine = (lane - s * 2 * PL::kSub) & 31;
+        const int zk = ((slot_of(w.layer) * 2 + 0) * p.b + w.beta) * p.g + w.j;
         const int zv = zk + p.b * p.g;
         const int y = w.tt * T;
         const uint32_t kdst = sbase + s * PL::kStageBytes;
         const uint32_t vdst = kdst + PL::kTileBytes;
-        if (nbox == 0) {
-#pragma unroll
-            for (int sub = 0; sub < PL::kSub; ++sub) {
-                tma_load_3d(kdst + sub * T * 128, &tmap, fb, sub * 64, y, zk);
-                tma_load_3d(vdst + sub * T * 128, &tmap, fb, sub * 64, y, zv);
-            }
-        } else {
-            for (int bx = 0; bx < nbox; ++bx) {
-#pragma unroll
-                for (int sub = 0; sub < PL::kSub; ++sub) {
-                    const uint32_t off = sub * T * 128 + bx * 64 * 128;
-                    tma_load_3d(kdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zk);
-                    tma_load_3d(vdst + off, &tmap_rows, fb, sub * 64, y + 64 * bx, zv);
-                }
-            }
+        if (mine < per_tile) {
+            // copy i: box bx = i / (2 kSub), then K or V, then the 64-column block
+            const int bx = mine / (2 * PL::kSub);
+            const int kv = (mine / PL::kSub) & 1;
+            const int sub = mine % PL::kSub;
+            const uint32_t dst = (kv ? vdst : kdst) + sub * T * 128 + bx * 64 * 128;
+            if (nbox == 0)
+                tma_load_3d(dst, &tmap, fb, sub * 64, y, kv ? zv : zk);
+            else
+                tma_load_3d(dst, &tmap_rows, fb, sub * 64, y + 64 * bx, kv ? zv : zk);
+        }
+        if (with_q) {
+            const __nv_bfloat16 *q0 = q_of(w.layer) + (static_cast<size_t>(w.beta) * p.h +
+                                                       static_cast<size_t>(w.j) * p.G) * D;
+            const int r = (mine - per_tile) & 31;
+            if (r < p.G)
+                bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2, fb);
         }
     };
-    // The ring's barriers belong to the producer lane.  With early fetch and one length for every
-    // sequence it also sends its first tile before the CTA barrier: a CTA that got its SM late
+    // The ring's barriers belong to the producer warp's lane 0.  With early fetch and one length
+    // for every sequence the warp also sends its first tile before the CTA barrier: a CTA that got its SM late
     // (the last ones of a layer decide the layer's end) then has data on the way at once.
     bool pre_issued = false;
     // The trigger comes first: the next launch (inside a decode step, the next layer's decode)
@@ -225,12 +248,17 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // dependency wait is fixed by p.early_fetch, and it finishes only after this grid.
     if (threadIdx.x == 0)
         grid_dependents_launch();
-    if (threadIdx.x == PL::kProducer * 32) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(bar_full + 8 * s, 1);
-            mbar_init(bar_empty + 8 * s, NCW);
+    if (warp == PL::kProducer) {
+        if (lane == 0) {
+            prefetch_tensormap(&tmap);   // kernel parameters: safe before the dependency wait
+            prefetch_tensormap(&tmap_rows);
+            for (int s = 0; s < STAGES; ++s) {
+                mbar_init(bar_full + 8 * s, 1);
+                mbar_init(bar_empty + 8 * s, NCW);
+            }
+            fence_barrier_init();
         }
-        fence_barrier_init();
+        __syncwarp();
         if (early && p.uniform_len > 0 && tile_lo < tile_hi) {
             TileWalk<T> w0;
             w0.init(p, s_len, s_start, tile_lo);
@@ -253,10 +281,6 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         }
         flags[0] = 0;   // abort
         fence_barrier_init();
-    }
-    if (threadIdx.x == PL::kProducer * 32) {
-        prefetch_tensormap(&tmap);   // kernel parameters: safe before the dependency wait
-        prefetch_tensormap(&tmap_rows);
     }
     if (p.uniform_len <= 0) {
         for (int i = threadIdx.x; i < p.b; i += blockDim.x) {
@@ -287,15 +311,18 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     // the queries cannot be the previous kernel's output; later pieces find theirs in a slot.
     uint32_t qa[KS][4];
     if (early && warp < NCW && tile_lo < tile_hi)
-        load_q_frag<D>(qa, p, wk.beta, wk.j, lane);
+        load_q_frag<D>(qa, p, q_of(wk.layer), wk.beta, wk.j, lane);
     if (warp != PL::kProducer && !early)
         grid_dependency_wait();
     if (warp == PL::kEpilogue && lane == 0)
         grid_dependency_wait();
 
     // -------------------------------- producer warp --------------------------------------------
+    // Every lane walks the same tiles; lane 0 waits (dependency, free stages) and announces each
+    // stage's bytes, and the copies go out from several lanes (issue_tile).
     if (warp == PL::kProducer) {
-        if (lane == 0) {
+        if (ml && p.pf_own && lane == 31)
+            prefetch_slots_share<D>(p, cta, P);
         int issued = pre_issued ? 1 : 0;
         int tile = tile_lo + issued;
         if (pre_issued)
@@ -305,8 +332,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             grid_dependency_wait();
         // The next layer's queries (an input of the whole step) go to L2 now: its CTAs load
         // them first thing, while this layer still streams.  Each CTA takes a 128-byte-aligned
-        // share.
-        if (p.Q_next != nullptr) {
+        // share.  Issued from the last lane, which issues no tile copies.
+        if (p.Q_next != nullptr && lane == 31) {
             const size_t qbytes = static_cast<size_t>(p.b) * p.h * D * 2;   // a multiple of 128
             const size_t lo = (qbytes * cta / P) & ~static_cast<size_t>(127);
             const size_t hi =
@@ -321,12 +348,16 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 waited = true;
             }
             const int s = issued % STAGES;
-            if (issued >= STAGES && !flags[0] &&
-                !mbar_wait(bar_empty + 8 * s, ((issued / STAGES) & 1) ^ 1)) {
-                flags[0] = 1;
-                atomicOr(p.err, kErrWaitEmpty);
+            int stop = 0;
+            if (lane == 0) {
+                if (issued >= STAGES && !flags[0] &&
+                    !mbar_wait(bar_empty + 8 * s, ((issued / STAGES) & 1) ^ 1)) {
+                    flags[0] = 1;
+                    atomicOr(p.err, kErrWaitEmpty);
+                }
+                stop = flags[0];
             }
-            if (flags[0])
+            if (__shfl_sync(0xffffffffu, stop, 0))
                 break;
             // A later piece starts here: its query rows come with the tile.
             issue_tile(wk, s, wk.tt == 0 && tile != tile_lo);
@@ -334,10 +365,11 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             wk.next(p, s_len, s_start);
         }
         // No copy may still be in flight when the CTA exits.
-        const int first = issued > STAGES ? issued - STAGES : 0;
-        for (int k = first; k < issued; ++k)
-            if (!mbar_wait(bar_full + 8 * (k % STAGES), (k / STAGES) & 1))
-                atomicOr(p.err, kErrDrain);
+        if (lane == 0) {
+            const int first = issued > STAGES ? issued - STAGES : 0;
+            for (int k = first; k < issued; ++k)
+                if (!mbar_wait(bar_full + 8 * (k % STAGES), (k / STAGES) & 1))
+                    atomicOr(p.err, kErrDrain);
         }
         __syncwarp();
         if (p.cluster_k > 1)
@@ -398,6 +430,15 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         const int j = wk.j;
         const int L = wk.L;
         const int seg = beta * p.g + j;
+        const int layer = wk.layer;
+        const int slot = slot_of(layer);
+        const int store_new = ml ? static_cast<int>(p.ml_store[layer]) : p.store_new;
+        const __nv_bfloat16 *k_new = p.K_new;
+        const __nv_bfloat16 *v_new = p.V_new;
+        if (ml && k_new != nullptr) {
+            k_new += static_cast<size_t>(slot) * p.ml_kv_stride;
+            v_new += static_cast<size_t>(slot) * p.ml_kv_stride;
+        }
         const int seg_first = wk.seg_first;
         const int seg_end = seg_first + wk.nt;
         const int piece_first = tile;
@@ -405,7 +446,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
 
         if (tile == tile_lo) {
             if (!early)
-                load_q_frag<D>(qa, p, beta, j, lane);
+                load_q_frag<D>(qa, p, q_of(layer), beta, j, lane);
         } else {
             // A later piece: its query rows arrive with its first tile (the loop's wait for that
             // tile then returns at once).
@@ -435,7 +476,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             if (!flags[0] && valid > 0) {
                 const uint32_t kt = sbase + s * PL::kStageBytes;
                 const uint32_t vt = kt + PL::kTileBytes;
-                if (p.K_new != nullptr && valid <= TW) {
+                if (k_new != nullptr && valid <= TW) {
                     // Fused append: this warp's slice holds position L-1, the new token.  Its K/V
                     // replace the tile rows (the copy may have read the cache before the token was
                     // stored) and, in the owner layer, are stored in the cache for the layers that
@@ -443,14 +484,14 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     const int r_new = row0 + valid - 1;
                     if (lane < 8 * PL::kSub) {
                         const size_t src = (static_cast<size_t>(beta) * p.g + j) * D + lane * 8;
-                        const uint4 kn = *reinterpret_cast<const uint4 *>(p.K_new + src);
-                        const uint4 vn = *reinterpret_cast<const uint4 *>(p.V_new + src);
+                        const uint4 kn = *reinterpret_cast<const uint4 *>(k_new + src);
+                        const uint4 vn = *reinterpret_cast<const uint4 *>(v_new + src);
                         uint8_t *st = smem + s * PL::kStageBytes;
                         *reinterpret_cast<uint4 *>(st + swz<T>(r_new, lane)) = kn;
                         *reinterpret_cast<uint4 *>(st + PL::kTileBytes + swz<T>(r_new, lane)) = vn;
-                        if (p.store_new) {
+                        if (store_new) {
                             const size_t dst =
-                                ((((static_cast<size_t>(p.slot) * 2) * p.b + beta) * p.g + j) *
+                                ((((static_cast<size_t>(slot) * 2) * p.b + beta) * p.g + j) *
                                      static_cast<size_t>(p.max_seq) + (L - 1)) * D + lane * 8;
                             *reinterpret_cast<uint4 *>(p.cache + dst) = kn;
                             *reinterpret_cast<uint4 *>(
@@ -670,6 +711,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     meta[kMetaFirst] = cta_of_tile(seg_first, N, P);
                     meta[kMetaLast] = cta_of_tile(seg_end - 1, N, P);
                     meta[kMetaStop] = 0;
+                    meta[kMetaLayer] = layer;
                 }
                 __syncwarp();
                 if (lane == 0)
@@ -702,8 +744,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             consumer_bar_sync<NCW>();
             const int ctid = threadIdx.x;
             const bool whole = (piece_first == seg_first && piece_end == seg_end);
-            __nv_bfloat16 *ob =
-                p.out + (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
+            __nv_bfloat16 *ob = p.out + static_cast<size_t>(layer) * p.ml_q_stride +
+                                (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
             constexpr int kPairs = NCW * 32;   // float2 outputs per pass
             static_assert(D == 2 * 32 || D == 4 * 32, "a warp's pass covers 64 elements of one row");
             // mode: 0 whole, 1 cluster sender, 2 cluster leader, 3 partial record
@@ -871,6 +913,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         }
     }
 }
+
 
 // ------------------------------------------------------------------------------------------------
 // combine kernel: merge of segments split over many CTAs

@@ -83,6 +83,14 @@ void setup_device(int dev, DeviceSetup &st)
         return;
     }
     st.max_smem = static_cast<size_t>(smem_optin);
+    // The error word (and the counters after it) start at zero; calls then clear only the
+    // counters, so an error stays recorded until mlkv_static_status reads it.
+    if ((e = cudaMemset(st.scratch, 0, 256)) != cudaSuccess ||
+        (e = cudaDeviceSynchronize()) != cudaSuccess) {
+        st.status = MLKV_ERR_CUDA;
+        st.error = std::string("clearing the static scratch: ") + cudaGetErrorString(e);
+        return;
+    }
     for (int d : {64, 128})
         for (int T : {64, 128, 256}) {
             const mlkv::DecodeVariant *v = mlkv::find_decode_variant(d, T);
@@ -108,6 +116,14 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
         return fail(MLKV_ERR_INVALID_ARG, "kv_slot, Q and out must be 16-byte aligned");
     if (batch < 1 || n_q_heads < 1 || kv_heads < 1 || max_seq < 1)
         return fail(MLKV_ERR_INVALID_ARG, "sizes must be positive");
+    {
+        // The kernel reads Q after other CTAs may have written out: they must not overlap.
+        const size_t qbytes = static_cast<size_t>(batch) * n_q_heads * head_dim * 2;
+        const char *qs = static_cast<const char *>(Q);
+        const char *os = static_cast<const char *>(out);
+        if (qs < os + qbytes && os < qs + qbytes)
+            return fail(MLKV_ERR_INVALID_ARG, "out overlaps Q");
+    }
     if (batch > MLKV_MAX_BATCH)
         return fail(MLKV_ERR_UNSUPPORTED, "batch exceeds MLKV_MAX_BATCH");
     if (kv_heads > n_q_heads || n_q_heads % kv_heads != 0)
@@ -135,9 +151,10 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     if (st.status != MLKV_OK)
         return fail(st.status, st.error.c_str());
 
-    // Tile length as on the regular path; fall back to 64 when the tables do not fit.
+    // Tile length by the regular path's default rule (mlkv::default_tile_tokens, over the
+    // batch * kv_heads segments); 64 when the per-sequence tables do not fit beside the ring.
     const double mean_len = static_cast<double>(len_sum) / batch;
-    int T = head_dim == 64 ? (mean_len >= 512 ? 256 : 128) : (mean_len >= 512 ? 128 : 64);
+    int T = mlkv::default_tile_tokens(head_dim, mean_len, batch * kv_heads);
     const mlkv::DecodeVariant *v = mlkv::find_decode_variant(head_dim, T);
     if (v == nullptr)
         return fail(MLKV_ERR_UNSUPPORTED, "no decode variant");
@@ -187,10 +204,10 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
         (static_cast<size_t>(S + grid) * G * 4 + 255) & ~size_t(255);
     float *part_o = reinterpret_cast<float *>(base + head_bytes + lse_bytes);
 
-    // The array keeps whatever the previous call left: the error word and the counters must
-    // start at zero.
+    // The array keeps whatever the previous call left: the counters must start at zero.  The
+    // error word is left alone (mlkv_static_status reads and clears it).
     cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-    e = cudaMemsetAsync(base, 0, head_bytes, stream);
+    e = cudaMemsetAsync(base + 256, 0, head_bytes - 256, stream);
     if (e != cudaSuccess)
         return fail(MLKV_ERR_CUDA, "clearing the static scratch failed");
 
@@ -236,6 +253,13 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.early_fetch = 0;
+    p.newest_ready = 0;
+    p.store_new = 0;
+    p.pf_own = 0;
+    p.ml_layers = 0;
+    p.ml_slots = 0;
+    p.ml_q_stride = 0;
+    p.ml_kv_stride = 0;
     p.Q_next = nullptr;
     p.deferred_merge =
         mlkv::max_pieces_per_segment(p, T, grid) > mlkv::kInlineMergeMaxPieces ? 1 : 0;
@@ -246,4 +270,32 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     if (p.deferred_merge && mlkv::launch_combine(p, head_dim, stream) != cudaSuccess)
         return fail(MLKV_ERR_CUDA, "combine launch failed");
     return MLKV_OK;
+}
+
+extern "C" int mlkv_static_status(void *cuda_stream)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return fail(MLKV_ERR_CUDA, "no usable current device");
+    DeviceSetup &st = g_setup[dev];
+    std::call_once(st.once, setup_device, dev, std::ref(st));
+    if (st.status != MLKV_OK)
+        return fail(st.status, st.error.c_str());
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    int word = 0;
+    if ((e = cudaMemcpyAsync(&word, st.scratch, sizeof(word), cudaMemcpyDeviceToHost, stream)) !=
+            cudaSuccess ||
+        (e = cudaStreamSynchronize(stream)) != cudaSuccess)
+        return fail(MLKV_ERR_CUDA, (std::string("reading the static error word: ") +
+                                    cudaGetErrorString(e)).c_str());
+    if (word == 0)
+        return MLKV_OK;
+    if ((e = cudaMemsetAsync(st.scratch, 0, sizeof(word), stream)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(stream)) != cudaSuccess)
+        return fail(MLKV_ERR_CUDA, (std::string("clearing the static error word: ") +
+                                    cudaGetErrorString(e)).c_str());
+    char msg[96];
+    std::snprintf(msg, sizeof(msg), "a static decode launch reported device error bits 0x%x", word);
+    return fail(MLKV_ERR_DEVICE, msg);
 }

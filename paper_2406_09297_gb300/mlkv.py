@@ -31,6 +31,7 @@ EXPORTED = [
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
     "mlkv_merge_kv_weights", "mlkv_decode_block_fused", "mlkv_decode_step_host",
+    "mlkv_static_status",
 ]
 
 
@@ -69,6 +70,7 @@ def _load():
     L.mlkv_block_owner_map.argtypes = [ci, ci, ip]
     L.mlkv_version.argtypes = []
     L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
+    L.mlkv_static_status.argtypes = [vp]
     L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
     L.mlkv_merge_kv_weights.argtypes = [ip, ci, ci, ci, i64, vp, vp, vp]
     L.mlkv_decode_block_fused.argtypes = [vp, ci, vp, vp, ip, vp]
@@ -222,6 +224,11 @@ def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, 
     return _check(lib.mlkv_decode_attention_static(
         ctypes.c_void_p(kv_slot), batch, n_q_heads, kv_heads, head_dim, max_seq, _ptr(Q),
         _ptr(out), p, _stream(stream)))
+
+
+def mlkv_static_status(stream=None):
+    """Error record of mlkv_decode_attention_static on the current device (waits for stream)."""
+    return _check(lib.mlkv_static_status(_stream(stream)))
 
 
 def mlkv_decode_block_fused(handle, owner_layer, Q, out, seq_lens, stream=None):

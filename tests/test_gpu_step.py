@@ -30,6 +30,9 @@ def _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref):
 @pytest.mark.parametrize("owner,h,g,d,b,lens,max_seq", [
     ([0, 0, 2, 2, 2, 5], 12, 2, 64, 5, [1, 300, 1000, 77, 640], 1024),
     ([0, 0, 0, 0], 12, 1, 64, 64, [2048] * 64, 2048),            # whole segments per CTA
+    # the benchmark's map (owner change at layer 6) with one length: whole segments per CTA,
+    # the later layers taking the owner's new token from the step input, slot 1 prefetched
+    ([0] * 6 + [6] * 6, 12, 1, 64, 64, [1024] * 64, 1024),
     ([0, 0, 2], 16, 4, 128, 3, [5000, 20, 4096], 5000),
 ])
 def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
@@ -63,10 +66,10 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
         torch.cuda.synchronize()
         uniform = bool((lens == lens[0]).all())
         if uniform:
-            # With one length the step's later layers run whole segments per CTA (no merge),
+            # With one length the step is one multi-layer launch of whole segments (no merge),
             # while the layer calls split segments into clusters: same results up to rounding.
+            assert cache.get_option("last_step_kernel") == 1
             assert cache.get_option("last_cluster_k") == 0
-            assert cache.get_option("last_grid") == b * g
         else:
             assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
         for n in range(l):
@@ -225,6 +228,7 @@ def test_step_single_long_segment():
         out = torch.full((len(owner), b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
         cache.decode_step(to_dev(qb), to_dev(kn), to_dev(vn), out, lens)
         torch.cuda.synchronize()
+        assert cache.get_option("last_step_kernel") == 0   # three items: per-layer launches
         assert cache.get_option("last_tile_tokens") == 128
         assert cache.get_option("last_grid") == 64
         ref.append(0, gen.bf16_bits_to_f64(kn[0]), gen.bf16_bits_to_f64(vn[0]), lens)
@@ -240,14 +244,16 @@ def test_step_single_long_segment():
     (64, 4, 4352, 64, 256),     # 256 segments of 17 tiles of 256: 64 CTAs of four segments
 ])
 def test_step_whole_segments_per_cta(b, g, L, grid, tile):
-    # Inside a step the later layers run whole segments per CTA, several per CTA here: each later
-    # segment's queries arrive with its first tile.
+    # With per-layer launches (option step_kernel 0) the later layers of a step run whole
+    # segments per CTA, several per CTA here: each later segment's queries arrive with its first
+    # tile.
     import torch
 
     import paper_2406_09297_gb300 as mlkv
     owner, h, d = [0, 0, 0], 12, 64
     lens = np.full(b, L, dtype=np.int32)
     with mlkv.MLKVCache(len(owner), h, d, owner, g, b, L) as cache:
+        cache.set_option("step_kernel", 0)
         ref = oracle.OracleCache(owner, h, g, d, b, L)
         qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 71, cache, ref)
         out = torch.full((len(owner), b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
@@ -262,3 +268,55 @@ def test_step_whole_segments_per_cta(b, g, L, grid, tile):
             mx, mean = errors(from_dev(out[n]), expect)
             assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
         cache.sync_status()
+
+
+@pytest.mark.parametrize("owner,h,g,d,b,L,grid", [
+    ([0] * 6 + [6] * 6, 12, 1, 64, 64, 2048, 256),     # the benchmark's shape: 768 items, 3 a CTA
+    ([0, 1, 2, 3], 12, 1, 64, 40, 700, 160),           # every layer an owner (MQA), ragged last tile
+    ([0, 0, 0, 3, 3, 3], 12, 4, 64, 16, 1000, 192),    # GQA groups of 3 under MLKV
+    ([0, 0, 2, 2], 32, 8, 128, 8, 1500, 128),          # head_dim 128, groups of 4
+    ([0, 0, 2, 2, 4, 4, 6, 6, 8, 8, 10, 10], 12, 1, 64, 1, 128, 12),   # short context: one wave
+    ([0, 0, 0], 16, 2, 64, 100, 77, 300),              # one partly visible tile per item
+    ([0] * 6, 12, 1, 64, 8, 2001, 48),                 # batch 8: one 256-position-tile item a CTA
+])
+def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
+    # One launch for the whole step: CTA c takes the (layer, segment) items c, c + P, ..., each a
+    # whole segment; every layer replaces its newest rows from the step's new tokens and owner
+    # layers store them.  Every output of every layer against the oracle; graph replay too.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    lens = np.full(b, L, dtype=np.int32)
+    l = len(owner)
+    owners = sorted(set(owner))
+    with mlkv.MLKVCache(l, h, d, owner, g, b, L) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, L)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 81, cache, ref)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        results = []
+        for rep in range(3):   # direct, record, replay
+            out.fill_(float("nan"))
+            cache.decode_step(Q, K, V, out, lens)
+            torch.cuda.synchronize()
+            results.append(out.clone())
+            assert cache.get_option("last_step_kernel") == 1
+            assert cache.get_option("last_grid") == grid
+        assert cache.get_option("step_graph_replays") == 2
+        for r in results[1:]:
+            assert torch.equal(r.view(torch.int16), results[0].view(torch.int16))
+        for n in range(l):
+            if owner[n] == n:
+                k = owners.index(n)
+                ref.append(n, gen.bf16_bits_to_f64(kn[k]), gen.bf16_bits_to_f64(vn[k]), lens)
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
+            mx, mean = errors(from_dev(results[0][n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        # the owners' new tokens are in the cache afterwards, at position L - 1, K and V
+        from tests.test_gpu_cache import _read_cache
+        whole = _read_cache(cache, b, g, L, d)          # int16 [m][2][b][g][L][d]
+        for k, n in enumerate(owners):
+            assert (whole[cache.owner_slot(n)[1], 0, :, :, L - 1] == kn[k].view(np.int16)).all()
+            assert (whole[cache.owner_slot(n)[1], 1, :, :, L - 1] == vn[k].view(np.int16)).all()
+        cache.sync_status()
+

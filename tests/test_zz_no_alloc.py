@@ -4,7 +4,8 @@ cudaMalloc while it runs).  It keeps its merge scratch in an array compiled into
 
 Each case calls it twice in a row through the C ABI and compares every output with the regular
 entry point's (mlkv_decode_attention) on the same inputs, within the parity tolerance of the other
-GPU tests.  This file is named to be collected last.
+GPU tests, and reads the static error record (mlkv_static_status) after each call.  This file is
+named to be collected last.
 """
 import numpy as np
 import pytest
@@ -39,6 +40,9 @@ def _check_two_calls(owner, h, g, d, b, lens, max_seq, seed):
             assert np.isfinite(s).all()
             mx, mean = errors(s, r)
             assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+            # no bounded wait expired in the static kernels (their error word lives in the
+            # static array; reading it allocates nothing either)
+            assert mlkv.mlkv_static_status() == mlkv.MLKV_OK
         cache.sync_status()
 
 
@@ -55,10 +59,28 @@ def test_static_entry_rejects_requests_beyond_its_scratch():
     import torch
 
     import paper_2406_09297_gb300 as mlkv
-    buf = torch.zeros(64, dtype=torch.bfloat16, device="cuda")
+    slot = torch.zeros((2, 1024, 16, 1, 128), dtype=torch.bfloat16, device="cuda")
+    q = torch.zeros((1024, 16, 128), dtype=torch.bfloat16, device="cuda")
+    out = torch.zeros_like(q)
     lens = np.ones(1024, dtype=np.int32)
     # 1024 sequences x 16 KV heads x (128 + 1) floats: more records than the 8 MiB scratch holds
     with pytest.raises(mlkv.MLKVError) as e:
-        mlkv.mlkv_decode_attention_static(buf.data_ptr(), 1024, 16, 16, 128, 1, buf, buf, lens)
+        mlkv.mlkv_decode_attention_static(slot.data_ptr(), 1024, 16, 16, 128, 1, q, out, lens)
     assert e.value.code == mlkv.MLKV_ERR_UNSUPPORTED
     assert "SCRATCH" in mlkv.mlkv_last_error()
+
+
+def test_static_entry_rejects_out_overlapping_q():
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    b, h, g, d, max_seq = 2, 12, 1, 64, 128
+    slot = torch.zeros((2, b, g, max_seq, d), dtype=torch.bfloat16, device="cuda")
+    buf = torch.zeros((2 * b * h * d,), dtype=torch.bfloat16, device="cuda")
+    lens = np.full(b, 16, dtype=np.int32)
+    with pytest.raises(mlkv.MLKVError) as e:   # out starts inside Q
+        mlkv.mlkv_decode_attention_static(slot.data_ptr(), b, h, g, d, max_seq, buf,
+                                          buf[b * h * d // 2:], lens)
+    assert e.value.code == mlkv.MLKV_ERR_INVALID_ARG
+    assert "overlap" in mlkv.mlkv_last_error()
+    assert mlkv.mlkv_static_status() == mlkv.MLKV_OK
