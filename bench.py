@@ -375,7 +375,8 @@ def run(args, w):
     del big_flush
     kernel_name = "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel"
     options = {k: int(cache.get_option(k)) for k in ("l2_prefetch", "l2_persist", "tc",
-                                                      "step_kernel")}
+                                                      "step_kernel", "l2_persist_bytes",
+                                                      "l2_window_max", "last_step_kernel")}
     traffic = _recorded_traffic(w, kernel_name)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
@@ -604,6 +605,37 @@ def _hbm_peak():
         return 6800.0, "fallback"
 
 
+def run_l2_peak(args):
+    """Read bandwidth of L2-resident data, the roofline of a decode layer whose owner slot an
+    earlier layer of its block has just brought into L2 (a Pythia-160M MLKV-2 slot at batch 64,
+    context 2048 is 32 MiB): the library's read-bandwidth probe (bulk copies into a shared-memory
+    ring, as the decode kernel moves K/V) over a 32 MiB and a 64 MiB buffer, 20 passes in one
+    launch, and over a 4 GiB buffer (HBM), CUDA events around each launch, best of five."""
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    torch.cuda.set_device(0)
+    res = {}
+    for name, nbytes, reps in (("l2_32MiB", 32 << 20, 20), ("l2_64MiB", 64 << 20, 20),
+                               ("hbm_4GiB", 4 << 30, 1)):
+        buf = torch.ones(nbytes // 2, dtype=torch.bfloat16, device="cuda")
+        best = 0.0
+        for _ in range(6):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            n = mlkv.mlkv_read_bandwidth_probe(buf, reps)
+            e1.record()
+            e1.synchronize()
+            best = max(best, n / (e0.elapsed_time(e1) / 1e3) / 1e9)
+        res[name + "_gbs"] = best
+        del buf
+    line = {"metric": "read bandwidth (bulk copies into shared memory)", "unit": "GB/s", **res,
+            "hbm_copy_gbs_measured_peaks": _hbm_peak()[0],
+            "how": "mlkv_read_bandwidth_probe: 2 CTAs per SM, 32 KiB copies, 2-stage ring; "
+                   "CUDA events around one launch; best of 6 (first one warms L2)"}
+    print(json.dumps(line), flush=True)
+
+
 def run_merge(args, w):
     """Sec. 4.2 conversion of the workload's model: its MHA K and V projections (l x h heads, each
     head_dim x d_model, d_model = h * head_dim, seeded bf16) merged by averaging into the owner
@@ -753,6 +785,8 @@ def main():
     ap.add_argument("--prefill-len", type=int, default=2048)
     ap.add_argument("--fused", action="store_true",
                     help="cross-layer fused decode of the --config workload (benchmark only)")
+    ap.add_argument("--l2-peak", action="store_true",
+                    help="measure the read bandwidth of an L2-resident buffer")
     ap.add_argument("--merge", action="store_true",
                     help="Sec. 4.2 KV-weight merge of the --config model's K and V projections")
     args = ap.parse_args()
@@ -763,6 +797,9 @@ def main():
     if args.prefill:
         from mlkv_synth import workloads
         run_prefill(args, workloads.by_name(args.config))
+        return
+    if args.l2_peak:
+        run_l2_peak(args)
         return
     if args.merge:
         from mlkv_synth import workloads

@@ -368,6 +368,24 @@ int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void
 int mlkv_merge_kv_weights(const int *layer_owner, int n_layers, int n_q_heads, int n_kv_heads,
                           int64_t row_elems, const void *W, void *W_merged, void *cuda_stream);
 
+/*
+ * mlkv_read_bandwidth_probe - benchmark support, not part of the decode path (the paper has no
+ * counterpart): queues one kernel that reads [buf, buf + bytes) `reps` times the way the decode
+ * kernel moves K/V -- bulk asynchronous copies of 32 KiB into a two-stage shared-memory ring,
+ * two CTAs per SM, each streaming its own contiguous share -- and does nothing else with the
+ * data.  Timed with CUDA events around it on an L2-resident buffer it gives the L2 read roofline
+ * of the decode layers that find their owner's slot in L2; on a buffer larger than L2, the HBM
+ * read rate.  Allocates nothing.
+ *
+ *   buf          device memory, 16-byte aligned, read only
+ *   bytes        size of buf; every CTA reads bytes / (2 * SMs) rounded down to 32 KiB
+ *   reps         passes over the buffer (>= 1)
+ *   bytes_read   host int64*: receives the bytes the kernel reads in all passes
+ * Errors: MLKV_ERR_INVALID_ARG (null, unaligned, too small), MLKV_ERR_CUDA.
+ */
+int mlkv_read_bandwidth_probe(const void *buf, int64_t bytes, int reps, int64_t *bytes_read,
+                              void *cuda_stream);
+
 /* Library version, major*10000 + minor*100 + patch. */
 int mlkv_version(void);
 

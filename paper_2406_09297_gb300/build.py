@@ -20,7 +20,7 @@ NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc" if os.path.exists(
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 SOURCES = ["mlkv_kernels.cu", "mlkv_decode_tc.cu", "mlkv_prefill.cu", "mlkv_merge.cu",
-           "mlkv_stage.cu", "mlkv_host.cpp", "mlkv_noalloc.cu"]
+           "mlkv_stage.cu", "mlkv_host.cpp", "mlkv_noalloc.cu", "mlkv_measure.cu"]
 
 
 def _sources():

@@ -133,6 +133,12 @@ __device__ __forceinline__ void load_q_frag_smem(uint32_t (&qa)[D / 16][4], cons
     }
 }
 
+// Margin (log2 units) by which a score may exceed a row's reference maximum before the reference
+// is raised: weights stay <= 2^8.
+constexpr float kLazyMax = 8.f;
+// Two bf16 ones, the B operand that turns P V's MMA into P's row sums.
+constexpr uint32_t kOnesBf16x2 = 0x3f803f80u;
+
 // ------------------------------------------------------------------------------------------------
 // decode kernel
 // ------------------------------------------------------------------------------------------------
@@ -463,7 +469,9 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         for (int n = 0; n < NO; ++n)
             o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
         float m_run[2] = {NEG_INF, NEG_INF};
-        float l_run[2] = {0.f, 0.f};
+        // Row sums of P, accumulated on the tensor core: P times a block of ones (every column
+        // of la holds its row's sum), in fp32 from the same bf16 weights P V uses.
+        float la[4] = {0.f, 0.f, 0.f, 0.f};
 
         for (; tile < piece_end; ++tile, ++it) {
             const int s = it % STAGES;
@@ -524,16 +532,45 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
                 const int mi = lane >> 3;   // which 8x8 matrix this lane addresses
                 const int mr = lane & 7;    // which row of it
+                // The K fragments of a group of up to 8 shared-memory loads go out together and
+                // the MMAs follow, so the loads' latency (~47 cycles each) is paid once per group.
+                constexpr int KG = (KS * (NT / 2) <= 8) ? KS : (8 / (NT / 2) > 0 ? 8 / (NT / 2) : 1);
 #pragma unroll
-                for (int ks = 0; ks < KS; ++ks) {
+                for (int k0 = 0; k0 < KS; k0 += KG) {
+                    uint32_t kf[KG][NT / 2][4];
 #pragma unroll
-                    for (int n = 0; n < NT; n += 2) {
-                        const int row = row0 + 8 * (n + (mi >> 1)) + mr;
-                        const int chunk = 2 * ks + (mi & 1);
-                        uint32_t b0, b1, b2, b3;
-                        ldsm_x4(kt + swz<T>(row, chunk), b0, b1, b2, b3);
-                        mma_bf16_16816(sc[n], qa[ks], b0, b1);
-                        mma_bf16_16816(sc[n + 1], qa[ks], b2, b3);
+                    for (int kg = 0; kg < KG; ++kg) {
+#pragma unroll
+                        for (int n2 = 0; n2 < NT / 2; ++n2) {
+                            const int row = row0 + 8 * (2 * n2 + (mi >> 1)) + mr;
+                            const int chunk = 2 * (k0 + kg) + (mi & 1);
+                            ldsm_x4(kt + swz<T>(row, chunk), kf[kg][n2][0], kf[kg][n2][1],
+                                    kf[kg][n2][2], kf[kg][n2][3]);
+                        }
+                    }
+#pragma unroll
+                    for (int kg = 0; kg < KG; ++kg) {
+#pragma unroll
+                        for (int n2 = 0; n2 < NT / 2; ++n2) {
+                            mma_bf16_16816(sc[2 * n2], qa[k0 + kg], kf[kg][n2][0], kf[kg][n2][1]);
+                            mma_bf16_16816(sc[2 * n2 + 1], qa[k0 + kg], kf[kg][n2][2],
+                                           kf[kg][n2][3]);
+                        }
+                    }
+                }
+                // The V fragments of the first group of P V (up to 8 loads) go out now: their
+                // latency overlaps the softmax below.
+                constexpr int VQ = NO / 2;                         // loads per 16 positions
+                constexpr int VG = (VQ * (NT / 2) <= 8) ? NT / 2 : (8 / VQ > 0 ? 8 / VQ : 1);
+                uint32_t vf[VG][VQ][4];
+#pragma unroll
+                for (int kg = 0; kg < VG; ++kg) {
+#pragma unroll
+                    for (int q = 0; q < VQ; ++q) {
+                        const int row = row0 + 16 * kg + 8 * (mi & 1) + mr;
+                        const int chunk = 2 * q + (mi >> 1);
+                        ldsm_x4_trans(vt + swz<T>(row, chunk), vf[kg][q][0], vf[kg][q][1],
+                                      vf[kg][q][2], vf[kg][q][3]);
                     }
                 }
 
@@ -555,19 +592,22 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     mx[0] = fmaxf(mx[0], fmaxf(sc[n][0], sc[n][1]));
                     mx[1] = fmaxf(mx[1], fmaxf(sc[n][2], sc[n][3]));
                 }
-                float alpha[2], m_use[2];
+                // The reference maximum moves only when a score exceeds it by more than 2^8 (in
+                // the exponent): weights then stay in [0, 256], exactly as accurate in bf16, and
+                // most tiles need neither the quad reduction nor a rescale.  When one does, the
+                // rows' exact maxima over this tile become the new references.
+                const bool raise = mx[0] * scale > m_run[0] + kLazyMax ||
+                                   mx[1] * scale > m_run[1] + kLazyMax;
+                if (__any_sync(0xffffffffu, raise)) {
+                    float alpha[2];
 #pragma unroll
-                for (int hr = 0; hr < 2; ++hr) {
-                    mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 1));
-                    mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 2));
-                    const float m_new = fmaxf(m_run[hr], mx[hr] * scale);
-                    m_use[hr] = (m_new == NEG_INF) ? 0.f : m_new;
-                    alpha[hr] = fast_exp2(m_run[hr] - m_use[hr]);
-                    m_run[hr] = m_new;
-                    l_run[hr] *= alpha[hr];
-                }
-                // Rescale the accumulators only when some row's running maximum moved.
-                if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
+                    for (int hr = 0; hr < 2; ++hr) {
+                        mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 1));
+                        mx[hr] = fmaxf(mx[hr], __shfl_xor_sync(0xffffffffu, mx[hr], 2));
+                        const float m_new = fmaxf(m_run[hr], mx[hr] * scale);
+                        alpha[hr] = (m_new == NEG_INF) ? 1.f : fast_exp2(m_run[hr] - m_new);
+                        m_run[hr] = m_new;
+                    }
 #pragma unroll
                     for (int n = 0; n < NO; ++n) {
                         o[n][0] *= alpha[0];
@@ -575,8 +615,14 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                         o[n][2] *= alpha[1];
                         o[n][3] *= alpha[1];
                     }
+                    la[0] *= alpha[0];
+                    la[1] *= alpha[0];
+                    la[2] *= alpha[1];
+                    la[3] *= alpha[1];
                 }
-                // P in bf16 (the mma A operand); the row sums use the same rounded weights.
+                const float m_use[2] = {m_run[0] == NEG_INF ? 0.f : m_run[0],
+                                        m_run[1] == NEG_INF ? 0.f : m_run[1]};
+                // P in bf16 (the mma A operand).
                 uint32_t pa[NT / 2][4];
 #pragma unroll
                 for (int n = 0; n < NT; ++n) {
@@ -584,25 +630,43 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     const float p1 = fast_exp2(fmaf(sc[n][1], scale, -m_use[0]));
                     const float p2 = fast_exp2(fmaf(sc[n][2], scale, -m_use[1]));
                     const float p3 = fast_exp2(fmaf(sc[n][3], scale, -m_use[1]));
-                    const uint32_t top = pack_bf16x2(p0, p1);
-                    const uint32_t bot = pack_bf16x2(p2, p3);
-                    l_run[0] += bf16_lo(top) + bf16_hi(top);
-                    l_run[1] += bf16_lo(bot) + bf16_hi(bot);
-                    pa[n >> 1][(n & 1) * 2 + 0] = top;
-                    pa[n >> 1][(n & 1) * 2 + 1] = bot;
+                    pa[n >> 1][(n & 1) * 2 + 0] = pack_bf16x2(p0, p1);
+                    pa[n >> 1][(n & 1) * 2 + 1] = pack_bf16x2(p2, p3);
                 }
 
                 // ---- O += P V ----
 #pragma unroll
-                for (int kk = 0; kk < NT / 2; ++kk) {
+                for (int kg = 0; kg < VG; ++kg) {
 #pragma unroll
-                    for (int q = 0; q < NO / 2; ++q) {
-                        const int row = row0 + 16 * kk + 8 * (mi & 1) + mr;
-                        const int chunk = 2 * q + (mi >> 1);
-                        uint32_t b0, b1, b2, b3;
-                        ldsm_x4_trans(vt + swz<T>(row, chunk), b0, b1, b2, b3);
-                        mma_bf16_16816(o[2 * q], pa[kk], b0, b1);
-                        mma_bf16_16816(o[2 * q + 1], pa[kk], b2, b3);
+                    for (int q = 0; q < VQ; ++q) {
+                        mma_bf16_16816(o[2 * q], pa[kg], vf[kg][q][0], vf[kg][q][1]);
+                        mma_bf16_16816(o[2 * q + 1], pa[kg], vf[kg][q][2], vf[kg][q][3]);
+                    }
+                    mma_bf16_16816(la, pa[kg], kOnesBf16x2, kOnesBf16x2);
+                }
+                // the remaining 16-position groups (longer tiles), a group's loads first
+#pragma unroll
+                for (int k0 = VG; k0 < NT / 2; k0 += VG) {
+                    uint32_t vg[VG][VQ][4];
+#pragma unroll
+                    for (int kg = 0; kg < VG; ++kg) {
+#pragma unroll
+                        for (int q = 0; q < VQ; ++q) {
+                            const int row = row0 + 16 * (k0 + kg) + 8 * (mi & 1) + mr;
+                            const int chunk = 2 * q + (mi >> 1);
+                            ldsm_x4_trans(vt + swz<T>(row, chunk), vg[kg][q][0], vg[kg][q][1],
+                                          vg[kg][q][2], vg[kg][q][3]);
+                        }
+                    }
+#pragma unroll
+                    for (int kg = 0; kg < VG; ++kg) {
+#pragma unroll
+                        for (int q = 0; q < VQ; ++q) {
+                            mma_bf16_16816(o[2 * q], pa[k0 + kg], vg[kg][q][0], vg[kg][q][1]);
+                            mma_bf16_16816(o[2 * q + 1], pa[k0 + kg], vg[kg][q][2],
+                                           vg[kg][q][3]);
+                        }
+                        mma_bf16_16816(la, pa[k0 + kg], kOnesBf16x2, kOnesBf16x2);
                     }
                 }
             }
@@ -615,11 +679,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         // ---------------- end of piece: merge the warps (no atomics) ----------------
         // Row statistics of every warp -> per-row maximum m* and total l*; each warp's
         // accumulators are weighted by 2^(m_w - m*) / l* and the warps summed.
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
-            l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 2);
-        }
+        const float l_run[2] = {la[0], la[2]};
         if ((lane & 3) == 0) {
             red_m[warp * 16 + qr] = m_run[0];
             red_m[warp * 16 + qr + 8] = m_run[1];

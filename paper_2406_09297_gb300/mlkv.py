@@ -31,7 +31,7 @@ EXPORTED = [
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
     "mlkv_merge_kv_weights", "mlkv_decode_block_fused", "mlkv_decode_step_host",
-    "mlkv_static_status",
+    "mlkv_static_status", "mlkv_read_bandwidth_probe",
 ]
 
 
@@ -71,6 +71,7 @@ def _load():
     L.mlkv_version.argtypes = []
     L.mlkv_decode_attention_static.argtypes = [vp, ci, ci, ci, ci, ci, vp, vp, ip, vp]
     L.mlkv_static_status.argtypes = [vp]
+    L.mlkv_read_bandwidth_probe.argtypes = [vp, i64, ci, ctypes.POINTER(i64), vp]
     L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
     L.mlkv_merge_kv_weights.argtypes = [ip, ci, ci, ci, i64, vp, vp, vp]
     L.mlkv_decode_block_fused.argtypes = [vp, ci, vp, vp, ip, vp]
@@ -224,6 +225,14 @@ def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, 
     return _check(lib.mlkv_decode_attention_static(
         ctypes.c_void_p(kv_slot), batch, n_q_heads, kv_heads, head_dim, max_seq, _ptr(Q),
         _ptr(out), p, _stream(stream)))
+
+
+def mlkv_read_bandwidth_probe(buf, reps, stream=None):
+    """Queues the read-bandwidth probe over the device tensor buf; returns the bytes it reads."""
+    n = ctypes.c_int64(0)
+    _check(lib.mlkv_read_bandwidth_probe(_ptr(buf), buf.numel() * buf.element_size(), reps,
+                                         ctypes.byref(n), _stream(stream)))
+    return n.value
 
 
 def mlkv_static_status(stream=None):
