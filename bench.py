@@ -376,7 +376,8 @@ def run(args, w):
     kernel_name = "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel"
     options = {k: int(cache.get_option(k)) for k in ("l2_prefetch", "l2_persist", "tc",
                                                       "step_kernel", "l2_persist_bytes",
-                                                      "l2_window_max", "last_step_kernel")}
+                                                      "l2_window_max", "last_step_kernel",
+                                                      "last_seg_major")}
     traffic = _recorded_traffic(w, kernel_name)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------

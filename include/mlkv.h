@@ -228,12 +228,15 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  prefetches its share of them into L2 (cp.async.bulk.prefetch); 0 (default) = no
  *                  prefetch, measured faster on GB300.  Results are identical.
  *   "step_kernel"  1 (default) = mlkv_decode_step issues the whole step as one launch of the
- *                  decode kernel over every (layer, sequence, KV head) item when every sequence
- *                  has one length, the tcgen05 kernel, a fixed grid and l2_persist (whose windows
- *                  are per layer) are off, the model has at
- *                  most 128 layers and the estimated makespan is no longer than per-layer
- *                  launches' (a few long segments, e.g. batch 1 at long context, keep per-layer
- *                  launches); 0 = always one launch per layer.  Same results within the tolerance.
+ *                  decode kernel over every (layer, sequence, KV head) item, each a whole segment,
+ *                  when the tcgen05 kernel, a fixed grid and l2_persist (whose windows are per
+ *                  layer) are off, the model has at most 128 layers and the estimated makespan is
+ *                  no longer than per-layer launches' (a few long segments, e.g. batch 1 at long
+ *                  context, keep per-layer launches).  Sequences are taken longest first; when the
+ *                  owner slots' visible rows do not fit in L2 the items are ranked segment-major
+ *                  (the layers of a block read each segment at about the same time, so L2 serves
+ *                  all but the first), else layer by layer.  0 = always one launch per layer.
+ *                  Same results within the tolerance.
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through
@@ -253,8 +256,9 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  * "last_deferred_merge", "last_tc" (1 if it ran the tcgen05 kernel), and "step_graph_replays"
  * (graph launches by mlkv_decode_step), "l2_persist_bytes" (the set-aside reserved while
  * l2_persist is on, else 0), "l2_window_max" (the device's largest access-policy window),
- * "last_step_kernel" (1 if the most recent mlkv_decode_step ran as one multi-layer launch) and
- * "last_l2_prefetch" (1 if that launch prefetched the slots into L2).
+ * "last_step_kernel" (1 if the most recent mlkv_decode_step ran as one multi-layer launch),
+ * "last_seg_major" (1 if that launch ranked its items segment-major) and "last_l2_prefetch" (1
+ * if it prefetched the slots into L2).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.
  */
 int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);

@@ -218,15 +218,49 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 template <int T>
 struct TileWalk {
     int beta, j, tt, nt, L, seg_first, layer, item;
+    int kk;   // multi-layer launch: index of the current item among the CTA's
 
-    // Multi-layer launch: (layer, beta, j) of item `item`.
-    __device__ __forceinline__ void set_item(const DecodeParams &p)
+    // Multi-layer launch: the rank of this CTA's k-th item, or -1 past its last: round k of the
+    // deal gives CTA c rank k P + c, or k P + P - 1 - c in odd rounds of a snake deal.
+    __device__ __forceinline__ static int ml_rank(const DecodeParams &p, int k)
     {
-        const int S = p.b * p.g;
-        layer = item / S;
-        const int seg = item - layer * S;
-        beta = seg / p.g;
-        j = seg - beta * p.g;
+        const int P = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
+        const int r = k * P + ((p.ml_snake && (k & 1)) ? P - 1 - c : c);
+        return r < p.ml_layers * p.b * p.g ? r : -1;
+    }
+
+    // Multi-layer launch: index into the sequence order of rank r's sequence.
+    __device__ __forceinline__ static int ml_seq_pos(const DecodeParams &p, int r)
+    {
+        return p.ml_seg_major ? r / (p.g * p.ml_layers) : (r % (p.b * p.g)) / p.g;
+    }
+
+    // Multi-layer launch: (layer, beta, j, L) of rank `item` (see DecodeParams).
+    __device__ __forceinline__ void set_item(const DecodeParams &p, const int *s_len,
+                                             const int *s_start)
+    {
+        int pb;
+        if (p.ml_seg_major) {
+            const int per_seq = p.g * p.ml_layers;
+            pb = item / per_seq;
+            const int rem = item - pb * per_seq;
+            j = rem / p.ml_layers;
+            layer = p.ml_order[rem - j * p.ml_layers];
+        } else {
+            const int S = p.b * p.g;
+            layer = item / S;
+            const int seg = item - layer * S;
+            pb = seg / p.g;
+            j = seg - pb * p.g;
+        }
+        if (p.uniform_len > 0) {
+            beta = pb;
+            L = p.uniform_len;
+        } else {
+            beta = s_start[pb];
+            L = s_len[beta];
+        }
+        nt = (L + T - 1) / T;
     }
 
     // `tile`: the flattened tile of a single-layer launch, or the CTA's own tile count in a
@@ -235,13 +269,12 @@ struct TileWalk {
                                          const int *s_start, int tile)
     {
         if (p.ml_layers > 0) {
-            L = p.uniform_len;
-            nt = (L + T - 1) / T;
-            const int k = tile / nt;
-            tt = tile - k * nt;
-            item = static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x);
-            seg_first = k * nt;
-            set_item(p);
+            // only ever started at the CTA's first tile (tile_lo = 0)
+            kk = 0;
+            item = ml_rank(p, 0);
+            tt = tile;
+            seg_first = 0;
+            set_item(p, s_len, s_start);
             return;
         }
         layer = 0;
@@ -280,9 +313,10 @@ struct TileWalk {
             return;
         tt = 0;
         if (p.ml_layers > 0) {
-            item += static_cast<int>(gridDim.x);
             seg_first += nt;
-            set_item(p);
+            item = ml_rank(p, ++kk);
+            if (item >= 0)
+                set_item(p, s_len, s_start);
             return;
         }
         if (p.uniform_len > 0) {

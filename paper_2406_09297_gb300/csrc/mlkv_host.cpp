@@ -118,6 +118,7 @@ struct mlkv_cache {
     int l2_prefetch = 0;        // multi-layer step: prefetch the step's slots into L2 when they fit
     int step_kernel = 1;        // mlkv_decode_step: one multi-layer launch where it applies
     int last_step_kernel = 0;   // 1 if the most recent step ran as one multi-layer launch
+    int last_seg_major = 0;     // 1 if that launch ranked its items segment-major
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
@@ -644,6 +645,8 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
 
     p.pf_own = 0;
     p.ml_layers = 0;
+    p.ml_seg_major = 0;
+    p.ml_snake = 0;
     p.ml_slots = 0;
     p.ml_q_stride = 0;
     p.ml_kv_stride = 0;
@@ -723,26 +726,71 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     c->last_step_kernel = 0;
     if (!c->step_kernel || c->tc || c->grid > 0 || c->l2_persist || c->l > mlkv::kMaxStepLayers)
         return MLKV_OK;
-    for (int beta = 1; beta < c->b; ++beta)
-        if (seq_lens[beta] != seq_lens[0])
-            return MLKV_OK;
-    const int L = seq_lens[0];
-    mlkv_cache::Variant *var = pick_variant(c, static_cast<double>(L));
+    bool uniform = true;
+    long long len_sum = 0;
+    for (int beta = 0; beta < c->b; ++beta) {
+        uniform = uniform && seq_lens[beta] == seq_lens[0];
+        len_sum += seq_lens[beta];
+    }
+    const double mean_len = static_cast<double>(len_sum) / c->b;
+    mlkv_cache::Variant *var = pick_variant(c, mean_len);
     if (var == nullptr || var->v->tc)
         return MLKV_OK;
+    if (!uniform && var->v->smem_bytes + mlkv::table_bytes(c->b) > c->max_smem) {
+        var = nullptr;   // the per-sequence tables need the small-ring variant
+        for (auto &v : c->variants)
+            if (v.v->tile_tokens == 64 && !v.v->tc &&
+                v.v->smem_bytes + mlkv::table_bytes(c->b) <= c->max_smem)
+                var = &v;
+        if (var == nullptr)
+            return MLKV_OK;
+    }
     const int T = var->v->tile_tokens;
-    const long long nt = (L + T - 1) / T;
     const long long S = static_cast<long long>(c->b) * c->g;
     const long long items = c->l * S;
     const long long slots = static_cast<long long>(var->ctas_per_sm) * c->sm_count;
-    // Makespans in tiles: one launch gives each CTA ceil(items / slots) whole segments; per-layer
-    // launches split every layer over the machine but pay a launch, a ramp and merges per layer
-    // (about 4 tiles' time each; they overlap only in part).  A few long segments (batch 1 at
-    // long context) stay with the per-layer split.
-    const long long per = (items + slots - 1) / slots;
-    if (per * nt > c->l * ((S * nt + slots - 1) / slots + 4) || items * nt > 0x7fffffffLL)
+    if (items > 0x7fffffffLL)
         return MLKV_OK;
-    const int grid = static_cast<int>((items + per - 1) / per);
+    // Sequences longest first (stable); items ranked segment-major over them.
+    static thread_local std::vector<int> perm;
+    perm.resize(c->b);
+    for (int beta = 0; beta < c->b; ++beta)
+        perm[beta] = beta;
+    if (!uniform)
+        std::stable_sort(perm.begin(), perm.end(),
+                         [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
+    // Grid: with one length the fewest CTAs that keep ceil(items / slots) items each; otherwise
+    // every resident slot.  Makespan in tiles: the heaviest CTA's items under the snake deal;
+    // per-layer launches split every layer over the machine but pay a launch, a ramp and merges
+    // per layer (about 4 tiles' time each; they overlap only in part).  A few long segments
+    // (batch 1 at long context) stay with the per-layer split.
+    const long long per = (items + slots - 1) / slots;
+    const int grid = static_cast<int>(uniform ? (items + per - 1) / per : std::min(items, slots));
+    long long total_tiles = 0;
+    for (int beta = 0; beta < c->b; ++beta)
+        total_tiles += static_cast<long long>(c->g) * ((seq_lens[beta] + T - 1) / T);
+    // Segment-major ranks when the slots' visible rows do not fit in L2 (the block's layers then
+    // share each segment's K/V while it is in L2); layer-major otherwise.  A snake deal balances
+    // varied lengths.
+    const long long all_kv = static_cast<long long>(c->m) * 2 * c->g * len_sum * c->d * 2;
+    const int seg_major = all_kv > static_cast<long long>(c->l2_bytes) * 5 / 8 ? 1 : 0;
+    const int snake = uniform ? 0 : 1;
+    long long heaviest = 0;
+    {
+        static thread_local std::vector<long long> load;
+        load.assign(grid, 0);
+        const long long per_seq = static_cast<long long>(c->g) * c->l;
+        for (long long r = 0; r < items; ++r) {
+            const long long k = r / grid, i = r - k * grid;
+            const long long cta = (snake && (k & 1)) ? grid - 1 - i : i;
+            const long long pb = seg_major ? r / per_seq : (r % S) / c->g;
+            load[cta] += (seq_lens[perm[pb]] + T - 1) / T;
+        }
+        for (long long x : load)
+            heaviest = std::max(heaviest, x);
+    }
+    if (heaviest > c->l * ((total_tiles + slots - 1) / slots + 4) || items * heaviest > 0x7fffffffLL)
+        return MLKV_OK;
 
     static thread_local mlkv::DecodeParams p;
     p.Q = reinterpret_cast<const __nv_bfloat16 *>(Q);
@@ -761,8 +809,13 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     p.g = c->g;
     p.G = c->G;
     p.slot = 0;
-    p.num_tiles = static_cast<int>(items * nt);
-    p.uniform_len = L;
+    p.num_tiles = static_cast<int>(total_tiles * c->l);
+    p.uniform_len = uniform ? seq_lens[0] : 0;
+    for (int beta = 0; beta < c->b; ++beta) {
+        p.seq_len[beta] = seq_lens[beta];
+        p.tile_start[beta] = perm[beta];
+    }
+    p.tile_start[c->b] = 0;
     p.cluster_k = 0;
     p.deferred_merge = 0;
     p.tile_tokens = T;
@@ -772,9 +825,11 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     p.newest_ready = 1;
     p.store_new = 0;
     // L2 prefetch of every slot's visible rows when they all fit with room to spare.
-    const long long all_kv = static_cast<long long>(c->m) * 2 * c->b * c->g * L * c->d * 2;
-    p.pf_own = (c->l2_prefetch && all_kv <= static_cast<long long>(c->l2_bytes) * 5 / 8) ? 1 : 0;
+    p.pf_own = (c->l2_prefetch && uniform &&
+                all_kv <= static_cast<long long>(c->l2_bytes) * 5 / 8) ? 1 : 0;
     p.ml_slots = c->m;
+    p.ml_seg_major = seg_major;
+    p.ml_snake = snake;
     p.ml_layers = c->l;
     p.ml_q_stride = static_cast<long long>(c->b) * c->h * c->d;
     p.ml_kv_stride = static_cast<long long>(c->b) * c->g * c->d;
@@ -782,14 +837,23 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
         p.ml_slot[n] = static_cast<unsigned char>(c->slot[n]);
         p.ml_store[n] = c->owner[n] == n ? 1 : 0;
     }
+    // the layers of one owner block next to each other, blocks in slot order
+    {
+        int k = 0;
+        for (int s = 0; s < c->m; ++s)
+            for (int n = 0; n < c->l; ++n)
+                if (c->slot[n] == s)
+                    p.ml_order[k++] = static_cast<unsigned char>(n);
+    }
     cudaError_t e = cudaSuccess;
     if (in_ready != nullptr)
         e = cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), in_ready, 0);
     if (e != cudaSuccess)
         return fail_cuda(e, "step event");
     DeviceGuard guard(c->device);
-    e = mlkv::launch_decode(*var->v, grid, var->v->smem_bytes, static_cast<cudaStream_t>(stream),
-                            &var->tmap, &var->tmap_rows, p, nullptr, c->pdl != 0);
+    const size_t smem = var->v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(c->b));
+    e = mlkv::launch_decode(*var->v, grid, smem, static_cast<cudaStream_t>(stream), &var->tmap,
+                            &var->tmap_rows, p, nullptr, c->pdl != 0);
     if (e != cudaSuccess)
         return fail_cuda(e, "decode launch (multi-layer step)");
     c->last_grid = grid;
@@ -799,6 +863,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     c->last_deferred = 0;
     c->last_l2_prefetch = p.pf_own;
     c->last_step_kernel = 1;
+    c->last_seg_major = seg_major;
     *done = true;
     return MLKV_OK;
 }
@@ -1620,6 +1685,10 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "last_step_kernel") == 0) {
         *value = c->last_step_kernel;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_seg_major") == 0) {
+        *value = c->last_seg_major;
         return MLKV_OK;
     }
     if (std::strcmp(key, "last_l2_prefetch") == 0) {

@@ -53,21 +53,32 @@ struct DecodeParams {
                               // layer's fused append); 0 = only replace the tiles' newest rows (a
                               // later layer of the block, whose owner's launch stores the token)
     int pf_own;               // multi-layer launch: 1 = prefetch the step's slots into L2
-    // Multi-layer launch (ml_layers > 0, every sequence of one length): one grid covers every
-    // (layer, segment) item of a decode step, item i = layer * b g + beta g + j, each a whole
-    // segment, CTA c taking items c, c + P, c + 2P, ...  Q and out then hold every layer
-    // ([layer][b][h][D], ml_q_stride elements apart) and K_new / V_new every owner's new token
-    // ([slot][b][g][D], ml_kv_stride elements apart); layer n reads slot ml_slot[n], and stores
-    // its new token in the cache if ml_store[n] (an owner layer), else only replaces its tiles'
-    // newest rows with it.  slot, store_new and Q_next are unused; pf_own = 1 has every CTA
-    // prefetch its share of the visible rows of all ml_slots slots into L2 at the start.
+    // Multi-layer launch (ml_layers > 0): one grid covers every (layer, sequence, KV head) item of
+    // a decode step, each item a whole segment.  Items are ranked either layer-major (layer n's
+    // segments n b g .. (n + 1) b g - 1) or, with ml_seg_major, segment-major: sequences in the
+    // order tile_start[0..b) holds, then KV head j, then the step's layers in the order ml_order[]
+    // lists them (owner blocks together), so the CTAs working at one time share a few segments'
+    // K/V (read once from HBM, the other layers of the block find it in L2) -- the order for slots
+    // larger than L2.  Sequences are ordered longest first; ranks are dealt to the CTAs round-robin
+    // (round k gives rank k P + c to CTA c) or, with ml_snake, as a snake (odd rounds k P + P-1-c),
+    // which balances varied lengths.  Q and out then
+    // hold every layer ([layer][b][h][D], ml_q_stride elements apart) and K_new / V_new every
+    // owner's new token ([slot][b][g][D], ml_kv_stride elements apart); layer n reads slot
+    // ml_slot[n], and stores its new token in the cache if ml_store[n] (an owner layer), else only
+    // replaces its tiles' newest rows with it.  slot, store_new and Q_next are unused; pf_own = 1
+    // has every CTA prefetch its share of the visible rows of all ml_slots slots into L2 first
+    // (every sequence of one length only).
     int ml_layers;
+    int ml_seg_major;         // 1: ranks segment-major (below); 0: layer-major, layer by layer
+    int ml_snake;             // 1: snake deal of ranks to CTAs; 0: plain round-robin
     int ml_slots;             // owner slots the step reads (with pf_own: all prefetched into L2)
     long long ml_q_stride, ml_kv_stride;
     unsigned char ml_slot[kMaxStepLayers];
     unsigned char ml_store[kMaxStepLayers];
+    unsigned char ml_order[kMaxStepLayers];
     int seq_len[MLKV_MAX_BATCH];
-    int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside)
+    int tile_start[MLKV_MAX_BATCH + 1];  // first flattened tile of sequence beta (j-major inside);
+                                         // a multi-layer launch: the sequences, longest first
 };
 
 // Causal prefill of one layer (mlkv_prefill.cu): one CTA per work unit, a unit being two query

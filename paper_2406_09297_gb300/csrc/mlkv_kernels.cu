@@ -181,10 +181,18 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     const bool narrow = static_cast<long long>(P) * N < (1ll << 32);
     int tile_lo, tile_hi;
     if (ml) {
-        const int items = p.ml_layers * p.b * p.g;
-        const int nt = (p.uniform_len + T - 1) / T;
+        // the tiles of this CTA's items (see TileWalk::ml_rank)
         tile_lo = 0;
-        tile_hi = (cta < items ? (items - 1 - cta) / P + 1 : 0) * nt;
+        tile_hi = 0;
+        for (int k = 0;; ++k) {
+            const int r = TileWalk<T>::ml_rank(p, k);
+            if (r < 0)
+                break;
+            const int L = p.uniform_len > 0
+                              ? p.uniform_len
+                              : p.seq_len[p.tile_start[TileWalk<T>::ml_seq_pos(p, r)]];
+            tile_hi += (L + T - 1) / T;
+        }
     } else {
         tile_lo = narrow ? static_cast<int>(static_cast<uint32_t>(cta) * N / P)
                          : static_cast<int>(static_cast<long long>(cta) * N / P);

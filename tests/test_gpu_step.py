@@ -64,14 +64,15 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
             else:
                 cache2.decode_attention(n, Q[n], out2[n], lens)
         torch.cuda.synchronize()
-        uniform = bool((lens == lens[0]).all())
-        if uniform:
-            # With one length the step is one multi-layer launch of whole segments (no merge),
-            # while the layer calls split segments into clusters: same results up to rounding.
-            assert cache.get_option("last_step_kernel") == 1
+        if cache.get_option("last_step_kernel"):
+            # The step is one multi-layer launch of whole segments (no merge), while the layer
+            # calls split segments over CTAs: same results up to rounding.
             assert cache.get_option("last_cluster_k") == 0
         else:
+            # per-layer launches of the step: the layer calls' shapes, bit for bit
             assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
+        if bool((lens == lens[0]).all()):
+            assert cache.get_option("last_step_kernel") == 1
         for n in range(l):
             if owner[n] == n:
                 s = owners.index(n)
@@ -320,3 +321,40 @@ def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
             assert (whole[cache.owner_slot(n)[1], 1, :, :, L - 1] == vn[k].view(np.int16)).all()
         cache.sync_status()
 
+
+
+@pytest.mark.parametrize("owner,h,g,d,lens", [
+    # varied lengths: segments sorted longest first and dealt in a snake round-robin
+    ([0, 0, 0, 3, 3, 3], 12, 4, 64, [1, 127, 128, 129, 3000, 64, 700, 2048, 5, 1999] * 4),
+    ([0, 0, 2, 2], 32, 8, 128, [300, 1, 1500, 900, 64, 65, 1024, 777]),
+    ([0, 1, 1, 3], 12, 1, 64, [int(x) for x in np.random.default_rng(7).integers(1, 4097, 96)]),
+])
+def test_multi_layer_step_varied_lengths(owner, h, g, d, lens):
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    lens = np.asarray(lens, dtype=np.int32)
+    b, max_seq, l = len(lens), int(lens.max()), len(owner)
+    owners = sorted(set(owner))
+    with mlkv.MLKVCache(l, h, d, owner, g, b, max_seq) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, max_seq)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, max_seq, 91, cache, ref)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        results = []
+        for rep in range(3):   # direct, record, replay
+            out.fill_(float("nan"))
+            cache.decode_step(Q, K, V, out, lens)
+            torch.cuda.synchronize()
+            results.append(out.clone())
+            assert cache.get_option("last_step_kernel") == 1
+        for r in results[1:]:
+            assert torch.equal(r.view(torch.int16), results[0].view(torch.int16))
+        for n in range(l):
+            if owner[n] == n:
+                k = owners.index(n)
+                ref.append(n, gen.bf16_bits_to_f64(kn[k]), gen.bf16_bits_to_f64(vn[k]), lens)
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
+            mx, mean = errors(from_dev(results[0][n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
