@@ -218,7 +218,9 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 template <int T>
 struct TileWalk {
     int beta, j, tt, nt, L, seg_first, layer, item;
-    int kk;   // multi-layer launch: index of the current item among the CTA's
+    int kk;    // multi-layer launch: index of the current item among the CTA's
+    int t0;    // first tile of the current piece's chunk (0 unless segments are chunked)
+    int rec;   // multi-layer launch with chunks: the piece's partial-record index
 
     // Multi-layer launch: the rank of this CTA's k-th item, or -1 past its last: round k of the
     // deal gives CTA c rank k P + c, or k P + P - 1 - c in odd rounds of a snake deal.
@@ -226,30 +228,43 @@ struct TileWalk {
     {
         const int P = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
         const int r = k * P + ((p.ml_snake && (k & 1)) ? P - 1 - c : c);
-        return r < p.ml_layers * p.b * p.g ? r : -1;
+        return r < p.ml_layers * p.b * p.g * p.ml_chunks ? r : -1;
     }
 
     // Multi-layer launch: index into the sequence order of rank r's sequence.
     __device__ __forceinline__ static int ml_seq_pos(const DecodeParams &p, int r)
     {
+        if (p.ml_chunks > 1)
+            r /= p.ml_chunks;
         return p.ml_seg_major ? r / (p.g * p.ml_layers) : (r % (p.b * p.g)) / p.g;
+    }
+
+    // Multi-layer launch: tiles of chunk c of a segment of nt tiles.
+    __device__ __forceinline__ static void ml_chunk(const DecodeParams &p, int nt, int c, int &a,
+                                                    int &b)
+    {
+        a = c * nt / p.ml_chunks;   // chunks <= 1024 and nt <= 2^20: fits in 32 bits
+        b = (c + 1) * nt / p.ml_chunks;
     }
 
     // Multi-layer launch: (layer, beta, j, L) of rank `item` (see DecodeParams).
     __device__ __forceinline__ void set_item(const DecodeParams &p, const int *s_len,
                                              const int *s_start)
     {
+        const bool chunked = p.ml_chunks > 1;
+        const int base = chunked ? item / p.ml_chunks : item;
+        const int chunk = chunked ? item - base * p.ml_chunks : 0;
         int pb;
         if (p.ml_seg_major) {
             const int per_seq = p.g * p.ml_layers;
-            pb = item / per_seq;
-            const int rem = item - pb * per_seq;
+            pb = base / per_seq;
+            const int rem = base - pb * per_seq;
             j = rem / p.ml_layers;
             layer = p.ml_order[rem - j * p.ml_layers];
         } else {
             const int S = p.b * p.g;
-            layer = item / S;
-            const int seg = item - layer * S;
+            layer = base / S;
+            const int seg = base - layer * S;
             pb = seg / p.g;
             j = seg - pb * p.g;
         }
@@ -260,7 +275,19 @@ struct TileWalk {
             beta = s_start[pb];
             L = s_len[beta];
         }
-        nt = (L + T - 1) / T;
+        // the piece is tiles [t0, nt) of the segment; seg_first stays the local index its tile 0
+        // would have, so that the piece is whole exactly when it is the whole segment
+        const int nt_seg = (L + T - 1) / T;
+        if (chunked) {
+            int t1;
+            ml_chunk(p, nt_seg, chunk, t0, t1);
+            nt = t1;
+            rec = ((layer * p.b + beta) * p.g + j) * p.ml_chunks + chunk;
+        } else {
+            t0 = 0;
+            nt = nt_seg;
+            rec = 0;
+        }
     }
 
     // `tile`: the flattened tile of a single-layer launch, or the CTA's own tile count in a
@@ -272,13 +299,15 @@ struct TileWalk {
             // only ever started at the CTA's first tile (tile_lo = 0)
             kk = 0;
             item = ml_rank(p, 0);
-            tt = tile;
-            seg_first = 0;
             set_item(p, s_len, s_start);
+            tt = t0 + tile;
+            seg_first = -t0;
             return;
         }
         layer = 0;
         item = 0;
+        t0 = 0;
+        rec = 0;
         if (p.uniform_len > 0) {
             L = p.uniform_len;
             nt = (L + T - 1) / T;
@@ -313,10 +342,13 @@ struct TileWalk {
             return;
         tt = 0;
         if (p.ml_layers > 0) {
-            seg_first += nt;
+            const int local_end = seg_first + nt;   // where the piece just finished ends
             item = ml_rank(p, ++kk);
-            if (item >= 0)
+            if (item >= 0) {
                 set_item(p, s_len, s_start);
+                tt = t0;
+                seg_first = local_end - t0;
+            }
             return;
         }
         if (p.uniform_len > 0) {
@@ -495,7 +527,9 @@ __device__ __forceinline__ void epilogue_piece(const DecodeParams &p, const floa
         }
         return;
     }
-    const size_t piece = static_cast<size_t>(seg + cta);
+    // a multi-layer launch's partial record index travels in kMetaFirst (its merge is deferred)
+    const size_t piece = p.ml_layers > 0 ? static_cast<size_t>(meta[kMetaFirst])
+                                         : static_cast<size_t>(seg + cta);
     float *po = p.part_o + piece * G * D;
     for (int i = lane * 4; i < G * D; i += 128)
         *reinterpret_cast<float4 *>(po + i) = *reinterpret_cast<const float4 *>(ro + i);

@@ -109,6 +109,7 @@ struct mlkv_cache {
     unsigned *counters = nullptr;
     int *err = nullptr;
     int max_ctas = 0;           // capacity of the partial buffers beyond b*g pieces
+    long long records = 0;      // partial records the scratch holds
     // options
     int tile_tokens = 0;
     int grid = 0;
@@ -360,7 +361,11 @@ int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_d
     c->max_ctas = std::max(c->max_ctas, 4 * c->sm_count);
 
     c->cache_bytes = static_cast<size_t>(rows) * c->max_seq * c->d * 2;
-    const size_t pieces = static_cast<size_t>(c->b) * c->g + c->max_ctas;
+    // partial records: a stream-K layer needs b g + grid; a chunked multi-layer step l b g C,
+    // C chosen to fit (about 2.5 waves of chunks)
+    const size_t pieces =
+        std::max(static_cast<size_t>(c->b) * c->g + c->max_ctas, 3 * static_cast<size_t>(c->max_ctas));
+    c->records = static_cast<long long>(pieces);
     if ((e = cudaMalloc(&c->cache, c->cache_bytes)) != cudaSuccess ||
         (e = cudaMalloc(reinterpret_cast<void **>(&c->part_o),
                         pieces * c->G * c->d * sizeof(float))) != cudaSuccess ||
@@ -645,6 +650,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
 
     p.pf_own = 0;
     p.ml_layers = 0;
+    p.ml_chunks = 1;
     p.ml_seg_major = 0;
     p.ml_snake = 0;
     p.ml_slots = 0;
@@ -745,12 +751,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
         if (var == nullptr)
             return MLKV_OK;
     }
-    const int T = var->v->tile_tokens;
     const long long S = static_cast<long long>(c->b) * c->g;
-    const long long items = c->l * S;
-    const long long slots = static_cast<long long>(var->ctas_per_sm) * c->sm_count;
-    if (items > 0x7fffffffLL)
-        return MLKV_OK;
     // Sequences longest first (stable); items ranked segment-major over them.
     static thread_local std::vector<int> perm;
     perm.resize(c->b);
@@ -759,38 +760,76 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     if (!uniform)
         std::stable_sort(perm.begin(), perm.end(),
                          [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
-    // Grid: with one length the fewest CTAs that keep ceil(items / slots) items each; otherwise
-    // every resident slot.  Makespan in tiles: the heaviest CTA's items under the snake deal;
-    // per-layer launches split every layer over the machine but pay a launch, a ramp and merges
-    // per layer (about 4 tiles' time each; they overlap only in part).  A few long segments
-    // (batch 1 at long context) stay with the per-layer split.
-    const long long per = (items + slots - 1) / slots;
-    const int grid = static_cast<int>(uniform ? (items + per - 1) / per : std::min(items, slots));
-    long long total_tiles = 0;
-    for (int beta = 0; beta < c->b; ++beta)
-        total_tiles += static_cast<long long>(c->g) * ((seq_lens[beta] + T - 1) / T);
     // Segment-major ranks when the slots' visible rows do not fit in L2 (the block's layers then
     // share each segment's K/V while it is in L2); layer-major otherwise.  A snake deal balances
     // varied lengths.
     const long long all_kv = static_cast<long long>(c->m) * 2 * c->g * len_sum * c->d * 2;
     const int seg_major = all_kv > static_cast<long long>(c->l2_bytes) * 5 / 8 ? 1 : 0;
     const int snake = uniform ? 0 : 1;
-    long long heaviest = 0;
-    {
+    // A plan: tile length, chunks per segment, grid; its makespan in tiles is the heaviest CTA's
+    // items under the deal.  Grid: with one length the fewest CTAs that keep ceil(items / slots)
+    // items each; otherwise every resident slot.
+    struct Plan {
+        mlkv_cache::Variant *var;
+        int T, chunks, grid;
+        long long items, heaviest, per_layer;
+    };
+    auto plan_for = [&](mlkv_cache::Variant *v, int chunks) {
+        Plan pl{v, v->v->tile_tokens, chunks, 0, S * c->l * chunks, 0, 0};
+        const long long slots = static_cast<long long>(v->ctas_per_sm) * c->sm_count;
+        const long long per = (pl.items + slots - 1) / slots;
+        pl.grid = static_cast<int>(uniform ? (pl.items + per - 1) / per : std::min(pl.items, slots));
+        long long total_tiles = 0;
+        for (int beta = 0; beta < c->b; ++beta)
+            total_tiles += static_cast<long long>(c->g) * ((seq_lens[beta] + pl.T - 1) / pl.T);
+        // per-layer launches split every layer over the machine but pay a launch, a ramp and
+        // merges per layer (about 4 tiles' time each; they overlap only in part)
+        pl.per_layer = c->l * ((total_tiles + slots - 1) / slots + 4);
         static thread_local std::vector<long long> load;
-        load.assign(grid, 0);
+        load.assign(pl.grid, 0);
         const long long per_seq = static_cast<long long>(c->g) * c->l;
-        for (long long r = 0; r < items; ++r) {
-            const long long k = r / grid, i = r - k * grid;
-            const long long cta = (snake && (k & 1)) ? grid - 1 - i : i;
-            const long long pb = seg_major ? r / per_seq : (r % S) / c->g;
-            load[cta] += (seq_lens[perm[pb]] + T - 1) / T;
+        for (long long r = 0; r < pl.items; ++r) {
+            const long long k = r / pl.grid, i = r - k * pl.grid;
+            const long long cta = (snake && (k & 1)) ? pl.grid - 1 - i : i;
+            const long long rb = r / chunks, ch = r - rb * chunks;
+            const long long pb = seg_major ? rb / per_seq : (rb % S) / c->g;
+            const long long nt = (seq_lens[perm[pb]] + pl.T - 1) / pl.T;
+            load[cta] += (ch + 1) * nt / chunks - ch * nt / chunks;
         }
         for (long long x : load)
-            heaviest = std::max(heaviest, x);
+            pl.heaviest = std::max(pl.heaviest, x);
+        if (chunks > 1)
+            pl.heaviest += 4;   // the merge launch
+        return pl;
+    };
+    Plan pl = plan_for(var, 1);
+    if (uniform && pl.heaviest > pl.per_layer) {
+        // Few long segments (batch 1 at long context): split every segment into C chunks of the
+        // 128-position tile (two CTAs per SM), each a partial record, merged by one combine
+        // launch for the whole step -- about 2.5 waves of items, chunks of >= 8 tiles.
+        mlkv_cache::Variant *v128 = pick_variant(c, -1.0, 128);
+        if (v128 != nullptr && !v128->v->tc) {
+            const long long slots = static_cast<long long>(v128->ctas_per_sm) * c->sm_count;
+            const long long nt = (seq_lens[0] + 127) / 128;
+            long long C = (5 * slots + 2 * S * c->l - 1) / (2 * S * c->l);
+            C = std::min<long long>({C, nt / 8, mlkv::kCombineMaxPiecesHost,
+                                     static_cast<long long>(c->records) / (S * c->l)});
+            if (C > 1) {
+                Plan pc = plan_for(v128, static_cast<int>(C));
+                if (pc.heaviest <= pc.per_layer)
+                    pl = pc;
+            }
+        }
     }
-    if (heaviest > c->l * ((total_tiles + slots - 1) / slots + 4) || items * heaviest > 0x7fffffffLL)
+    if (pl.heaviest > pl.per_layer || pl.items > 0x7fffffffLL ||
+        pl.items * pl.heaviest > 0x7fffffffLL)
         return MLKV_OK;
+    var = pl.var;
+    const int T = pl.T;
+    const int grid = pl.grid;
+    long long total_tiles = 0;
+    for (int beta = 0; beta < c->b; ++beta)
+        total_tiles += static_cast<long long>(c->g) * ((seq_lens[beta] + T - 1) / T);
 
     static thread_local mlkv::DecodeParams p;
     p.Q = reinterpret_cast<const __nv_bfloat16 *>(Q);
@@ -817,7 +856,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     }
     p.tile_start[c->b] = 0;
     p.cluster_k = 0;
-    p.deferred_merge = 0;
+    p.deferred_merge = pl.chunks > 1 ? 1 : 0;
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.Q_next = nullptr;
@@ -830,6 +869,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     p.ml_slots = c->m;
     p.ml_seg_major = seg_major;
     p.ml_snake = snake;
+    p.ml_chunks = pl.chunks;
     p.ml_layers = c->l;
     p.ml_q_stride = static_cast<long long>(c->b) * c->h * c->d;
     p.ml_kv_stride = static_cast<long long>(c->b) * c->g * c->d;
@@ -856,11 +896,16 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
                             &var->tmap_rows, p, nullptr, c->pdl != 0);
     if (e != cudaSuccess)
         return fail_cuda(e, "decode launch (multi-layer step)");
+    if (p.deferred_merge) {
+        e = mlkv::launch_combine(p, c->d, static_cast<cudaStream_t>(stream), c->pdl != 0);
+        if (e != cudaSuccess)
+            return fail_cuda(e, "combine launch (multi-layer step)");
+    }
     c->last_grid = grid;
     c->last_tile = T;
     c->last_cluster_k = 0;
     c->last_tc = 0;
-    c->last_deferred = 0;
+    c->last_deferred = p.deferred_merge;
     c->last_l2_prefetch = p.pf_own;
     c->last_step_kernel = 1;
     c->last_seg_major = seg_major;

@@ -71,6 +71,10 @@ struct DecodeParams {
     int ml_layers;
     int ml_seg_major;         // 1: ranks segment-major (below); 0: layer-major, layer by layer
     int ml_snake;             // 1: snake deal of ranks to CTAs; 0: plain round-robin
+    int ml_chunks;            // C >= 1: every segment is C items (chunk c: tiles [c nt / C,
+                              // (c + 1) nt / C)); rank r is chunk r mod C of the item ranked
+                              // r / C.  With C > 1 every item writes a partial record at
+                              // (layer b g + beta g + j) C + c and combine_kernel merges them
     int ml_slots;             // owner slots the step reads (with pf_own: all prefetched into L2)
     long long ml_q_stride, ml_kv_stride;
     unsigned char ml_slot[kMaxStepLayers];

@@ -191,7 +191,13 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             const int L = p.uniform_len > 0
                               ? p.uniform_len
                               : p.seq_len[p.tile_start[TileWalk<T>::ml_seq_pos(p, r)]];
-            tile_hi += (L + T - 1) / T;
+            if (p.ml_chunks > 1) {
+                int a, b;
+                TileWalk<T>::ml_chunk(p, (L + T - 1) / T, r % p.ml_chunks, a, b);
+                tile_hi += b - a;
+            } else {
+                tile_hi += (L + T - 1) / T;
+            }
         }
     } else {
         tile_lo = narrow ? static_cast<int>(static_cast<uint32_t>(cta) * N / P)
@@ -374,7 +380,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             if (__shfl_sync(0xffffffffu, stop, 0))
                 break;
             // A later piece starts here: its query rows come with the tile.
-            issue_tile(wk, s, wk.tt == 0 && tile != tile_lo);
+            issue_tile(wk, s, wk.tt == wk.t0 && tile != tile_lo);
             ++issued;
             wk.next(p, s_len, s_start);
         }
@@ -445,6 +451,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
         const int L = wk.L;
         const int seg = beta * p.g + j;
         const int layer = wk.layer;
+        const int rec = wk.rec;   // partial-record index of a chunked multi-layer piece
+        const bool part = p.ml_chunks > 1;   // chunks are always partial records
         const int slot = slot_of(layer);
         const int store_new = ml ? static_cast<int>(p.ml_store[layer]) : p.store_new;
         const __nv_bfloat16 *k_new = p.K_new;
@@ -775,8 +783,9 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                     meta[kMetaBeta] = beta;
                     meta[kMetaJ] = j;
                     meta[kMetaSeg] = seg;
-                    meta[kMetaWhole] = (piece_first == seg_first && piece_end == seg_end) ? 1 : 0;
-                    meta[kMetaFirst] = cta_of_tile(seg_first, N, P);
+                    meta[kMetaWhole] =
+                        (piece_first == seg_first && piece_end == seg_end && !part) ? 1 : 0;
+                    meta[kMetaFirst] = ml ? rec : cta_of_tile(seg_first, N, P);
                     meta[kMetaLast] = cta_of_tile(seg_end - 1, N, P);
                     meta[kMetaStop] = 0;
                     meta[kMetaLayer] = layer;
@@ -811,7 +820,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 cluster_wait();   // the partner CTAs' barriers exist
             consumer_bar_sync<NCW>();
             const int ctid = threadIdx.x;
-            const bool whole = (piece_first == seg_first && piece_end == seg_end);
+            const bool whole = (piece_first == seg_first && piece_end == seg_end && !part);
             __nv_bfloat16 *ob = p.out + static_cast<size_t>(layer) * p.ml_q_stride +
                                 (static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G) * D;
             constexpr int kPairs = NCW * 32;   // float2 outputs per pass
@@ -828,7 +837,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 remote = map_to_rank(cslots + (rank - 1) * PL::kResBytes, 0);
                 remote_bar = map_to_rank(bar_cluster, 0);
             }
-            const size_t piece = static_cast<size_t>(seg + cta);
+            const size_t piece = ml ? static_cast<size_t>(rec) : static_cast<size_t>(seg + cta);
             float *po = p.part_o + piece * G * D;
 #pragma unroll 2
             for (int i = 2 * ctid; i < G * D; i += 2 * kPairs) {
@@ -1004,21 +1013,37 @@ __global__ void __launch_bounds__(kCombineThreads)
     // writes partials only after its own dependency wait (after this grid).
     grid_dependents_launch();
     grid_dependency_wait();
-    const int seg = blockIdx.x;
     const int row = blockIdx.y;
     const int G = p.G;
-    const int T = p.tile_tokens;
+    int seg, np;
+    size_t rec0;
+    __nv_bfloat16 *out = p.out;
+    if (p.ml_layers > 0) {
+        // a chunked multi-layer launch: blockIdx.x = layer b g + beta g + j, chunk records
+        // blockIdx.x C .. blockIdx.x C + C - 1
+        const int S = p.b * p.g;
+        const int layer = static_cast<int>(blockIdx.x) / S;
+        seg = static_cast<int>(blockIdx.x) - layer * S;
+        out += static_cast<size_t>(layer) * p.ml_q_stride;
+        np = p.ml_chunks;
+        rec0 = static_cast<size_t>(blockIdx.x) * p.ml_chunks;
+    } else {
+        seg = blockIdx.x;
+        const int T = p.tile_tokens;
+        const int beta = seg / p.g;
+        const int jj = seg - beta * p.g;
+        const int L = p.uniform_len > 0 ? p.uniform_len : p.seq_len[beta];
+        const int nt = (L + T - 1) / T;
+        const int seg_first = p.uniform_len > 0 ? seg * nt : p.tile_start[beta] + jj * nt;
+        const int c_first = cta_of_tile(seg_first, p.num_tiles, p.decode_grid);
+        const int c_last = cta_of_tile(seg_first + nt - 1, p.num_tiles, p.decode_grid);
+        if (c_first == c_last)
+            return;   // one CTA held the whole segment and wrote the output itself
+        np = c_last - c_first + 1;
+        rec0 = static_cast<size_t>(seg + c_first);
+    }
     const int beta = seg / p.g;
     const int j = seg - beta * p.g;
-    const int L = p.uniform_len > 0 ? p.uniform_len : p.seq_len[beta];
-    const int nt = (L + T - 1) / T;
-    const int seg_first = p.uniform_len > 0 ? seg * nt : p.tile_start[beta] + j * nt;
-    const int c_first = cta_of_tile(seg_first, p.num_tiles, p.decode_grid);
-    const int c_last = cta_of_tile(seg_first + nt - 1, p.num_tiles, p.decode_grid);
-    if (c_first == c_last)
-        return;   // one CTA held the whole segment and wrote the output itself
-    const int np = c_last - c_first + 1;
-    const size_t rec0 = static_cast<size_t>(seg + c_first);
     const int tid = threadIdx.x;
     const float NEG_INF = -__int_as_float(0x7f800000);
 
@@ -1079,7 +1104,7 @@ __global__ void __launch_bounds__(kCombineThreads)
 #pragma unroll
         for (int q = 0; q < kGroups; ++q)
             sum += s_red[q * D + e];
-        p.out[(static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G + row) * D + e] =
+        out[(static_cast<size_t>(beta) * p.h + static_cast<size_t>(j) * G + row) * D + e] =
             __float2bfloat16_rn(sum * inv);
     }
 }
@@ -1227,7 +1252,8 @@ int max_pieces_per_segment(const DecodeParams &p, int T, int grid)
 cudaError_t launch_combine(const DecodeParams &p, int head_dim, cudaStream_t stream, bool pdl)
 {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(p.b * p.g), static_cast<unsigned>(p.G));
+    const int segs = p.b * p.g * (p.ml_layers > 0 ? p.ml_layers : 1);
+    cfg.gridDim = dim3(static_cast<unsigned>(segs), static_cast<unsigned>(p.G));
     cfg.blockDim = dim3(kCombineThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

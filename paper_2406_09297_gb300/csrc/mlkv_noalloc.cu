@@ -257,6 +257,7 @@ extern "C" int mlkv_decode_attention_static(const void *kv_slot, int batch, int 
     p.store_new = 0;
     p.pf_own = 0;
     p.ml_layers = 0;
+    p.ml_chunks = 1;
     p.ml_seg_major = 0;
     p.ml_snake = 0;
     p.ml_slots = 0;
