@@ -242,10 +242,11 @@ def _kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def _recorded_traffic(w, kernel):
+def _recorded_traffic(w, kernel, launch):
     """DRAM bytes per decode launch (dram__bytes_read.sum + dram__bytes_write.sum) from the ncu
-    capture recorded in profiles/decode_traffic.json for this workload and kernel, or None when
-    there is none or the kernel source changed since it was taken."""
+    capture recorded in profiles/decode_traffic.json for this workload, kernel and launch kind
+    ("multi-layer": one launch for the step, "per-layer"), or None when there is none or the
+    kernel source changed since it was taken."""
     try:
         with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
             rec = json.load(f)
@@ -254,7 +255,7 @@ def _recorded_traffic(w, kernel):
     entry = rec.get(w.name)
     if not entry or entry.get("kernel_source_sha256_16") != _kernel_source_hash():
         return None
-    if entry.get("kernel", "decode_kernel") != kernel:
+    if entry.get("kernel", "decode_kernel") != kernel or entry.get("launch") != launch:
         return None
     return entry.get("dram_bytes_per_launch")
 
@@ -310,8 +311,10 @@ def run(args, w):
     step()
     cache.sync_status()
     step_kernel = bool(cache.get_option("last_step_kernel"))   # one launch for every layer
-    launches_per_step = 1 if step_kernel else (
-        w.l * (2 if cache.get_option("last_deferred_merge") else 1))
+    # a decode launch per layer, or one for the whole step; each followed by a merge launch when
+    # the split pieces' partials are merged after the decode (deferred merge)
+    merges = 2 if cache.get_option("last_deferred_merge") else 1
+    launches_per_step = merges * (1 if step_kernel else w.l)
 
     def barrier():
         if dist is not None:
@@ -356,7 +359,7 @@ def run(args, w):
     torch.cuda.synchronize()
     kms = [[a.elapsed_time(b) for a, b in row] for row in kev]
     layer_ms = [statistics.median(kms[k][n] for k in range(args.steps)) for n in range(w.l)]
-    mean_kernel_ms = ms / w.l   # decode launches (a combine launch, if any, rides with each)
+    mean_kernel_ms = ms / w.l   # per layer; a merge launch, if any, is counted in with its decode
     kv_layer = kv_bytes_per_layer(w, seq_lens)
     qo_layer = 2 * w.b * w.h * w.d * 2
     alg_bytes = kv_layer + qo_layer
@@ -378,7 +381,7 @@ def run(args, w):
                                                       "step_kernel", "l2_persist_bytes",
                                                       "l2_window_max", "last_step_kernel",
                                                       "last_seg_major")}
-    traffic = _recorded_traffic(w, kernel_name)
+    traffic = _recorded_traffic(w, kernel_name, "multi-layer" if step_kernel else "per-layer")
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
     host_q = Qs.cpu().pin_memory()
@@ -429,6 +432,8 @@ def run(args, w):
                          "frac_vs_8tbs": achieved / 8000.0,
                          "kernel": kernel_name, "alg_bytes_per_launch": launch_bytes,
                          "mean_launch_ms": launch_ms, "launches_per_step": launches_per_step,
+                         # the merge launch's time is inside mean_launch_ms (timed together)
+                         "merge_time_included": merges == 2,
                          "step_ms_per_layer": mean_kernel_ms,
                          "dram_unique_bytes_per_step": unique_bytes,
                          "dram_unique_gbs": unique_gbs,

@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(TcPlan<D, T, STAGES>::kThreads, 1)
     const int tile_lo = static_cast<int>(static_cast<long long>(cta) * N / P);
     const int tile_hi = static_cast<int>(static_cast<long long>(cta + 1) * N / P);
     const int G = p.G;
-    const bool early = p.early_fetch != 0;
+    const bool early = p.early_fetch == 1;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {

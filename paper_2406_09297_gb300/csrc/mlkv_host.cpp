@@ -725,8 +725,11 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
 // scratch is shared; every layer takes its segments' newest rows from the step's new tokens,
 // and owner layers store them.  *done tells whether it was issued.  With in_ready, the launch
 // waits for it (queries still arriving).
+// With `stage`, the copy of the step's inputs it describes is launched right before the step's
+// kernel, which may then start (and fetch its first cache tiles) while the copy runs.
 static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
-                         const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done)
+                         const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
+                         const mlkv::StageParams *stage = nullptr)
 {
     *done = false;
     c->last_step_kernel = 0;
@@ -860,7 +863,8 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     p.tile_tokens = T;
     p.decode_grid = grid;
     p.Q_next = nullptr;
-    p.early_fetch = 0;
+    // After this library's input copy the first tile of each CTA goes out before the wait.
+    p.early_fetch = (stage != nullptr && c->pdl) ? 2 : 0;
     p.newest_ready = 1;
     p.store_new = 0;
     // L2 prefetch of every slot's visible rows when they all fit with room to spare.
@@ -891,6 +895,9 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     if (e != cudaSuccess)
         return fail_cuda(e, "step event");
     DeviceGuard guard(c->device);
+    if (stage != nullptr && (e = mlkv::launch_stage_copy(*stage, static_cast<cudaStream_t>(stream))) !=
+                                cudaSuccess)
+        return fail_cuda(e, "copy-in of the step's inputs");
     const size_t smem = var->v->smem_bytes + (uniform ? 0 : mlkv::table_bytes(c->b));
     e = mlkv::launch_decode(*var->v, grid, smem, static_cast<cudaStream_t>(stream), &var->tmap,
                             &var->tmap_rows, p, nullptr, c->pdl != 0);
@@ -1144,8 +1151,20 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
     }
     auto issue = [&](cudaStream_t s) {
         if (mapped) {
-            // Layer 0's queries and the new tokens first; the other layers' queries on a side
-            // branch while layer 0 runs (joined before layer 1).
+            // One multi-layer launch: a single copy of every input right before it.
+            mlkv::StageParams all{};
+            all.n = 3;
+            all.src[0] = dev[0]; all.dst[0] = dq; all.bytes[0] = qo_bytes;
+            all.src[1] = dev[1]; all.dst[1] = dk; all.bytes[1] = kv_bytes;
+            all.src[2] = dev[2]; all.dst[2] = dv; all.bytes[2] = kv_bytes;
+            bool done = false;
+            const int rc = issue_step_ml(c, dq, dk, dv,
+                                         static_cast<char *>(const_cast<void *>(dev[3])), seq_lens,
+                                         s, nullptr, &done, &all);
+            if (rc != MLKV_OK || done)
+                return rc;
+            // Per-layer launches: layer 0's queries and the new tokens first; the other layers'
+            // queries on a side branch while layer 0 runs (joined before layer 1).
             const size_t q1 = qo_bytes / c->l;   // one layer
             const bool split = c->l > 1;
             mlkv::StageParams a{};

@@ -46,7 +46,9 @@ struct DecodeParams {
     int early_fetch;          // 1: the previous kernel is this library's decode of the preceding
                               // layer, which writes neither Q nor any cache row but a segment's
                               // newest: Q and the tiles without that row are read before the
-                              // dependency wait
+                              // dependency wait.  2: the previous kernel is this library's copy of
+                              // the step's inputs (Q, K_new, V_new), which writes no cache row:
+                              // only the CTA's first tile is fetched before the wait
     int newest_ready;         // 1: the segments' newest rows are replaced from K_new/V_new by this
                               // grid: no wait before a segment's last tile
     int store_new;            // with K_new: 1 = also store the new token in the cache (the owner

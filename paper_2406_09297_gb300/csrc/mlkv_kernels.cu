@@ -212,7 +212,8 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
     };
     auto slot_of = [&](int layer) { return ml ? static_cast<int>(p.ml_slot[layer]) : p.slot; };
 
-    const bool early = p.early_fetch != 0;
+    const bool early = p.early_fetch == 1;
+    const bool pre_tile = p.early_fetch != 0;   // the first tile may go out before the wait
     // The producer warp's copy of one tile into stage `s` (query rows too when a later piece
     // starts); called by all 32 lanes with the same arguments.  On GB300 one issuing thread
     // completes about one bulk copy per ~0.5 us whatever its size (measured: 8 to 64 KB, from L2
@@ -259,9 +260,10 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
                 bulk_load(sbase + PL::kQ + s * PL::kQSlot + r * PL::kQRow, q0 + r * D, D * 2, fb);
         }
     };
-    // The ring's barriers belong to the producer warp's lane 0.  With early fetch and one length
-    // for every sequence the warp also sends its first tile before the CTA barrier: a CTA that got its SM late
-    // (the last ones of a layer decide the layer's end) then has data on the way at once.
+    // The ring's barriers belong to the producer warp's lane 0.  With early fetch (either kind) and
+    // one length for every sequence the warp also sends its first tile before the CTA barrier: a
+    // CTA that got its SM late (the last ones of a layer decide the layer's end), or one that
+    // starts while the step's inputs are still being copied in, then has data on the way at once.
     bool pre_issued = false;
     // The trigger comes first: the next launch (inside a decode step, the next layer's decode)
     // may start as soon as every CTA of this grid is resident.  What it reads before its own
@@ -279,7 +281,7 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
             fence_barrier_init();
         }
         __syncwarp();
-        if (early && p.uniform_len > 0 && tile_lo < tile_hi) {
+        if (pre_tile && p.uniform_len > 0 && tile_lo < tile_hi) {
             TileWalk<T> w0;
             w0.init(p, s_len, s_start, tile_lo);
             if (w0.tt != w0.nt - 1 || p.newest_ready) {   // not a newest row still to wait for

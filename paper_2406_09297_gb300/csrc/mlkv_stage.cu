@@ -2,7 +2,7 @@
 // as kernels: for the small tensors of one decode step (a few MB), a copy-engine transfer costs
 // ~12 us of fixed latency each, while a kernel of plain 16-byte loads and stores over the
 // CPU-GPU link costs a launch.  Used by mlkv_decode_step_host to bring a step's Q and new K/V in
-// (one launch for all three) and every layer's output out (one launch).
+// (one launch for all three); the decode kernels store the outputs into host memory themselves.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -13,6 +13,9 @@ namespace {
 
 __global__ void __launch_bounds__(256) stage_copy_kernel(const __grid_constant__ StageParams p)
 {
+    // The next launch (the step's decode) may start at once: it reads nothing this kernel writes
+    // before its own dependency wait, which returns only once this grid has finished.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const size_t stride = static_cast<size_t>(gridDim.x) * blockDim.x;
     for (int s = 0; s < p.n; ++s) {
         const uint4 *src = static_cast<const uint4 *>(p.src[s]);

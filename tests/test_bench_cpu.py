@@ -46,3 +46,24 @@ def test_reference_arm_line():
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["cpu_baseline"]["value"] == pytest.approx(line["value"])
     assert line["config"]["workload"] == SMALL
+
+
+def test_recorded_traffic_needs_current_kernel_and_launch_kind():
+    """The roofline's `traffic` is taken from a recorded ncu capture only when the capture was of
+    the kernel sources as they are and of the same launch kind (one multi-layer launch per step,
+    or one launch per layer); otherwise it is null."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from mlkv_synth import workloads
+    with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
+        rec = json.load(f)
+    for name, entry in rec.items():
+        assert entry["launch"] in ("multi-layer", "per-layer")
+        assert entry["dram_bytes_per_launch"] > 0
+        w = workloads.by_name(name)
+        current = entry["kernel_source_sha256_16"] == bench._kernel_source_hash()
+        got = bench._recorded_traffic(w, entry["kernel"], entry["launch"])
+        assert got == (entry["dram_bytes_per_launch"] if current else None)
+        other = "per-layer" if entry["launch"] == "multi-layer" else "multi-layer"
+        assert bench._recorded_traffic(w, entry["kernel"], other) is None
+        assert bench._recorded_traffic(w, "no_such_kernel", entry["launch"]) is None
