@@ -32,8 +32,8 @@
 // scores, and their V rows are zeroed in shared memory so that 0 * V stays 0.
 //
 // Warp roles (384 threads): warps 0-3 query tile A, 4-7 query tile B (softmax and output), warp 8
-// TMA producer (both query tiles, then K_0, V_0, K_1, V_1, ... through a ring), warp 9 MMA issuer,
-// warps 10-11 idle.  The block launches with 168 registers a thread (three warps per SM
+// TMA producer (both query tiles, then K_0, V_0, K_1, V_1, ... through a ring), warp 9 MMA issuer
+// (for head_dim 64 only of S; warp 10 then issues the P V products), the rest idle.  The block launches with 168 registers a thread (three warps per SM
 // sub-partition); the last warpgroup gives registers back (72 or 88) and the softmax warpgroups
 // take them (216 or 208, head_dim 64 or 128): 128 * low + 256 * high <= 384 * 168.
 // Every wait is bounded; on expiry the kernel records an error bit, stops, lets its copies and MMAs
@@ -56,9 +56,9 @@ struct PrefillPlan {
     static constexpr int kQ = 0;                             // [2] query tiles
     static constexpr int kRing = kQ + 2 * kTileBytes;
     static constexpr int kFlags = kRing + kRingTiles * kTileBytes;   // int [4], TMEM base at +16
-    // u64 barriers: q, full[R], empty[R], s_ready[2], s_free[2], p_ready[2], pv_done[2], fin
+    // u64 barriers: q, full[R], empty[R], s_ready[2], s_free[2], p_ready[2], pv_done[2], fin[2]
     static constexpr int kBars = kFlags + 32;
-    static constexpr int kNumBars = 1 + 2 * kRingTiles + 8 + 1;
+    static constexpr int kNumBars = 1 + 2 * kRingTiles + 8 + 2;
     static constexpr int kBytes = kBars + kNumBars * 8;
     static constexpr int kAlloc = kBytes + 1024;             // base aligned up to 1024
     static constexpr int kTmemCols = 512;
@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     const uint32_t bar_s_free = bar_s_ready + 16;
     const uint32_t bar_p_ready = bar_s_free + 16;
     const uint32_t bar_pv_done = bar_p_ready + 16;
-    const uint32_t bar_fin = bar_pv_done + 16;
+    const uint32_t bar_fin = bar_pv_done + 16;   // [2]: one per issuing thread
     volatile int *flags = reinterpret_cast<volatile int *>(smem + PL::kFlags);
 
     const int warp = threadIdx.x >> 5;
@@ -151,6 +151,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             mbar_init(bar_pv_done + 8 * g, 1);
         }
         mbar_init(bar_fin, 1);
+        mbar_init(bar_fin + 8, 1);
         flags[0] = 0;
         fence_barrier_init();
     }
@@ -242,9 +243,16 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                     atomicOr(p.err, kErrDrain);
         }
         __syncwarp();
-    } else if (warp == PL::kMma) {
-        // ------------------------------------ MMA issuer ----------------------------------------
+    } else if (warp == PL::kMma || (PL::kPSep && warp == PL::kMma + 1)) {
+        // ------------------------------------ MMA issuers ---------------------------------------
+        // With P in columns of its own (head_dim 64) warp kMma issues every S = Q K^T and warp
+        // kMma + 1 every O += P V: the two never touch the same tensor-memory columns, each waits
+        // only for what its own products need, and the tensor core gets both streams.  (One thread
+        // issuing both spent about a third of each key tile on barrier checks while the tensor core
+        // ran dry.)  With P over S (head_dim 128) one thread issues both, in order.
         setmaxnreg_dec<PL::kRegsLow>();
+        const bool do_s = warp == PL::kMma, do_pv = !PL::kPSep || warp == PL::kMma + 1;
+        const uint32_t my_fin = bar_fin + (warp == PL::kMma ? 0 : 8);
         if (lane == 0) {
             constexpr uint32_t kIdS = umma_idesc(128, 128, 0, 0);
             constexpr uint32_t kIdPV = umma_idesc(128, D, 0, 1);
@@ -263,7 +271,18 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                     ok = false;
                 return ok;
             };
-            auto tile_full = [&](int idx) { return wait(bar_full + 8 * (idx % R), idx / R); };
+            // Each ring tile is checked once: the K tile serves both query tiles' S, the V tile
+            // both P V (a check costs ~150 cycles while the MMAs keep shared memory busy).
+            int seen0 = -1, seen1 = -1;
+            auto tile_full = [&](int idx) {
+                if (idx == seen0 || idx == seen1)
+                    return ok;
+                if (wait(bar_full + 8 * (idx % R), idx / R)) {
+                    seen1 = seen0;
+                    seen0 = idx;
+                }
+                return ok;
+            };
             auto issue_s = [&](int g, int t) {
                 const uint64_t qa = dq + g * kSlot;
                 const uint64_t kb = dk + ((2 * t) % R) * kSlot;
@@ -285,7 +304,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 if (PL::kPSep || last)
                     umma_commit(bar_pv_done + 8 * g);
             };
-            if (wait(bar_q, 0) && tile_full(0)) {
+            if (do_s && wait(bar_q, 0) && tile_full(0)) {
                 tmem_fence_after();
                 if (n_a > 0)
                     issue_s(0, 0);
@@ -295,13 +314,12 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             // complete), not by commits: a commit costs the tensor pipe about as much as a short MMA.
             for (int t = 0; ok && t < n_b; ++t) {
                 if (PL::kPSep) {
-                    // Both tiles' next S as soon as each tile's S has been read (early in its
-                    // softmax), then both P V as their P arrive: neither softmax waits for the
-                    // other tile's P before its next scores are computed.
+                    // S issuer: both tiles' next S as soon as each tile's S has been read (early in
+                    // its softmax).  P V issuer: both P V as their P arrive.
 #pragma unroll
                     for (int g = 0; g < 2; ++g) {
                         const int ng = g ? n_b : n_a;
-                        if (!ok || t + 1 >= ng)
+                        if (!do_s || !ok || t + 1 >= ng)
                             continue;
                         if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
                             break;
@@ -311,7 +329,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
 #pragma unroll
                     for (int g = 0; g < 2; ++g) {
                         const int ng = g ? n_b : n_a;
-                        if (!ok || t >= ng)
+                        if (!do_pv || !ok || t >= ng)
                             continue;
                         if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
                             break;
@@ -342,8 +360,8 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 flags[0] = 1;
                 atomicOr(p.err, kErrWaitFull);
             }
-            umma_commit(bar_fin);
-            if (!mbar_wait(bar_fin, 0))
+            umma_commit(my_fin);
+            if (!mbar_wait(my_fin, 0))
                 atomicOr(p.err, kErrDrain);
         }
         __syncwarp();
@@ -443,22 +461,13 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 l_run *= alpha;
                 m_run = m_new;
             }
-            // The P buffer of the previous tile must have been read by its P V.
-            if (PL::kPSep && t > 0) {
-                wait(pv_done, t - 1);
-                if (releaser) {
-                    mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
-                    mbar_arrive(bar_empty + 8 * ((2 * t) % R));
-                }
-            }
-            tmem_fence_after();
             const float2 sc2 = make_float2(scale, scale);
             const float2 nm2 = make_float2(-m_run, -m_run);
             float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                              make_float2(0.f, 0.f)};
+            uint32_t w[2][32];
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
-                uint32_t w[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const int c = half * 64 + 2 * i;   // keys c, c + 1
@@ -467,10 +476,21 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                                    nm2);
                     const float2 pr = make_float2(fast_exp2(x.x), fast_exp2(x.y));
                     acc[i & 3] = __fadd2_rn(acc[i & 3], pr);
-                    w[i] = pack_bf16x2(pr.x, pr.y);
+                    w[half][i] = pack_bf16x2(pr.x, pr.y);
                 }
-                tmem_st32_nowait(col_p + half * 32, w);
             }
+            // The P buffer of the previous tile must have been read by its P V; the weights above
+            // were computed while that product ran.
+            if (PL::kPSep && t > 0) {
+                wait(pv_done, t - 1);
+                if (releaser) {
+                    mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
+                    mbar_arrive(bar_empty + 8 * ((2 * t) % R));
+                }
+            }
+            tmem_fence_after();
+            tmem_st32_nowait(col_p, w[0]);
+            tmem_st32_nowait(col_p + 32, w[1]);
             const float2 s01 = __fadd2_rn(acc[0], acc[1]), s23 = __fadd2_rn(acc[2], acc[3]);
             const float2 s4 = __fadd2_rn(s01, s23);
             l_run += s4.x + s4.y;
@@ -550,7 +570,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             tmem_fence_before();
         }
     } else {
-        setmaxnreg_dec<PL::kRegsLow>();   // warps 10-11: no role
+        setmaxnreg_dec<PL::kRegsLow>();   // warp 11 (and 10 with head_dim 128): no role
     }
 
     __syncthreads();
