@@ -660,19 +660,26 @@ size_t prefill_smem_bytes(int head_dim)
     return head_dim == 64 ? PrefillPlan<64>::kAlloc : PrefillPlan<128>::kAlloc;
 }
 
-cudaError_t prepare_prefill(int head_dim)
+// The warpgroups' register split (setmaxnreg) adds up to the registers the block is launched with;
+// a kernel built with another per-thread count would wait forever in setmaxnreg.inc, so it is
+// refused here instead of launched.
+cudaError_t prepare(int head_dim, bool fused)
 {
-    return cudaFuncSetAttribute(kernel_fn(head_dim, false),
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, kernel_fn(head_dim, fused));
+    if (e != cudaSuccess)
+        return e;
+    const int want = head_dim == 64 ? PrefillPlan<64>::kRegsLaunch : PrefillPlan<128>::kRegsLaunch;
+    if (fa.numRegs != want)
+        return cudaErrorInvalidKernelImage;
+    return cudaFuncSetAttribute(kernel_fn(head_dim, fused),
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(prefill_smem_bytes(head_dim)));
 }
 
-cudaError_t prepare_fused(int head_dim)
-{
-    return cudaFuncSetAttribute(kernel_fn(head_dim, true),
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(prefill_smem_bytes(head_dim)));
-}
+cudaError_t prepare_prefill(int head_dim) { return prepare(head_dim, false); }
+
+cudaError_t prepare_fused(int head_dim) { return prepare(head_dim, true); }
 
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream)
