@@ -1344,16 +1344,18 @@ int mlkv_prefill(mlkv_cache_t c, int layer, const void *Q, const void *K, const 
     p.fused_L = p.fused_L1 = 0;
     for (int beta = 0; beta < c->b; ++beta)
         p.prompt_len[beta] = prompt_lens[beta];
-    // Work units, those that see the most keys first: two heads of a group at the same block when
-    // the group size is even, else the blocks 2p and 2p+1 of one head (the unit of block 2p+1).
-    p.head_pairs = (c->G % 2 == 0) ? 1 : 0;
+    // Work units, those that see the most keys first.  head_dim 64: one query block of one head
+    // per CTA (two CTAs per SM).  head_dim 128: two heads of a group at the same block when the
+    // group size is even, else the blocks 2p and 2p+1 of one head (the unit of block 2p+1).
+    const bool one_tile = c->d == 64;
+    p.head_pairs = (!one_tile && c->G % 2 == 0) ? 1 : 0;
     const int sels = p.head_pairs ? c->h / 2 : c->h;
     const int max_blocks = (max_len + 127) / 128;
     int n = 0;
     for (int qb = max_blocks - 1; qb >= 0; --qb) {
         for (int beta = 0; beta < c->b; ++beta) {
             const int nb = (prompt_lens[beta] + 127) / 128;
-            if (qb >= nb || (!p.head_pairs && qb % 2 == 0 && qb != nb - 1))
+            if (qb >= nb || (!one_tile && !p.head_pairs && qb % 2 == 0 && qb != nb - 1))
                 continue;
             for (int sel = 0; sel < sels; ++sel) {
                 p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(qb) << 10) |

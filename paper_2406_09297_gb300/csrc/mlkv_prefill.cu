@@ -5,11 +5,14 @@
 // attention, Eqs. 2-3 with the MLKV maps of Eqs. 13-18).  Owner layers first store the prompt's
 // K/V in their slot (mlkv_host.cpp); every layer of the block then attends over it.
 //
-// Work unit (one CTA): two query tiles A and B of 128 prompt positions that read the same KV head,
-// so that every K/V tile is loaded once for both.  With an even group size G they are two heads of
-// one group at the same positions (identical causal triangles); otherwise they are the blocks
-// 2p and 2p+1 of one head (B sees one tile more; a last block without a partner runs alone as B).
-// Units that see the most keys run first.
+// Work unit (one CTA), head_dim 128 and the fused decode: two query tiles A and B of 128 prompt
+// positions that read the same KV head, so that every K/V tile is loaded once for both.  With an
+// even group size G they are two heads of one group at the same positions (identical causal
+// triangles); otherwise they are the blocks 2p and 2p+1 of one head (B sees one tile more; a last
+// block without a partner runs alone as B).  Prefill at head_dim 64: one query tile (as B) per CTA
+// and two CTAs per SM, each with half the tensor memory; the two CTAs' starts, first loads and
+// outputs overlap each other's key-tile loops (measured 8% faster than two tiles per CTA, although
+// every K/V tile is then fetched once per query tile).  Units that see the most keys run first.
 //
 // Per key tile t and query tile X (all MMAs tcgen05.mma kind::f16, bf16 in, fp32 accumulate):
 //   S_X = Q_X K_t^T  M = 128 queries (A = Q_X, K-major, 128-byte swizzle as TMA wrote it),
@@ -23,19 +26,21 @@
 //                    N = head_dim, K = 128 keys; O_X stays in TMEM for the whole unit.
 // While one warpgroup turns S into P, the tensor core works on the other query tile.
 //
-// TMEM (512 columns): S_A, S_B (128 each), O_A, O_B (head_dim each).  For head_dim 64, P has
-// columns of its own (so S of the next tile can be computed while P of this one is being written);
-// for head_dim 128, P overwrites the first 64 columns of its S (tcgen05.mma of one thread execute
-// in order, so S of the next tile is written after P V has read P).
+// TMEM (512 columns, 256 with one query tile): S per tile (128 columns), O per tile (head_dim).
+// For head_dim 64, P has columns of its own (so S of the next tile can be computed while P of this
+// one is being written); for head_dim 128, P overwrites the first 64 columns of its S (tcgen05.mma
+// of one thread execute in order, so S of the next tile is written after P V has read P).
 //
 // The diagonal tile masks keys after the query; keys past the prompt's end only meet such masked
 // scores, and their V rows are zeroed in shared memory so that 0 * V stays 0.
 //
-// Warp roles (384 threads): warps 0-3 query tile A, 4-7 query tile B (softmax and output), warp 8
-// TMA producer (both query tiles, then K_0, V_0, K_1, V_1, ... through a ring), warp 9 MMA issuer
-// (for head_dim 64 only of S; warp 10 then issues the P V products), the rest idle.  The block launches with 168 registers a thread (three warps per SM
-// sub-partition); the last warpgroup gives registers back (72 or 88) and the softmax warpgroups
-// take them (216 or 208, head_dim 64 or 128): 128 * low + 256 * high <= 384 * 168.
+// Warp roles: 4 softmax warps per query tile (warps 0-3 tile A, 4-7 tile B; the one-tile CTA's
+// warps 0-3 take its tile), then the TMA producer (query tiles, then K_0, V_0, K_1, V_1, ...
+// through a ring), the MMA issuer (for head_dim 64 only of S, the next warp issuing the P V
+// products), the rest idle.  Registers: the two-tile block launches with 168 a thread and its last
+// warpgroup gives registers back (72 or 88) to the softmax warpgroups (216 or 208, head_dim 64 or
+// 128): 128 * low + 256 * high <= 384 * 168; the one-tile block launches with 128 (two blocks per
+// SM) and splits 56 / 200: 128 * 56 + 128 * 200 = 256 * 128.
 // Every wait is bounded; on expiry the kernel records an error bit, stops, lets its copies and MMAs
 // land and frees its TMEM.
 #include "mlkv_device.cuh"
@@ -44,32 +49,45 @@
 namespace mlkv {
 namespace {
 
-template <int D>
+// kOne: one query tile per CTA and two CTAs per SM (prefill at head_dim 64): each CTA holds half
+// the tensor memory and a third of the registers of the two-tile form, and two independent CTAs
+// hide each other's start, first loads and output; the key tiles are fetched once per query tile.
+// Otherwise two query tiles per CTA share every K/V tile, one CTA per SM.
+template <int D, bool kOne>
 struct PrefillPlan {
-    static constexpr int kThreads = 12 * 32;
-    static constexpr int kRegsLaunch = 168;
-    static constexpr int kRegsLow = D == 64 ? 72 : 88, kRegsHigh = D == 64 ? 216 : 208;
-    static constexpr int kProducer = 8, kMma = 9;
+    static constexpr int kTiles = kOne ? 1 : 2;              // query tiles per CTA
+    static constexpr int kSoftWarps = 4 * kTiles;
+    static constexpr int kThreads = (kSoftWarps + 4) * 32;
+    static constexpr int kMinBlocks = kOne ? 2 : 1;
+    static constexpr int kRegsLaunch = kOne ? 128 : 168;
+    static constexpr int kRegsLow = kOne ? 56 : (D == 64 ? 72 : 88);
+    static constexpr int kRegsHigh = kOne ? 200 : (D == 64 ? 216 : 208);
+    static constexpr int kProducer = kSoftWarps, kMma = kSoftWarps + 1;
     static constexpr int kSub = D / 64;                      // 64-channel blocks of a row
     static constexpr int kTileBytes = 128 * D * 2;           // 128 rows of Q, K or V
-    static constexpr int kRingTiles = D == 64 ? 8 : 4;       // K_t and V_t alternate in the ring
-    static constexpr int kQ = 0;                             // [2] query tiles
-    static constexpr int kRing = kQ + 2 * kTileBytes;
+    static constexpr int kRingTiles = kOne ? 5 : (D == 64 ? 8 : 4);   // K_t and V_t alternate
+    static constexpr int kQ = 0;                             // [kTiles] query tiles
+    static constexpr int kRing = kQ + kTiles * kTileBytes;
     static constexpr int kFlags = kRing + kRingTiles * kTileBytes;   // int [4], TMEM base at +16
     // u64 barriers: q, full[R], empty[R], s_ready[2], s_free[2], p_ready[2], pv_done[2], fin[2]
     static constexpr int kBars = kFlags + 32;
     static constexpr int kNumBars = 1 + 2 * kRingTiles + 8 + 2;
     static constexpr int kBytes = kBars + kNumBars * 8;
     static constexpr int kAlloc = kBytes + 1024;             // base aligned up to 1024
-    static constexpr int kTmemCols = 512;
+    static_assert(kMinBlocks * (kAlloc + 1024) <= 228 * 1024, "shared memory of the resident CTAs");
+    static constexpr int kTmemCols = kOne ? 256 : 512;
     static constexpr bool kPSep = D == 64;                   // P in columns of its own
     static constexpr int kColS = 0;                          // + 128 per query tile
-    static constexpr int kColO = 256;                        // + D per query tile
-    static constexpr int kColP = 384;                        // + 64 per query tile (kPSep)
+    static constexpr int kColO = 128 * kTiles;               // + D per query tile
+    static constexpr int kColP = kColO + D * kTiles;         // + 64 per query tile (kPSep)
     static_assert(D == 64 || D == 128, "head_dim 64 or 128");
+    static_assert(!kOne || D == 64, "one query tile per CTA only at head_dim 64");
     static_assert(kRing % 1024 == 0 && kTileBytes % 1024 == 0, "swizzled tiles 1024-aligned");
-    static_assert(kColO + 2 * D <= (kPSep ? kColP : kTmemCols), "TMEM columns overlap");
-    static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kRegsLaunch, "register split");
+    static_assert((kPSep ? kColP + 64 * kTiles : kColO + D * kTiles) <= kTmemCols,
+                  "TMEM columns overlap");
+    static_assert(128 * kRegsLow + 32 * kSoftWarps * kRegsHigh <= kThreads * kRegsLaunch,
+                  "register split");
+    static_assert(kMinBlocks * kThreads * kRegsLaunch <= 65536, "registers of the resident CTAs");
 };
 
 template <int N>
@@ -91,13 +109,20 @@ __device__ __forceinline__ float max3f(float a, float b, float c)
     return d;
 }
 
+// The plan of a launch: one query tile per CTA for the head_dim 64 prefill.
 template <int D, bool kFused>
-__global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
+using PlanOf = PrefillPlan<D, D == 64 && !kFused>;
+
+template <int D, bool kFused>
+__global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>::kMinBlocks)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_q,
                    const __grid_constant__ CUtensorMap tmap_kv,
                    const __grid_constant__ PrefillParams p)
 {
-    using PL = PrefillPlan<D>;
+    using PL = PlanOf<D, kFused>;
+    // Query tile g's shared-memory slot and tensor-memory columns (the only tile of a one-tile CTA
+    // is tile B, in slot 0).
+    auto slot_of = [](int g) { return PL::kTiles == 1 ? 0 : g; };
     constexpr int R = PL::kRingTiles;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -132,8 +157,9 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
     const int head_a = p.head_pairs ? 2 * sel : sel;
     const int head_b = p.head_pairs ? 2 * sel + 1 : sel;
     const int n_b = qb_b + 1;                                   // key tiles 0 .. qb_b
-    const int n_a = kFused ? (p.fused_L > p.fused_L1 ? n_b : 0)
-                           : (p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0));   // 0: no tile A
+    const int n_a = PL::kTiles == 1 ? 0
+                    : kFused ? (p.fused_L > p.fused_L1 ? n_b : 0)
+                             : (p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0));   // 0: no tile A
     const int j = kFused ? sel : head_b / p.G;                  // Eq. 15
     const int zk = ((p.slot * 2 + 0) * p.b + beta) * p.g + j;
     const int zv = zk + p.b * p.g;
@@ -166,7 +192,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    if (kFused && warp < 8) {
+    if (kFused && warp < PL::kSoftWarps) {
         // The tiles' rows past the TMA box (box_rows = G x min(L1, L)) are never loaded; zero them
         // so that their (discarded) scores stay finite.  TMA writes only rows below box_rows.
         const int grp = warp >> 2, r = threadIdx.x & 127;
@@ -211,8 +237,8 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                     if (n_a > 0)
                         tma_load_4d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64,
                                     head_a, (n_a - 1) * 128, beta);
-                    tma_load_4d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
-                                sub * 64, head_b, qb_b * 128, beta);
+                    tma_load_4d(sbase + PL::kQ + slot_of(1) * PL::kTileBytes + sub * 16384, &tmap_q,
+                                bar_q, sub * 64, head_b, qb_b * 128, beta);
                 }
             }
             const int n_idx = 2 * n_b;   // K_0, V_0, K_1, V_1, ...
@@ -284,21 +310,24 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 return ok;
             };
             auto issue_s = [&](int g, int t) {
-                const uint64_t qa = dq + g * kSlot;
+                const uint64_t qa = dq + slot_of(g) * kSlot;
                 const uint64_t kb = dk + ((2 * t) % R) * kSlot;
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
                     const uint32_t off = (k >> 2) * 1024 + (k & 3) * 2;   // 16384 B, 32 B
-                    umma_f16(tmem + PL::kColS + 128 * g, qa + off, kb + off, kIdS, k > 0 ? 1 : 0);
+                    umma_f16(tmem + PL::kColS + 128 * slot_of(g), qa + off, kb + off, kIdS,
+                             k > 0 ? 1 : 0);
                 }
                 umma_commit(bar_s_ready + 8 * g);
             };
             auto issue_pv = [&](int g, int t, bool last) {
                 const uint64_t vb = dv + ((2 * t + 1) % R) * kSlot;
-                const uint32_t pc = tmem + (PL::kPSep ? PL::kColP + 64 * g : PL::kColS + 128 * g);
+                const int sg = slot_of(g);
+                const uint32_t pc =
+                    tmem + (PL::kPSep ? PL::kColP + 64 * sg : PL::kColS + 128 * sg);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)   // 16 keys = 2048 B of V, 8 TMEM columns of P
-                    umma_f16_ts(tmem + PL::kColO + D * g, pc + 8 * k, vb + k * 128, kIdPV,
+                    umma_f16_ts(tmem + PL::kColO + D * sg, pc + 8 * k, vb + k * 128, kIdPV,
                                 (t > 0 || k > 0) ? 1 : 0);
                 // With P over S, the next S's completion already implies this product's.
                 if (PL::kPSep || last)
@@ -365,19 +394,20 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
                 atomicOr(p.err, kErrDrain);
         }
         __syncwarp();
-    } else if (warp < 8) {
+    } else if (warp < PL::kSoftWarps) {
         // ------------------------------------ softmax warpgroups --------------------------------
         setmaxnreg_inc<PL::kRegsHigh>();
-        const int grp = warp >> 2;                  // 0: query tile A, 1: query tile B
+        const int grp = PL::kTiles == 1 ? 1 : warp >> 2;   // 0: query tile A, 1: query tile B
         const int r = threadIdx.x & 127;            // query row of the tile = TMEM lane
         const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
         const int n_g = grp ? n_b : n_a;
         const int head = grp ? head_b : head_a;
         const int q0 = (kt0 + n_g - 1) * 128;       // first position of the unit's last tile
-        const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * grp;
-        const uint32_t col_o = tmem + lane_off + PL::kColO + D * grp;
+        const int sg = slot_of(grp);
+        const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * sg;
+        const uint32_t col_o = tmem + lane_off + PL::kColO + D * sg;
         const uint32_t col_p =
-            tmem + lane_off + (PL::kPSep ? PL::kColP + 64 * grp : PL::kColS + 128 * grp);
+            tmem + lane_off + (PL::kPSep ? PL::kColP + 64 * sg : PL::kColS + 128 * sg);
         const uint32_t s_ready = bar_s_ready + 8 * grp, s_free = bar_s_free + 8 * grp;
         const uint32_t p_ready = bar_p_ready + 8 * grp, pv_done = bar_pv_done + 8 * grp;
         // The prompt's last block holds keys past its end; the first tile to reach it zeroes them.
@@ -396,7 +426,7 @@ __global__ void __launch_bounds__(PrefillPlan<D>::kThreads, 1)
             wait(s_ready, t);
             // Tile B's first warp frees ring slots whose readers have all completed: K_0 once S_B(0)
             // is done; V_{t-1} and K_t once S_B(t) (P over S) or P_B V_{t-1} (own P) is done.
-            const bool releaser = grp == 1 && warp == 4 && lane == 0;
+            const bool releaser = grp == 1 && (warp & 3) == 0 && lane == 0;
             if (releaser && t == 0)
                 mbar_arrive(bar_empty);
             if (releaser && t > 0 && !PL::kPSep) {
@@ -627,6 +657,27 @@ const void *prefill_fn()
     return reinterpret_cast<const void *>(&prefill_kernel<D, kFused>);
 }
 
+template <typename F>
+auto plan_value(int head_dim, bool fused, F f)
+{
+    if (fused)
+        return head_dim == 64 ? f(PlanOf<64, true>{}) : f(PlanOf<128, true>{});
+    return head_dim == 64 ? f(PlanOf<64, false>{}) : f(PlanOf<128, false>{});
+}
+int threads_of(int head_dim, bool fused)
+{
+    return plan_value(head_dim, fused, [](auto pl) { return decltype(pl)::kThreads; });
+}
+int regs_of(int head_dim, bool fused)
+{
+    return plan_value(head_dim, fused, [](auto pl) { return decltype(pl)::kRegsLaunch; });
+}
+size_t smem_of(int head_dim, bool fused)
+{
+    return plan_value(head_dim, fused,
+                      [](auto pl) { return static_cast<size_t>(decltype(pl)::kAlloc); });
+}
+
 const void *kernel_fn(int head_dim, bool fused)
 {
     if (fused)
@@ -639,9 +690,8 @@ cudaError_t launch(int head_dim, bool fused, const CUtensorMap *tmap_q, const CU
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
-    cfg.blockDim = dim3(static_cast<unsigned>(head_dim == 64 ? PrefillPlan<64>::kThreads
-                                                             : PrefillPlan<128>::kThreads));
-    cfg.dynamicSmemBytes = head_dim == 64 ? PrefillPlan<64>::kAlloc : PrefillPlan<128>::kAlloc;
+    cfg.blockDim = dim3(static_cast<unsigned>(threads_of(head_dim, fused)));
+    cfg.dynamicSmemBytes = smem_of(head_dim, fused);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -655,10 +705,7 @@ cudaError_t launch(int head_dim, bool fused, const CUtensorMap *tmap_q, const CU
 
 }  // namespace
 
-size_t prefill_smem_bytes(int head_dim)
-{
-    return head_dim == 64 ? PrefillPlan<64>::kAlloc : PrefillPlan<128>::kAlloc;
-}
+size_t prefill_smem_bytes(int head_dim) { return smem_of(head_dim, false); }
 
 // The warpgroups' register split (setmaxnreg) adds up to the registers the block is launched with;
 // a kernel built with another per-thread count would wait forever in setmaxnreg.inc, so it is
@@ -669,12 +716,11 @@ cudaError_t prepare(int head_dim, bool fused)
     cudaError_t e = cudaFuncGetAttributes(&fa, kernel_fn(head_dim, fused));
     if (e != cudaSuccess)
         return e;
-    const int want = head_dim == 64 ? PrefillPlan<64>::kRegsLaunch : PrefillPlan<128>::kRegsLaunch;
-    if (fa.numRegs != want)
+    if (fa.numRegs != regs_of(head_dim, fused))
         return cudaErrorInvalidKernelImage;
     return cudaFuncSetAttribute(kernel_fn(head_dim, fused),
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(prefill_smem_bytes(head_dim)));
+                                static_cast<int>(smem_of(head_dim, fused)));
 }
 
 cudaError_t prepare_prefill(int head_dim) { return prepare(head_dim, false); }
