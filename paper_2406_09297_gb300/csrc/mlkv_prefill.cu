@@ -433,81 +433,112 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                 mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
                 mbar_arrive(bar_empty + 8 * ((2 * t) % R));
             }
-            tmem_fence_after();
+            const bool diag = t == n_g - 1 && has_end;
+            // This tile's scores, with the causal (or sequence-end) mask of the last tile.
             float sv[4][32];
+            auto load_scores = [&]() {
+                tmem_fence_after();
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                tmem_ld32_nowait(col_s + c * 32, sv[c]);
-            tmem_wait_ld();
+                for (int c = 0; c < 4; ++c)
+                    tmem_ld32_nowait(col_s + c * 32, sv[c]);
+                tmem_wait_ld();
+                if (diag) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+#pragma unroll
+                        for (int k = 0; k < 32; ++k)
+                            if (kFused ? q0 + c * 32 + k >= S   // past the sequence
+                                       : c * 32 + k > r)        // a later position: causal mask
+                                sv[c][k] = NEG_INF;
+                }
+            };
+            // Raises the reference maximum to the tile's when a score exceeds it by more than 2^8
+            // (the thread then rescales its O row in TMEM).
+            auto raise_to_tile_max = [&]() {
+                float mx[4];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    float a = max3f(sv[c][0], sv[c][1], sv[c][2]);
+                    float b = max3f(sv[c][3], sv[c][4], sv[c][5]);
+#pragma unroll
+                    for (int k = 6; k < 30; k += 4) {
+                        a = max3f(a, sv[c][k], sv[c][k + 1]);
+                        b = max3f(b, sv[c][k + 2], sv[c][k + 3]);
+                    }
+                    mx[c] = max3f(a, b, fmaxf(sv[c][30], sv[c][31]));
+                }
+                const float m_tile = max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * scale;
+                const bool raise = (m_run == NEG_INF) || (m_tile > m_run + 8.f);
+                if (__any_sync(0xffffffffu, raise)) {
+                    const float m_new = raise ? fmaxf(m_run, m_tile) : m_run;
+                    const float alpha = fast_exp2(m_run - m_new);   // 0 while nothing is summed
+                    if (t > 0) {
+                        // Rescale this row of O once the previous tile's product has landed.
+                        if (PL::kPSep)
+                            wait(pv_done, t - 1);
+                        tmem_fence_after();
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            float ov[32];
+                            tmem_ld32_nowait(col_o + c * 32, ov);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int k = 0; k < 32; ++k)
+                                ov[k] *= alpha;
+                            tmem_st32(col_o + c * 32, ov);
+                        }
+                    }
+                    l_run *= alpha;
+                    m_run = m_new;
+                }
+            };
+            const float2 sc2 = make_float2(scale, scale);
+            float2 acc[4];
+            uint32_t w[2][32];
+            // p = 2^(s log2(e)/sqrt(d) - m) as bf16 pairs, and the row's sum in fp32.
+            auto weights = [&]() {
+                const float m_use = m_run == NEG_INF ? 0.f : m_run;   // all masked so far: p = 0
+                const float2 nm2 = make_float2(-m_use, -m_use);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    acc[q] = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int c = half * 64 + 2 * i;   // keys c, c + 1
+                        const float2 x = __ffma2_rn(
+                            make_float2(sv[c >> 5][c & 31], sv[c >> 5][(c & 31) + 1]), sc2, nm2);
+                        const float2 pr = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+                        acc[i & 3] = __fadd2_rn(acc[i & 3], pr);
+                        w[half][i] = pack_bf16x2(pr.x, pr.y);
+                    }
+                }
+            };
+            load_scores();
+            if (__any_sync(0xffffffffu, m_run == NEG_INF)) {
+                raise_to_tile_max();
+                weights();
+            } else {
+                // Most tiles: the weights against the current reference, without the tile's
+                // maximum.  A row whose weights add up to more than 2^8 (or overflow) may hold one
+                // above 2^8: the scores are read again (S is still in TMEM: its columns are freed
+                // only below) and the reference raised as above.
+                weights();
+                const float2 s01 = __fadd2_rn(acc[0], acc[1]), s23 = __fadd2_rn(acc[2], acc[3]);
+                const float2 s4 = __fadd2_rn(s01, s23);
+                if (__any_sync(0xffffffffu, !(s4.x + s4.y <= 256.f))) {
+                    load_scores();
+                    raise_to_tile_max();
+                    weights();
+                }
+            }
             if (PL::kPSep) {
+                // S's columns may now take the next tile's scores.
                 tmem_fence_before();
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(s_free);
-            }
-            const bool diag = t == n_g - 1 && has_end;
-            if (diag) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int k = 0; k < 32; ++k)
-                        if (kFused ? q0 + c * 32 + k >= S   // past the sequence
-                                   : c * 32 + k > r)        // a later position: causal mask
-                            sv[c][k] = NEG_INF;
-            }
-            float mx[4];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float a = max3f(sv[c][0], sv[c][1], sv[c][2]);
-                float b = max3f(sv[c][3], sv[c][4], sv[c][5]);
-#pragma unroll
-                for (int k = 6; k < 30; k += 4) {
-                    a = max3f(a, sv[c][k], sv[c][k + 1]);
-                    b = max3f(b, sv[c][k + 2], sv[c][k + 3]);
-                }
-                mx[c] = max3f(a, b, fmaxf(sv[c][30], sv[c][31]));
-            }
-            const float m_tile = max3f(mx[0], mx[1], fmaxf(mx[2], mx[3])) * scale;
-            const bool raise = (m_run == NEG_INF) || (m_tile > m_run + 8.f);
-            if (__any_sync(0xffffffffu, raise)) {
-                const float m_new = raise ? fmaxf(m_run, m_tile) : m_run;
-                const float alpha = fast_exp2(m_run - m_new);   // 0 while nothing is summed
-                if (t > 0) {
-                    // Rescale this row of O once the previous tile's product has landed.
-                    if (PL::kPSep)
-                        wait(pv_done, t - 1);
-                    tmem_fence_after();
-#pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        float ov[32];
-                        tmem_ld32_nowait(col_o + c * 32, ov);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int k = 0; k < 32; ++k)
-                            ov[k] *= alpha;
-                        tmem_st32(col_o + c * 32, ov);
-                    }
-                }
-                l_run *= alpha;
-                m_run = m_new;
-            }
-            const float2 sc2 = make_float2(scale, scale);
-            const float2 nm2 = make_float2(-m_run, -m_run);
-            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                             make_float2(0.f, 0.f)};
-            uint32_t w[2][32];
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int c = half * 64 + 2 * i;   // keys c, c + 1
-                    const float2 x =
-                        __ffma2_rn(make_float2(sv[c >> 5][c & 31], sv[c >> 5][(c & 31) + 1]), sc2,
-                                   nm2);
-                    const float2 pr = make_float2(fast_exp2(x.x), fast_exp2(x.y));
-                    acc[i & 3] = __fadd2_rn(acc[i & 3], pr);
-                    w[half][i] = pack_bf16x2(pr.x, pr.y);
-                }
             }
             // The P buffer of the previous tile must have been read by its P V; the weights above
             // were computed while that product ran.
