@@ -135,12 +135,15 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
  * owner's block reads that owner's new token from K and V (the later layers take their newest
  * row from there rather than from the cache), so K and V, like Q, must stay valid until the stream
  * has run the whole step.
- * With option "step_graph" = 1 (default) a call whose pointers, lengths and options equal those of
- * the previous call replays a CUDA graph of the step's launches (recorded on the second such call;
- * new values in the same buffers are fine); a call with arguments different from the previous
- * call's issues the launches directly, which costs the host about half of recording them -- the
- * case of a decode loop, whose lengths grow every step.  When cuda_stream is itself being captured
- * the launches are issued directly, into the caller's graph.
+ * Option "step_graph": with 1 a call whose pointers, lengths and options equal those of the
+ * previous call replays a CUDA graph of the step's launches (recorded on the second such call; new
+ * values in the same buffers are fine); a call with arguments different from the previous call's
+ * issues the launches directly, which costs the host about half of recording them -- the case of a
+ * decode loop, whose lengths grow every step.  With 2 (default) a step that runs as one
+ * multi-layer launch (and its merge launch) is always issued directly -- a replayed one-node graph
+ * measured ~2 us slower per step -- and a step of per-layer launches is recorded and replayed as
+ * with 1.  0 issues every step directly.  When cuda_stream is itself being captured the launches
+ * are issued directly, into the caller's graph.
  */
 int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
                      const int *seq_lens, void *cuda_stream);
@@ -152,7 +155,8 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
  * cudaMemcpyAsync per tensor.  Layouts as for mlkv_decode_step, in host memory.
  * With page-locked buffers (cudaHostAlloc, cudaHostRegister) and option "step_graph" = 1 the copies
  * and the launches of a step are recorded into one CUDA graph the second time the same arguments
- * come and replayed after (as for mlkv_decode_step); pageable buffers run directly, and their
+ * come and replayed after (as for mlkv_decode_step; with 2, the default, a one-launch step and
+ * its input copy are issued directly); pageable buffers run directly, and their
  * copies synchronise with the host as CUDA's pageable copies do.  out holds the step's outputs
  * once the stream has reached the end of the call's work.  The staging buffers, 2 * (l*b*h*d +
  * m*b*g*d) bf16, are allocated on the first call and kept until mlkv_cache_destroy.
@@ -246,7 +250,9 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *   "pdl"          1 (default) = programmatic dependent launch: a decode launch's set-up overlaps
  *                  the previous kernel of the stream (it touches no global memory before that
  *                  kernel has completed); 0 = plain stream order
- *   "step_graph"   1 (default) = mlkv_decode_step replays a recorded CUDA graph (see there)
+ *   "step_graph"   2 (default) = mlkv_decode_step issues a one-launch step directly and replays a
+ *                  recorded CUDA graph of a per-layer step; 1 = always the graph; 0 = never (see
+ *                  mlkv_decode_step)
  *   "tc"           0 (default) = the decode kernel on mma.sync tensor-core instructions; 1 = the
  *                  tcgen05 kernel (tensor-memory accumulators) for 128- and 256-position tiles,
  *                  the mma.sync kernel otherwise.  Same results within the tolerance; the tcgen05

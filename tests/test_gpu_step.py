@@ -49,6 +49,7 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
         _inputs(owner, h, g, d, b, lens, max_seq, seed, cache2, None)
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.full((l, b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cache.set_option("step_graph", 1)   # always through the recorded graph
         for rep in range(4):   # direct, record, then replay twice
             out.fill_(float("nan"))
             cache.decode_step(Q, K, V, out, lens)
@@ -204,14 +205,17 @@ def test_step_host_buffers_match_device_step():
             out = torch.full((w.l, w.b, w.h, w.d), float("nan"), dtype=torch.bfloat16)
             if pinned:
                 hq, hk, hv, out = hq.pin_memory(), hk.pin_memory(), hv.pin_memory(), out.pin_memory()
-            before = cache.get_option("step_graph_replays")
-            for _ in range(4):
-                out.fill_(float("nan"))
-                cache.decode_step_host(hq, hk, hv, out, seq_lens)
-                torch.cuda.synchronize()
-                assert torch.equal(out.view(torch.int16), want.view(torch.int16))
-            replays = cache.get_option("step_graph_replays") - before
-            assert replays == (3 if pinned else 0), (pinned, replays)
+            for graph in (1, 2):   # always recorded; the default (direct for one launch)
+                cache.set_option("step_graph", graph)
+                before = cache.get_option("step_graph_replays")
+                for _ in range(4):
+                    out.fill_(float("nan"))
+                    cache.decode_step_host(hq, hk, hv, out, seq_lens)
+                    torch.cuda.synchronize()
+                    assert torch.equal(out.view(torch.int16), want.view(torch.int16))
+                replays = cache.get_option("step_graph_replays") - before
+                direct = graph == 2 and cache.get_option("last_step_kernel") == 1
+                assert replays == (3 if pinned and not direct else 0), (pinned, graph, replays)
         cache.sync_status()
 
 
@@ -304,6 +308,7 @@ def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
         qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 81, cache, ref)
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        cache.set_option("step_graph", 1)   # always through the recorded graph
         results = []
         for rep in range(3):   # direct, record, replay
             out.fill_(float("nan"))

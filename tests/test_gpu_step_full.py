@@ -10,8 +10,9 @@ that call on every workload of the benchmark suite at full batch and context:
   * the cache holds the generator's K/V at every position; the step's new tokens come from
     another seed, so the newest row (position L-1) of every owner's slot changes in the step and
     a layer that read it from the cache before its owner stored it would be caught;
-  * the first call is issued directly, the second records the graph, the third replays it; the
-    outputs of the first and of the replay are both checked;
+  * the first call is issued directly, the second records the graph, the third replays it (with
+    the default step_graph 2 a step that runs as one multi-layer launch is issued directly every
+    time); the outputs of the first and of the third call are both checked;
   * for sampled (sequence, KV head) pairs -- the first and last sequence and seeded random ones
     -- the oracle recomputes that KV head's query group in every layer (Eqs. 2-3 with the maps of
     Eqs. 15 and 18) from the generator's values rebuilt on the host, and every sampled output must
@@ -99,13 +100,16 @@ def check_step_full_size(w, n_betas=4, seed=0, options=None, host_buffers=False)
                     checked.append(out.float().numpy().copy())
         else:
             out = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
-            for rep in range(3):   # direct, record, replay
+            for rep in range(3):   # direct, record, replay (or three direct launches)
                 out.fill_(float("nan"))
                 cache.decode_step(Q, K, V, out, seq_lens)
                 torch.cuda.synchronize()
                 if rep != 1:
                     checked.append(out.float().cpu().numpy())
-            assert cache.get_option("step_graph_replays") == 2
+            # step_graph 2 (default) issues one multi-layer launch directly, else it replays
+            direct = (cache.get_option("step_graph") == 2 and
+                      cache.get_option("last_step_kernel") == 1)
+            assert cache.get_option("step_graph_replays") == (0 if direct else 2)
         cache.sync_status()
         worst = 0.0
         for own in w.owners():
@@ -147,12 +151,13 @@ def test_step_host_buffers_config2_full_size():
     check_step_full_size(workloads.config(2), seed=12, host_buffers=True)
 
 
-@pytest.mark.parametrize("options", [{"l2_prefetch": 0}, {"l2_persist": 1}, {"step_kernel": 0}])
+@pytest.mark.parametrize("options", [{"l2_prefetch": 0}, {"l2_persist": 1}, {"step_kernel": 0},
+                                     {"step_graph": 1}])
 def test_step_options_full_size(options):
     """Options that change where bytes come from or how the step is launched, never the result:
     the default workload and the varied-length GQA workload (slots larger than L2) with the L2
-    prefetch off, with L2 persistence on, and with per-layer launches instead of one multi-layer
-    launch."""
+    prefetch off, with L2 persistence on, with per-layer launches instead of one multi-layer
+    launch, and with the multi-layer launch replayed from a recorded graph."""
     import paper_2406_09297_gb300 as mlkv
     for index in (2, 3):
         try:
