@@ -808,22 +808,68 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     };
     Plan pl = plan_for(var, 1);
     if (uniform && pl.heaviest > pl.per_layer) {
-        // Few long segments (batch 1 at long context): split every segment into C chunks of the
-        // 128-position tile (two CTAs per SM), each a partial record, merged by one combine
-        // launch for the whole step -- about 2.5 waves of items, chunks of >= 8 tiles.
-        mlkv_cache::Variant *v128 = pick_variant(c, -1.0, 128);
-        if (v128 != nullptr && !v128->v->tc) {
-            const long long slots = static_cast<long long>(v128->ctas_per_sm) * c->sm_count;
-            const long long nt = (seq_lens[0] + 127) / 128;
-            long long C = (5 * slots + 2 * S * c->l - 1) / (2 * S * c->l);
-            C = std::min<long long>({C, nt / 8, mlkv::kCombineMaxPiecesHost,
-                                     static_cast<long long>(c->records) / (S * c->l)});
-            if (C > 1) {
-                Plan pc = plan_for(v128, static_cast<int>(C));
-                if (pc.heaviest <= pc.per_layer)
-                    pl = pc;
+        // Few long segments (batch 1 at long context): split every segment into C chunks, each a
+        // partial record, merged by one combine launch for the whole step.  C: chunks of >= 8
+        // tiles, 2 to 4 waves of items, rounded so that the items fill whole waves of resident
+        // CTAs where that is possible; per tile size the plan with the lightest heaviest CTA (its
+        // tiles, plus one tile's worth for each partial record it writes) is taken.  Between the
+        // 256-position tile (one CTA per SM, three stages) and the 128-position one (two CTAs per
+        // SM) the 256 one is taken unless it gives a CTA more than one item beyond the 128 one's
+        // (measured at batch 1, 131072 positions: MLKV-2 59.4 -> 52.9 us, MLKV-6 71.6 -> 62.8,
+        // MQA 93.4 -> 89.4; GQA-4, 9 items a CTA against 5: 250 -> 260, so 128 there).  A forced
+        // tile size (option "tile") is used as it is.
+        struct Chunked {
+            bool ok = false;
+            Plan plan{};
+            long long per = 0;
+        };
+        auto best_chunks = [&](int T_chunk) {
+            Chunked best;
+            mlkv_cache::Variant *vch = pick_variant(c, -1.0, T_chunk);
+            if (vch == nullptr || vch->v->tc)
+                return best;
+            const long long slots = static_cast<long long>(vch->ctas_per_sm) * c->sm_count;
+            const long long nt = (seq_lens[0] + T_chunk - 1) / T_chunk;
+            const long long sl = S * c->l;
+            long long a = slots, bq = sl;   // gcd: C a multiple of slots / gcd fills whole waves
+            while (bq != 0) {
+                const long long r = a % bq;
+                a = bq;
+                bq = r;
             }
+            const long long unit = slots / a;
+            const long long c_max = std::min<long long>(
+                {nt / 8, mlkv::kCombineMaxPiecesHost, static_cast<long long>(c->records) / sl});
+            long long best_cost = -1;
+            for (int waves = 2; waves <= 4; ++waves) {
+                long long C = (waves * slots + sl - 1) / sl;
+                const long long Cr = (C + unit - 1) / unit * unit;
+                C = Cr <= c_max ? Cr : std::min(C, c_max);
+                if (C <= 1)
+                    continue;
+                Plan pc = plan_for(vch, static_cast<int>(C));
+                if (pc.heaviest > pc.per_layer)
+                    continue;
+                const long long per = (pc.items + pc.grid - 1) / pc.grid;
+                const long long cost = pc.heaviest + per;
+                if (best_cost < 0 || cost < best_cost) {
+                    best_cost = cost;
+                    best.ok = true;
+                    best.plan = pc;
+                    best.per = per;
+                }
+            }
+            return best;
+        };
+        Chunked pick;
+        if (c->tile_tokens > 0) {
+            pick = best_chunks(c->tile_tokens);
+        } else {
+            const Chunked c256 = best_chunks(256), c128 = best_chunks(128);
+            pick = (c256.ok && (!c128.ok || c256.per <= c128.per + 1)) ? c256 : c128;
         }
+        if (pick.ok)
+            pl = pick.plan;
     }
     if (pl.heaviest > pl.per_layer || pl.items > 0x7fffffffLL ||
         pl.items * pl.heaviest > 0x7fffffffLL)

@@ -222,7 +222,7 @@ def test_step_host_buffers_match_device_step():
 @pytest.mark.parametrize("step_kernel", [1, 0])
 def test_step_single_long_segment(step_kernel):
     # Batch 1, one KV head, 16384 positions.  One multi-layer launch splits every layer's
-    # segment into 16 chunks of 8 tiles of 128 positions (48 CTAs), each a partial record, and
+    # segment into 8 chunks of 8 tiles of 256 positions (24 CTAs), each a partial record, and
     # one combine launch merges them; per-layer launches (step_kernel 0) run the later layers'
     # 128-position tile over 64 CTAs with a merge launch per layer.
     import torch
@@ -238,9 +238,9 @@ def test_step_single_long_segment(step_kernel):
         cache.decode_step(to_dev(qb), to_dev(kn), to_dev(vn), out, lens)
         torch.cuda.synchronize()
         assert cache.get_option("last_step_kernel") == step_kernel
-        assert cache.get_option("last_tile_tokens") == 128
+        assert cache.get_option("last_tile_tokens") == (256 if step_kernel else 128)
         assert cache.get_option("last_deferred_merge") == 1
-        assert cache.get_option("last_grid") == (48 if step_kernel else 64)
+        assert cache.get_option("last_grid") == (24 if step_kernel else 64)
         ref.append(0, gen.bf16_bits_to_f64(kn[0]), gen.bf16_bits_to_f64(vn[0]), lens)
         for n in range(len(owner)):
             expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens)
@@ -289,9 +289,9 @@ def test_step_whole_segments_per_cta(b, g, L, grid, tile):
     ([0, 0, 0], 16, 2, 64, 100, 77, 300),              # one partly visible tile per item
     ([0] * 6, 12, 1, 64, 8, 2001, 48),                 # batch 8: one 256-position-tile item a CTA
     # few long segments: every segment in chunks, partial records, one merge launch
-    ([0] * 6 + [6] * 6, 12, 1, 64, 1, 131072, 256),    # 64 chunks of 16 tiles a segment
-    ([0, 0, 2, 2], 12, 4, 64, 2, 9000, 256),           # ragged last tile in the last chunk
-    ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 128),         # head_dim 128
+    ([0] * 6 + [6] * 6, 12, 1, 64, 1, 131072, 152),    # 38 chunks of 13-14 256-tiles: 3 waves
+    ([0, 0, 2, 2], 12, 4, 64, 2, 9000, 128),           # ragged last tile in the last chunk
+    ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 152),         # head_dim 128: 19 chunks, 4 waves of 152
 ])
 def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
     # One launch for the whole step: CTA c takes the (layer, segment) items c, c + P, ..., each a
