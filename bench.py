@@ -340,31 +340,37 @@ def run(args, w):
 
     # ---- the same step as a model runs it: one layer after another -----------------------------
     # A model computes layer n's queries from layer n-1's output, so its attention for layer n
-    # starts only after layer n-1's has ended.  The step above is given every layer's queries at
-    # once (the step call), which lets one launch cover every layer; here the same call runs as
-    # one launch per layer in plain stream order (options step_kernel 0, pdl 0: no layer's grid
-    # starts before the previous one has finished), L2 flushed before each step as above.
-    saved = {k: int(cache.get_option(k)) for k in ("step_kernel", "pdl")}
-    cache.set_option("step_kernel", 0)
-    cache.set_option("pdl", 0)
-    for _ in range(args.warmup):
-        flush.zero_()
-        step()
-    sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
-    barrier()
-    for k in range(args.steps):
-        flush.zero_()
-        sev[k][0].record()
-        step()
-        sev[k][1].record()
-    barrier()
-    seq_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in sev) / args.steps, dist, "cuda")
-    seq_launches = w.l * (2 if cache.get_option("last_deferred_merge") else 1)
-    for key, val in saved.items():
-        cache.set_option(key, val)
-    step()   # back to the measured configuration
+    # reads nothing before layer n-1's has ended.  The step above is given every layer's queries
+    # at once (the step call), which lets one launch cover every layer.  Here the same call runs
+    # as one launch per layer (step_kernel 0) with no layer reading anything before the previous
+    # one has finished: in plain stream order (pdl 0), and with each grid's launch and set-up
+    # overlapping the previous one's end but every read after it (pdl 1, early_fetch 0).  L2 is
+    # flushed before each step as above.
+    def time_with(options):
+        saved = {k: int(cache.get_option(k)) for k in options}
+        for key, val in options.items():
+            cache.set_option(key, val)
+        for _ in range(args.warmup):
+            flush.zero_()
+            step()
+        sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        barrier()
+        for k in range(args.steps):
+            flush.zero_()
+            sev[k][0].record()
+            step()
+            sev[k][1].record()
+        barrier()
+        t = max_over_ranks(sum(a.elapsed_time(b) for a, b in sev) / args.steps, dist, "cuda")
+        n_launch = w.l * (2 if cache.get_option("last_deferred_merge") else 1)
+        for key, val in saved.items():
+            cache.set_option(key, val)
+        return t, n_launch
 
+    seq_ms, seq_launches = time_with({"step_kernel": 0, "pdl": 0})
+    seqp_ms, _ = time_with({"step_kernel": 0, "pdl": 1, "early_fetch": 0})
+    step()   # back to the measured configuration
     # ---- decode kernel durations ---------------------------------------------------------------
     # The graph-timed step is nothing but the l decode launches back to back, so its device time
     # divided by l is the mean launch duration inside the step.  Eager launches bracketed by events
@@ -456,9 +462,13 @@ def run(args, w):
             "sequential_layers": {
                 "value": job_value(w.b, world, seq_ms), "unit": UNIT, "ms_per_step": seq_ms,
                 "launches_per_step": seq_launches,
-                "how": "the same step as one launch per layer in plain stream order (options "
-                       "step_kernel 0, pdl 0): no layer starts before the previous one ends, as "
-                       "in a model whose layer n queries come from layer n-1"},
+                "overlapped_launch": {"value": job_value(w.b, world, seqp_ms),
+                                      "ms_per_step": seqp_ms},
+                "how": "the same step as one launch per layer, no layer reading anything before "
+                       "the previous one has finished, as in a model whose layer n queries come "
+                       "from layer n-1: plain stream order (options step_kernel 0, pdl 0); "
+                       "overlapped_launch: each grid's launch and set-up overlap the previous "
+                       "one's end (step_kernel 0, pdl 1, early_fetch 0)"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind,

@@ -122,6 +122,7 @@ struct mlkv_cache {
     int last_seg_major = 0;     // 1 if that launch ranked its items segment-major
     int cluster = 1;            // allow the DSMEM cluster merge
     int pdl = 1;                // programmatic dependent launch
+    int early_fetch = 1;        // per-layer step: later layers read Q and tiles before the wait
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
     int fused_ready = 0;        // the same for the fused-decode instance
@@ -137,11 +138,13 @@ struct mlkv_cache {
         std::vector<int> lens;
         int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1, tc = -1, pf = -1, sk = -1;
         int sg = -1;   // step_graph: a graph recorded under one mode is not replayed under another
+        int ef = -1;
         bool operator==(const StepKey &o) const
         {
             return Q == o.Q && K == o.K && V == o.V && out == o.out && lens == o.lens &&
                    tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
-                   l2 == o.l2 && tc == o.tc && pf == o.pf && sk == o.sk && sg == o.sg;
+                   l2 == o.l2 && tc == o.tc && pf == o.pf && sk == o.sk && sg == o.sg &&
+                   ef == o.ef;
         }
     } step_key, pending_key;   // recorded arguments; arguments seen once, not yet recorded
     int step_graph_replays = 0;
@@ -993,7 +996,7 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         if (e != cudaSuccess)
             return fail_cuda(e, "step event");
         // Layers after the first follow this library's own launch of the preceding layer.
-        const int early = (n > 0 && c->pdl) ? 1 : 0;
+        const int early = (n > 0 && c->pdl && c->early_fetch) ? 1 : 0;
         const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
         // A segment's newest row is the step's new token of the owner: the owner layer appends
         // it itself (fused); a later layer of the block replaces that row of its tiles from the
@@ -1039,6 +1042,7 @@ mlkv_cache::StepKey step_key_of(const mlkv_cache *c, const void *Q, const void *
     key.pf = c->l2_prefetch;
     key.sk = c->step_kernel;
     key.sg = c->step_graph;
+    key.ef = c->early_fetch;
     return key;
 }
 
@@ -1776,6 +1780,12 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->pdl = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "early_fetch") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "early_fetch must be 0 or 1");
+        c->early_fetch = static_cast<int>(value);
+        return MLKV_OK;
+    }
     if (std::strcmp(key, "step_graph") == 0) {
         if (value < 0 || value > 2)
             return fail(MLKV_ERR_INVALID_ARG, "step_graph must be 0, 1 or 2");
@@ -1841,6 +1851,10 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "pdl") == 0) {
         *value = c->pdl;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "early_fetch") == 0) {
+        *value = c->early_fetch;
         return MLKV_OK;
     }
     if (std::strcmp(key, "step_graph") == 0) {
