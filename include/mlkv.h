@@ -375,6 +375,9 @@ int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void
  *   W_merged     device bf16 [m][n_kv_heads][row_elems], m = owner layers, in increasing layer
  *                order (the slot order of mlkv_owner_slot); 16-byte aligned; must not overlap W
  *   cuda_stream  the stream the kernel is queued on (asynchronous; nothing is allocated)
+ * A model's K and V projections can go through one call: stacked as 2 * n_layers layers (K's, then
+ * V's) with layer_owner[n + n_layers] = layer_owner[n] + n_layers, the merged heads come out K's
+ * then V's, each equal to a call of its own (no merged head mixes layers of different owners).
  * Errors: MLKV_ERR_INVALID_ARG (null or unaligned pointers, sizes, overlap), MLKV_ERR_MAP (owner
  * map, g not dividing h), MLKV_ERR_UNSUPPORTED (more than 1024 layers or 65535 merged heads),
  * MLKV_ERR_CUDA.

@@ -145,3 +145,19 @@ def test_rejects_bad_arguments():
     with pytest.raises(mlkv.MLKVError) as e:                   # 12 elements: not a multiple of 8
         mlkv.mlkv_merge_kv_weights([0, 0], 4, 2, Wodd, out)
     assert e.value.code == mlkv.MLKV_ERR_INVALID_ARG
+
+
+def test_k_and_v_in_one_call():
+    """K and V of a model merged by one call, stacked as 2 l layers with V's layers owned by
+    owner + l (the benchmark's form): the output is K's merged heads then V's, bit for bit those
+    of one call per projection, and both agree with the oracle."""
+    owner, h, g, row = [0] * 6 + [6] * 6, 12, 1, 64 * 768
+    l = len(owner)
+    Wk = _weights(31, l, h, row)
+    Wv = _weights(32, l, h, row)
+    both = _merge(owner + [o + l for o in owner], h, g, np.concatenate([Wk, Wv]))
+    m = len(set(owner))
+    assert np.array_equal(both[:m], _merge(owner, h, g, Wk))
+    assert np.array_equal(both[m:], _merge(owner, h, g, Wv))
+    _check(owner, h, g, Wk, both[:m])
+    _check(owner, h, g, Wv, both[m:])
