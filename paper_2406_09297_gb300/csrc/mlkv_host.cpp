@@ -588,23 +588,28 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                 grid = static_cast<int>(S);
             }
             if (c->cluster) {
-                // With two CTAs per SM, a grid that fits twice lets the next layer's CTAs all be
-                // resident, streaming their tiles, while this layer's finish; that hides the
-                // ramp of each layer, which the tile-unit model does not see.  So the largest
-                // cluster size whose grid fits twice wins while each CTA keeps >= 4 tiles and the
-                // grid still holds a quarter of the resident CTAs, enough copies in flight to
-                // stream (measured, 64 segments of 16 tiles of 128: 2-CTA clusters 80.5 us per
-                // 12-layer step against 84.7 us for 4-CTA clusters; with 32 segments 4-CTA
-                // clusters, 128 CTAs, stay the better).
-                if (c->cluster == 1 && var->ctas_per_sm >= 2) {
+                // Inside a step whose next layer reads its tiles early (early_fetch), with two
+                // CTAs per SM, a grid that fits twice lets the next layer's CTAs all be resident,
+                // streaming their tiles, while this layer's finish; that hides the ramp of each
+                // layer, which the tile-unit model does not see.  So there the largest cluster
+                // size whose grid fits twice wins while each CTA keeps >= 4 tiles and the grid
+                // still holds a quarter of the resident CTAs, enough copies in flight to stream
+                // (measured, 64 segments of 16 tiles of 128: 2-CTA clusters 80.5 us per 12-layer
+                // step against 84.7 us for 4-CTA clusters; with 32 segments 4-CTA clusters, 128
+                // CTAs, stay the better).  A layer that nothing overlaps (a standalone call, the
+                // first layer of a step, a step without early fetch) takes the model's choice:
+                // 4-CTA clusters there, 99.8 against 123.9 us for the default workload's 12
+                // layers one after another.
+                if (c->cluster == 1 && var->ctas_per_sm >= 2 && early_fetch) {
                     for (int k : {4, 2}) {
                         if (cluster_k == 0 && nt % k == 0 && nt / k >= 4 && 2 * S * k <= wave &&
                             4 * S * k >= wave && var->clusters[k] >= 2 * S)
                             cluster_k = k;
                     }
                 }
+                const bool by_rule = cluster_k > 1;
                 for (int k : {2, 4}) {
-                    if (cluster_k > 1 && c->cluster == 1)
+                    if (by_rule)
                         break;      // chosen above
                     if (c->cluster > 1 && k != c->cluster)
                         continue;   // one cluster size asked for

@@ -168,15 +168,14 @@ def test_few_pieces_merge_inline():
                    options={"grid": 3, "tile_tokens": 64}, expect={"last_deferred_merge": 0})
 
 
-@pytest.mark.parametrize("b,L,tile,k,want_tile", [(64, 2048, 256, 2, 256), (64, 2048, 0, 2, 128),
+@pytest.mark.parametrize("b,L,tile,k,want_tile", [(64, 2048, 256, 2, 256), (64, 2048, 0, 4, 128),
                                                    (32, 2048, 0, 4, 128), (64, 256, 64, 4, 64)])
 @pytest.mark.parametrize("fused", [False, True])
 def test_cluster_merge(b, L, tile, k, want_tile, fused):
-    # One length for every sequence.  64 segments of 8 tiles of 256: 2-CTA clusters keep the
-    # one-wave makespan; by default 64 segments of 16 tiles of 128 (two CTAs per SM): 2-CTA
-    # clusters, so that the next layer's 128 CTAs fit beside them; 32 such segments: 4-CTA
-    # clusters; 64 segments of 4 tiles of 64: 4-CTA clusters.  The pieces of a segment are merged
-    # through DSMEM.
+    # One length for every sequence, layer calls one by one.  64 segments of 8 tiles of 256: 2-CTA
+    # clusters keep the one-wave makespan; by default 64 segments of 16 tiles of 128 (two CTAs per
+    # SM): 4-CTA clusters; 32 such segments: 4-CTA clusters; 64 segments of 4 tiles of 64: 4-CTA
+    # clusters.  The pieces of a segment are merged through DSMEM.
     opts = {"tile_tokens": tile} if tile else None
     run_small_case([0, 0, 2], 12, 1, 64, b, [L] * b, L, seed=17, fused=fused, options=opts,
                    expect={"last_cluster_k": k, "last_tile_tokens": want_tile})
