@@ -252,8 +252,10 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  kernel has completed); 0 = plain stream order
  *   "early_fetch"  1 (default) = in a step of per-layer launches, a layer's grid reads its queries
  *                  and every cache tile but the newest row's before the preceding layers' grids have
- *                  finished (the step is given every layer's queries); 0 = it reads nothing before
- *                  they have, as a layer whose queries come from the previous layer must
+ *                  finished (the step is given every layer's queries); 2 = only its first cache
+ *                  tile before then, its queries after (what a layer whose queries come from the
+ *                  previous layer may do: the cache and the owner's new token exist already);
+ *                  0 = nothing before then
  *   "step_graph"   2 (default) = mlkv_decode_step issues a one-launch step directly and replays a
  *                  recorded CUDA graph of a per-layer step; 1 = always the graph; 0 = never (see
  *                  mlkv_decode_step)

@@ -550,7 +550,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
     const long long slots = std::min<long long>(var->ctas_per_sm * c->sm_count, c->max_ctas);
     const long long S_all = static_cast<long long>(c->b) * c->g;
     long long whole = 0;   // CTAs of a whole-segment grid inside a decode step, or 0
-    if (c->grid <= 0 && c->cluster == 1 && uniform && early_fetch) {
+    if (c->grid <= 0 && c->cluster == 1 && uniform && early_fetch == 1) {
         // Inside a decode step the layers' grids overlap (each triggers the next at once), so
         // a layer need not fill the GPU: a grid of whole segments (no merge, hence no wait for
         // the previous layer before writing partials) of at most half the resident slots lets
@@ -600,7 +600,7 @@ static int decode_impl(mlkv_cache_t c, int layer, const void *K_new, const void 
                 // first layer of a step, a step without early fetch) takes the model's choice:
                 // 4-CTA clusters there, 99.8 against 123.9 us for the default workload's 12
                 // layers one after another.
-                if (c->cluster == 1 && var->ctas_per_sm >= 2 && early_fetch) {
+                if (c->cluster == 1 && var->ctas_per_sm >= 2 && early_fetch == 1) {
                     for (int k : {4, 2}) {
                         if (cluster_k == 0 && nt % k == 0 && nt / k >= 4 && 2 * S * k <= wave &&
                             4 * S * k >= wave && var->clusters[k] >= 2 * S)
@@ -1001,8 +1001,11 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
         if (e != cudaSuccess)
             return fail_cuda(e, "step event");
         // Layers after the first follow this library's own launch of the preceding layer.
-        const int early = (n > 0 && c->pdl && c->early_fetch) ? 1 : 0;
-        const char *q_next = n + 1 < c->l ? Q + qo * (n + 1) : nullptr;
+        // 1: queries and tiles before the previous layers' grids end; 2: only the first cache
+        // tile (the queries after) -- what a layer whose queries come from the previous layer
+        // may do
+        const int early = (n > 0 && c->pdl) ? c->early_fetch : 0;
+        const char *q_next = (early == 1 && n + 1 < c->l) ? Q + qo * (n + 1) : nullptr;
         // A segment's newest row is the step's new token of the owner: the owner layer appends
         // it itself (fused); a later layer of the block replaces that row of its tiles from the
         // same input without storing it.  So no layer waits for another's launch to store it
@@ -1786,8 +1789,8 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         return MLKV_OK;
     }
     if (std::strcmp(key, "early_fetch") == 0) {
-        if (value != 0 && value != 1)
-            return fail(MLKV_ERR_INVALID_ARG, "early_fetch must be 0 or 1");
+        if (value < 0 || value > 2)
+            return fail(MLKV_ERR_INVALID_ARG, "early_fetch must be 0, 1 or 2");
         c->early_fetch = static_cast<int>(value);
         return MLKV_OK;
     }

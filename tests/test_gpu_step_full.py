@@ -153,13 +153,14 @@ def test_step_host_buffers_config2_full_size():
 
 @pytest.mark.parametrize("options", [{"l2_prefetch": 0}, {"l2_persist": 1}, {"step_kernel": 0},
                                      {"step_graph": 1}, {"step_kernel": 0, "early_fetch": 0},
+                                     {"step_kernel": 0, "early_fetch": 2},
                                      {"step_kernel": 0, "pdl": 0}])
 def test_step_options_full_size(options):
     """Options that change where bytes come from or how the step is launched, never the result:
     the default workload and the varied-length GQA workload (slots larger than L2) with the L2
     prefetch off, with L2 persistence on, with per-layer launches instead of one multi-layer
-    launch (overlapping, overlapping with no read before the previous layer's end, and in plain
-    stream order), and with the multi-layer launch replayed from a recorded graph."""
+    launch (overlapping; with no read, or only the first cache tile, before the previous layer's
+    end; in plain stream order), and with the multi-layer launch replayed from a recorded graph."""
     import paper_2406_09297_gb300 as mlkv
     for index in (2, 3):
         try:
