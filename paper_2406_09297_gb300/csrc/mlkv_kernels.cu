@@ -998,10 +998,10 @@ __global__ void __launch_bounds__(Plan<D, T, STAGES, NCW>::kThreads,
 // combine kernel: merge of segments split over many CTAs
 // ------------------------------------------------------------------------------------------------
 
-// One CTA per (segment, query row of its group).  The CTA first turns the pieces' log-sum-exps
-// into normalised weights w_c = 2^(lse_c - M) / sum_c' 2^(lse_c' - M) (M = max_c lse_c), then
-// each thread sums w_c * o_c[e] for one column e over a strided subset of the pieces, with up to
-// 16 loads in flight, and the subsets are added through shared memory.
+// One CTA per (segment, query row of its group).  The CTA turns the pieces' log-sum-exps into
+// weights w_c = 2^(lse_c - M) (M = max_c lse_c) and each thread sums w_c * o_c[e] for one column
+// e over a strided subset of the pieces, 16 loads in flight (the first 16 issued with the
+// log-sum-exps); the subsets are added through shared memory and scaled by 1 / sum_c w_c.
 constexpr int kCombineThreads = 256;
 constexpr int kCombineMaxPieces = 1024;
 
@@ -1047,46 +1047,64 @@ __global__ void __launch_bounds__(kCombineThreads)
     const int beta = seg / p.g;
     const int j = seg - beta * p.g;
     const int tid = threadIdx.x;
+    const int lane = tid & 31, wid = tid >> 5;
+    constexpr int kWarps = kCombineThreads / 32;
     const float NEG_INF = -__int_as_float(0x7f800000);
-
+    constexpr int kGroups = kCombineThreads / D;   // pieces summed side by side per column
+    const int e = tid % D;
+    const int grp = tid / D;
+    const float *src = p.part_o + rec0 * G * D + static_cast<size_t>(row) * D + e;
+    // The first 16 pieces' values of this thread go out together with the pieces' log-sum-exps:
+    // one round trip to memory before the weights are known.
+    float v[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+        const int k = grp + m * kGroups;
+        v[m] = k < np ? __ldcg(src + static_cast<size_t>(k) * G * D) : 0.f;
+    }
     float mx = NEG_INF;
     for (int k = tid; k < np; k += kCombineThreads) {
-        const float v = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
-        s_w[k] = v;
-        mx = fmaxf(mx, v);
+        const float l = __ldcg(&p.part_lse[(rec0 + k) * G + row]);
+        s_w[k] = l;
+        mx = fmaxf(mx, l);
     }
-    s_red[tid] = mx;
+    // block reductions: within each warp by shuffles, then across the warps through s_red
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    if (lane == 0)
+        s_red[wid] = mx;
     __syncthreads();
-    for (int off = kCombineThreads / 2; off > 0; off >>= 1) {
-        if (tid < off)
-            s_red[tid] = fmaxf(s_red[tid], s_red[tid + off]);
-        __syncthreads();
-    }
     mx = s_red[0];
-    __syncthreads();
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w)
+        mx = fmaxf(mx, s_red[w]);
     float tot = 0.f;
     for (int k = tid; k < np; k += kCombineThreads) {
         const float w = fast_exp2(s_w[k] - mx);
         s_w[k] = w;
         tot += w;
     }
-    s_red[tid] = tot;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+        tot += __shfl_xor_sync(0xffffffffu, tot, off);
+    __syncthreads();   // every warp has read s_red's maxima; s_w holds the weights
+    if (lane == 0)
+        s_red[wid] = tot;
     __syncthreads();
-    for (int off = kCombineThreads / 2; off > 0; off >>= 1) {
-        if (tid < off)
-            s_red[tid] += s_red[tid + off];
-        __syncthreads();
-    }
-    const float inv = fast_rcp(s_red[0]);
-    __syncthreads();
-
-    constexpr int kGroups = kCombineThreads / D;   // pieces summed side by side per column
-    const int e = tid % D;
-    const int grp = tid / D;
-    const float *src = p.part_o + rec0 * G * D + static_cast<size_t>(row) * D + e;
+    tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w)
+        tot += s_red[w];
+    const float inv = fast_rcp(tot);
     float acc = 0.f;
-    for (int k0 = grp; k0 < np; k0 += kGroups * 16) {
-        float v[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+        const int k = grp + m * kGroups;
+        if (k < np)
+            acc += s_w[k] * v[m];
+    }
+    for (int k0 = grp + 16 * kGroups; k0 < np; k0 += kGroups * 16) {
 #pragma unroll
         for (int m = 0; m < 16; ++m) {
             const int k = k0 + m * kGroups;
@@ -1099,6 +1117,7 @@ __global__ void __launch_bounds__(kCombineThreads)
                 acc += s_w[k] * v[m];
         }
     }
+    __syncthreads();   // every thread has read the warps' sums
     s_red[tid] = acc;
     __syncthreads();
     if (grp == 0) {
