@@ -229,35 +229,42 @@ def _config_dict(w):
             "l2": "flushed before every timed step (512 MiB write)", "parallelism": "replicas"}
 
 
-KERNEL_SOURCES = ("mlkv_kernels.cu", "mlkv_device.cuh")   # what decode_kernel is built from
+# What each kernel is built from (the fused decode is the prefill kernel's fused form).
+KERNEL_SOURCES = {
+    "decode_kernel": ("mlkv_kernels.cu", "mlkv_device.cuh"),
+    "prefill_kernel": ("mlkv_prefill.cu", "mlkv_tcgen05.cuh", "mlkv_device.cuh"),
+}
 
 
-def _kernel_source_hash():
-    """sha256[:16] over the kernel sources, in KERNEL_SOURCES order."""
+def _kernel_source_hash(kernel="decode_kernel"):
+    """sha256[:16] over a kernel's sources, in KERNEL_SOURCES order."""
     import hashlib
     h = hashlib.sha256()
-    for name in KERNEL_SOURCES:
+    for name in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2406_09297_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
 def _recorded_traffic(w, kernel, launch):
-    """DRAM bytes per decode launch (dram__bytes_read.sum + dram__bytes_write.sum) from the ncu
-    capture recorded in profiles/decode_traffic.json for this workload, kernel and launch kind
-    ("multi-layer": one launch for the step, "per-layer"), or None when there is none or the
-    kernel source changed since it was taken."""
+    """DRAM bytes per launch of the step's dominant kernel (dram__bytes_read.sum +
+    dram__bytes_write.sum) from the ncu capture recorded in profiles/decode_traffic.json for this
+    workload, kernel and step form ("multi-layer": one decode launch for the step, "fused": the
+    cross-layer fused form, "per-layer"), or None when there is none or the kernel's sources
+    changed since it was taken."""
     try:
         with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
             rec = json.load(f)
     except Exception:
         return None
-    entry = rec.get(w.name)
-    if not entry or entry.get("kernel_source_sha256_16") != _kernel_source_hash():
+    if kernel not in KERNEL_SOURCES:
         return None
-    if entry.get("kernel", "decode_kernel") != kernel or entry.get("launch") != launch:
-        return None
-    return entry.get("dram_bytes_per_launch")
+    for entry in rec.get("entries", []):
+        if (entry.get("workload") == w.name and entry.get("kernel") == kernel and
+                entry.get("launch") == launch and
+                entry.get("kernel_source_sha256_16") == _kernel_source_hash(kernel)):
+            return entry.get("dram_bytes_per_launch")
+    return None
 
 
 def kv_bytes_per_layer(w, seq_lens):
@@ -290,6 +297,10 @@ def run(args, w):
         cache.set_option("l2_prefetch", args.l2_prefetch)
     if args.step_kernel >= 0:
         cache.set_option("step_kernel", args.step_kernel)
+    if args.step_fused >= 0:
+        cache.set_option("step_fused", args.step_fused)
+    if args.fused_kc > 0:
+        cache.set_option("fused_kc", args.fused_kc)
     if args.no_pdl:
         cache.set_option("pdl", 0)
     cache.set_option("tc", args.tc)
@@ -310,11 +321,19 @@ def run(args, w):
 
     step()
     cache.sync_status()
-    step_kernel = bool(cache.get_option("last_step_kernel"))   # one launch for every layer
+    step_info = {k: int(cache.get_option(k)) for k in ("last_step_kernel", "last_step_fused",
+                                                        "last_step_launches", "last_fused_kc",
+                                                        "last_grid", "last_tile_tokens",
+                                                        "last_deferred_merge", "last_seg_major")}
+    step_kernel = bool(step_info["last_step_kernel"])   # one launch for every layer
+    fused = bool(step_info["last_step_fused"])          # ... in the cross-layer fused form
     # a decode launch per layer, or one for the whole step; each followed by a merge launch when
-    # the split pieces' partials are merged after the decode (deferred merge)
+    # the split pieces' partials are merged after the decode (deferred merge); the fused form
+    # stores the owners' new tokens in a launch of its own before its decode launch
     merges = 2 if cache.get_option("last_deferred_merge") else 1
-    launches_per_step = merges * (1 if step_kernel else w.l)
+    launches_per_step = (int(cache.get_option("last_step_launches")) if step_kernel
+                         else merges * w.l)
+    form = "fused" if fused else ("multi-layer" if step_kernel else "per-layer")
 
     def barrier():
         if dist is not None:
@@ -410,12 +429,13 @@ def run(args, w):
     cold = [layer_ms[n] for n in range(w.l) if w.owner[n] == n]
     cold_gbs = alg_bytes / (statistics.mean(cold) / 1e3) / 1e9
     del big_flush
-    kernel_name = "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel"
+    kernel_name = ("prefill_kernel" if fused else
+                   "decode_tc_kernel" if cache.get_option("last_tc") else "decode_kernel")
     options = {k: int(cache.get_option(k)) for k in ("l2_prefetch", "l2_persist", "tc",
-                                                      "step_kernel", "l2_persist_bytes",
-                                                      "l2_window_max", "last_step_kernel",
-                                                      "last_seg_major")}
-    traffic = _recorded_traffic(w, kernel_name, "multi-layer" if step_kernel else "per-layer")
+                                                      "step_kernel", "step_fused",
+                                                      "l2_persist_bytes", "l2_window_max")}
+    options.update(step_info)   # the measured step's launch, read right after its first call
+    traffic = _recorded_traffic(w, kernel_name, form)
 
     # ---- end to end through the C ABI with host buffers --------------------------------------
     host_q = Qs.cpu().pin_memory()
@@ -474,10 +494,13 @@ def run(args, w):
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind,
                          "frac_vs_8tbs": achieved / 8000.0,
-                         "kernel": kernel_name, "alg_bytes_per_launch": launch_bytes,
+                         "kernel": kernel_name, "step_form": form,
+                         "alg_bytes_per_launch": launch_bytes,
                          "mean_launch_ms": launch_ms, "launches_per_step": launches_per_step,
-                         # the merge launch's time is inside mean_launch_ms (timed together)
+                         # the merge launch's time is inside mean_launch_ms (timed together),
+                         # and in the fused form the new tokens' store launch's
                          "merge_time_included": merges == 2,
+                         "append_time_included": fused,
                          "step_ms_per_layer": mean_kernel_ms,
                          "dram_unique_bytes_per_step": unique_bytes,
                          "dram_unique_gbs": unique_gbs,
@@ -532,6 +555,10 @@ def run_loop(args):
                 cache.set_option("grid", args.grid)
             if args.cluster >= 0:
                 cache.set_option("cluster", args.cluster)
+            if args.step_fused >= 0:
+                cache.set_option("step_fused", args.step_fused)
+            if args.fused_kc > 0:
+                cache.set_option("fused_kc", args.fused_kc)
             for n in owners:
                 kp, vp, strides = cache.kv_ptr(cache.owner_slot(n)[1])
                 device.fill_slot(kp, vp, strides, seed, n, b, g, d, max_seq)
@@ -822,6 +849,10 @@ def main():
                     help="option l2_prefetch (-1: the library's default)")
     ap.add_argument("--step-kernel", type=int, default=-1, choices=[-1, 0, 1],
                     help="option step_kernel (-1: the library's default)")
+    ap.add_argument("--step-fused", type=int, default=-1, choices=[-1, 0, 1, 2],
+                    help="option step_fused (-1: the library's default)")
+    ap.add_argument("--fused-kc", type=int, default=0,
+                    help="option fused_kc: key tiles per unit of the fused step (0: planned)")
     ap.add_argument("--no-pdl", action="store_true")
     ap.add_argument("--tc", type=int, default=0, choices=[0, 1],
                     help="0: the mma.sync decode kernel (default); 1: the tcgen05 kernel")

@@ -130,11 +130,22 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
  *   K, V     device bf16 [m][batch][g][d], every owner layer's new token, in slot order
  *   out      device bf16 [l][batch][h][d]
  *   seq_lens host int32[batch], as for mlkv_decode_attention
+ * All four device buffers 16-byte aligned (else MLKV_ERR_INVALID_ARG).
  * The results equal those of the layer calls up to rounding: inside a step the layers' launches
  * overlap and may split a layer's work differently (whole segments per CTA).  Every layer of an
  * owner's block reads that owner's new token from K and V (the later layers take their newest
  * row from there rather than from the cache), so K and V, like Q, must stay valid until the stream
  * has run the whole step.
+ * Cross-layer fused form (option "step_fused"): for maps of equal contiguous owner blocks
+ * (owner[n] = n - n mod (l/m), the layout of Sec. 3, Eq. 18) whose (l/m) * (h/g) query rows per KV
+ * head fit two tiles of 128, the step is one launch that stores every owner's new token, one
+ * tcgen05 launch in which each unit (sequence, KV head, block, chunk of the context) loads every
+ * K/V tile of its chunk once for all the block's layers' query rows, and, when a segment is split
+ * into chunks, one merge launch.  Other maps, option "step_fused" = 0, and the
+ * options that select the decode kernel's shapes ("grid", "tile_tokens", "tc", "l2_prefetch",
+ * "l2_persist") take the decode kernel's multi-layer launch.  Option "last_step_fused" reads
+ * back 1 if the most recent step ran in the fused form, "last_step_launches" the number of this
+ * library's launches of that step, "last_fused_kc" the key tiles of 128 positions per unit.
  * Option "step_graph": with 1 a call whose pointers, lengths and options equal those of the
  * previous call replays a CUDA graph of the step's launches (recorded on the second such call; new
  * values in the same buffers are fine); a call with arguments different from the previous call's
@@ -241,6 +252,15 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  (the layers of a block read each segment at about the same time, so L2 serves
  *                  all but the first), else layer by layer.  0 = always one launch per layer.
  *                  Same results within the tolerance.
+ *   "step_fused"   1 (default) = where "step_kernel" gives one launch for the step, the map has
+ *                  equal contiguous owner blocks of >= 3 layers whose query rows fit two 128-row
+ *                  tiles, and the owner slots hold >= 4 tiles of 128 visible positions per SM, the
+ *                  step runs in the cross-layer fused form (see mlkv_decode_step); 2 = that form
+ *                  wherever the map allows it (blocks of any size, any step); 0 = the decode
+ *                  kernel's multi-layer launch.  Same results within the tolerance.
+ *   "fused_kc"     > 0 = key tiles of 128 positions per unit of the fused form (clamped to what
+ *                  the unit word holds); 0 (default) = planned: a sequence is split only as far
+ *                  as the units still number at most the SMs.
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through
@@ -268,9 +288,12 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  * "last_deferred_merge", "last_tc" (1 if it ran the tcgen05 kernel), and "step_graph_replays"
  * (graph launches by mlkv_decode_step), "l2_persist_bytes" (the set-aside reserved while
  * l2_persist is on, else 0), "l2_window_max" (the device's largest access-policy window),
- * "last_step_kernel" (1 if the most recent mlkv_decode_step ran as one multi-layer launch),
- * "last_seg_major" (1 if that launch ranked its items segment-major) and "last_l2_prefetch" (1
- * if it prefetched the slots into L2).
+ * "last_step_kernel" (1 if the most recent mlkv_decode_step ran as one multi-layer launch or in
+ * the fused form), "last_step_fused" (1 if in the fused form; "last_grid" is then its units and
+ * "last_fused_kc" the 128-position key tiles per unit), "last_step_launches" (this library's
+ * launches of that step when it ran in either form, else 0), "last_seg_major" (1 if the
+ * multi-layer launch ranked its items segment-major) and "last_l2_prefetch" (1 if it prefetched
+ * the slots into L2).
  * Unknown keys or values return MLKV_ERR_INVALID_ARG.
  */
 int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value);

@@ -125,9 +125,15 @@ struct mlkv_cache {
     int early_fetch = 1;        // per-layer step: later layers read Q and tiles before the wait
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
-    int fused_ready = 0;        // the same for the fused-decode instance
-    float *fused_part = nullptr;   // context-chunk partials of mlkv_decode_block_fused
+    int fused_ready = 0;        // the same for the fused-decode forms (bit 1: two tiles, 2: one)
+    float *fused_part = nullptr;   // context-chunk partials of the fused decode
     size_t fused_part_floats = 0;
+    int step_fused = 1;         // mlkv_decode_step: the cross-layer fused form where it pays (1),
+                                // wherever the map allows it (2), never (0)
+    int last_step_fused = 0;    // 1 if the most recent step ran in that form
+    int last_step_launches = 0;   // this library's launches in the most recent step
+    int last_fused_kc = 0;      // key tiles per unit (chunk) of the most recent fused decode
+    int fused_kc = 0;           // > 0: key tiles per unit of the fused decode, else planned
     // mlkv_decode_step's recorded graph and the arguments it was recorded for
     int step_graph = 2;         // 2: direct when one multi-layer launch, else record/replay
     cudaStream_t record_stream = nullptr;   // private stream the step graph is recorded on
@@ -138,13 +144,13 @@ struct mlkv_cache {
         std::vector<int> lens;
         int tile = -1, grid = -1, cluster = -1, pdl = -1, l2 = -1, tc = -1, pf = -1, sk = -1;
         int sg = -1;   // step_graph: a graph recorded under one mode is not replayed under another
-        int ef = -1;
+        int ef = -1, sf = -1;
         bool operator==(const StepKey &o) const
         {
             return Q == o.Q && K == o.K && V == o.V && out == o.out && lens == o.lens &&
                    tile == o.tile && grid == o.grid && cluster == o.cluster && pdl == o.pdl &&
                    l2 == o.l2 && tc == o.tc && pf == o.pf && sk == o.sk && sg == o.sg &&
-                   ef == o.ef;
+                   ef == o.ef && sf == o.sf;
         }
     } step_key, pending_key;   // recorded arguments; arguments seen once, not yet recorded
     int step_graph_replays = 0;
@@ -463,6 +469,7 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
     p.d = c->d;
     p.max_seq = c->max_seq;
     p.slot = c->slot[layer];
+    p.n_slots = 1;
     std::memcpy(p.seq_len, seq_lens, sizeof(int) * c->b);
     DeviceGuard guard(c->device);
     cudaError_t e = mlkv::launch_append(p, static_cast<cudaStream_t>(cuda_stream));
@@ -736,14 +743,311 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
 // waits for it (queries still arriving).
 // With `stage`, the copy of the step's inputs it describes is launched right before the step's
 // kernel, which may then start (and fetch its first cache tiles) while the copy runs.
+// The fused decode's context split for nblk blocks: kc key tiles of 128 positions a unit; *units
+// (if given) the units it makes.  Measured on GB300 (batch 64 x 2048 positions, 72 rows a unit):
+// one CTA keeps an SM's softmax and tensor core about as busy as two do, while every unit costs
+// ~5 us outside its key tiles (start, first loads, output) and a split adds the merge launch (16
+// tiles a unit, 128 units: 31 us per step; 8 tiles, 256 units: 39; 4: 43; 1: 63).  So a sequence is
+// split only as far as the units still fit one per SM: the smallest kc whose units number at most
+// the SMs; no split when the (sequence, KV head, block) units alone exceed them.  The unit word
+// holds chunk indices below kFusedMaxChunks.
+static int fused_plan(const mlkv_cache *c, const int *seq_lens, int nblk, long long *units)
+{
+    int n_kt_max = 0;
+    bool uniform = true;
+    for (int beta = 0; beta < c->b; ++beta) {
+        n_kt_max = std::max(n_kt_max, (seq_lens[beta] + 127) / 128);
+        uniform = uniform && seq_lens[beta] == seq_lens[0];
+    }
+    const long long per_seq = static_cast<long long>(nblk) * c->g;
+    const int kc_min = std::max(1, (n_kt_max + mlkv::kFusedMaxChunks - 2) /
+                                       (mlkv::kFusedMaxChunks - 1));
+    auto units_for = [&](int k) {
+        if (uniform)
+            return per_seq * c->b * ((n_kt_max + k - 1) / k);
+        long long u = 0;
+        for (int beta = 0; beta < c->b; ++beta)
+            u += per_seq * (((seq_lens[beta] + 127) / 128 + k - 1) / k);
+        return u;
+    };
+    int kc = n_kt_max;
+    if (units_for(n_kt_max) < c->sm_count) {
+        // units_for falls as k grows: the smallest k with units <= SMs, by bisection
+        int lo = kc_min, hi = n_kt_max;
+        while (lo < hi) {
+            const int mid = lo + (hi - lo) / 2;
+            if (units_for(mid) <= c->sm_count)
+                hi = mid;
+            else
+                lo = mid + 1;
+        }
+        kc = lo;
+    }
+    if (c->fused_kc > 0)
+        kc = std::max(kc_min, std::min(c->fused_kc, n_kt_max));
+    if (units != nullptr)
+        *units = units_for(kc);
+    return kc;
+}
+
+// The cross-layer fused decode (the fused form of prefill_kernel) over nblk owner blocks of L
+// layers each: block k reads slot slot0 + k and attends for the layers k*L .. k*L + L - 1 of Q and
+// out ([n_q_layers][b][h][d]).  A unit (sequence, KV head, block, chunk of the context) loads each
+// K/V tile of its chunk once for all L*G query rows of the block (Sec. 3: the block's layers read
+// one cache); a sequence's chunks are merged by one combine_fused launch.  Launches issued are
+// added to *launches.
+static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers, int L, int nblk,
+                       int slot0, const int *seq_lens, cudaStream_t stream, int *launches,
+                       bool after_store = false)
+{
+    const int L1 = 128 / c->G;
+    const bool one = c->d == 64 && L <= L1;   // one query tile per CTA, two CTAs per SM
+    const int form = one ? 2 : 1;
+    cudaError_t e;
+    if (!(c->fused_ready & form)) {
+        if ((e = mlkv::prepare_fused(c->d, one)) != cudaSuccess)
+            return fail_cuda(e, "cudaFuncSetAttribute(fused decode)");
+        c->fused_ready |= form;
+    }
+    static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
+    if (encode == nullptr)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+    // Q [layers][b][h][d] as (channel, head in group, group, sequence, layer); a box of 64
+    // channels x G heads x min(L1, L) layers is one tile's rows, layer-major.
+    CUtensorMap tmap_q;
+    const cuuint64_t dims[5] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->G),
+                                static_cast<cuuint64_t>(c->g), static_cast<cuuint64_t>(c->b),
+                                static_cast<cuuint64_t>(n_q_layers)};
+    const cuuint64_t strides[4] = {static_cast<cuuint64_t>(c->d) * 2,
+                                   static_cast<cuuint64_t>(c->G) * c->d * 2,
+                                   static_cast<cuuint64_t>(c->h) * c->d * 2,
+                                   static_cast<cuuint64_t>(c->b) * c->h * c->d * 2};
+    const cuuint32_t box[5] = {64u, static_cast<cuuint32_t>(c->G), 1u, 1u,
+                               static_cast<cuuint32_t>(L < L1 ? L : L1)};
+    const cuuint32_t estr[5] = {1u, 1u, 1u, 1u, 1u};
+    CUresult r = encode(&tmap_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(Q), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled(fused Q) failed (CUresult %d)",
+                    static_cast<int>(r));
+    const CUtensorMap *tmap_kv = nullptr;
+    for (auto &v : c->variants)
+        if (v.v->tile_tokens == 128)
+            tmap_kv = &v.tmap;
+    if (tmap_kv == nullptr)
+        return fail(MLKV_ERR_UNSUPPORTED, "no 128-position cache map for d=%d", c->d);
+
+    static thread_local mlkv::PrefillParams p;
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.err = c->err;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
+    p.b = c->b;
+    p.h = c->h;
+    p.g = c->g;
+    p.G = c->G;
+    p.s_max = c->max_seq;
+    p.slot = slot0;
+    p.head_pairs = 0;
+    p.fused_L = L;
+    p.fused_L1 = L1;
+    p.fused_nblk = nblk;
+    p.fused_early = after_store ? 1 : 0;
+    int n_kt_max = 0;
+    long long kt_sum = 0;
+    bool uniform = true;
+    for (int beta = 0; beta < c->b; ++beta) {
+        p.prompt_len[beta] = seq_lens[beta];
+        const int nkt = (seq_lens[beta] + 127) / 128;
+        n_kt_max = std::max(n_kt_max, nkt);
+        kt_sum += nkt;
+        uniform = uniform && seq_lens[beta] == seq_lens[0];
+    }
+    const int kc = fused_plan(c, seq_lens, nblk, nullptr);
+    (void)kt_sum;
+    const int cmax = (n_kt_max + kc - 1) / kc;
+    p.fused_kc = kc;
+    p.fused_cmax = cmax;
+    // merge: one warp per output row up to 8 chunks, then 2, 4 or 8 warps sharing a row's chunks
+    p.fused_combine_w = cmax <= 8 ? 1 : cmax <= 16 ? 2 : cmax <= 32 ? 4 : 8;
+    p.part = p.part_lse = nullptr;
+    if (cmax > 1) {
+        const size_t rows = static_cast<size_t>(nblk) * c->b * c->g * cmax * L * c->G;
+        const size_t floats = rows * (c->d + 1);
+        if (floats > c->fused_part_floats) {
+            if (c->fused_part)
+                cudaFree(c->fused_part);
+            c->fused_part = nullptr;
+            c->fused_part_floats = 0;
+            if ((e = cudaMalloc(&c->fused_part, floats * sizeof(float))) != cudaSuccess) {
+                c->fused_part = nullptr;
+                return fail(MLKV_ERR_OOM, "fused-decode partials (%zu bytes): %s",
+                            floats * sizeof(float), cudaGetErrorString(e));
+            }
+            c->fused_part_floats = floats;
+        }
+        p.part = c->fused_part;
+        p.part_lse = c->fused_part + rows * c->d;
+    }
+    // Units: the longest sequences first; within a sequence block, KV head, chunk.
+    static thread_local std::vector<int> order;
+    order.resize(c->b);
+    for (int beta = 0; beta < c->b; ++beta)
+        order[beta] = beta;
+    if (!uniform)
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
+    int n = 0;
+    long long total_units = 0;
+    for (int beta : order)
+        for (int blk = 0; blk < nblk; ++blk)
+            for (int j = 0; j < c->g; ++j)
+                for (int ch = 0; ch * kc < (seq_lens[beta] + 127) / 128; ++ch) {
+                    p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(ch) << 10) |
+                                 (static_cast<uint32_t>(blk) << 18) |
+                                 (static_cast<uint32_t>(j) << 24);
+                    ++total_units;
+                    if (++n == mlkv::kPrefillMaxUnits) {
+                        p.n_units = n;
+                        if ((e = mlkv::launch_fused(c->d, one, &tmap_q, tmap_kv, p, stream)) !=
+                            cudaSuccess)
+                            return fail_cuda(e, "fused decode launch");
+                        ++*launches;
+                        n = 0;
+                    }
+                }
+    if (n > 0) {
+        p.n_units = n;
+        if ((e = mlkv::launch_fused(c->d, one, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+            return fail_cuda(e, "fused decode launch");
+        ++*launches;
+    }
+    if (cmax > 1) {
+        if ((e = mlkv::launch_fused_combine(c->d, p, stream)) != cudaSuccess)
+            return fail_cuda(e, "fused decode merge launch");
+        ++*launches;
+    }
+    c->last_grid = static_cast<int>(std::min<long long>(total_units, 0x7fffffffLL));
+    c->last_tile = 128;
+    c->last_deferred = cmax > 1 ? 1 : 0;
+    c->last_fused_kc = kc;
+    return MLKV_OK;
+}
+
+// mlkv_decode_step in the cross-layer fused form: one append launch for every owner's new token,
+// then the fused decode of every block in one launch (and one merge).  Applies to maps of equal
+// contiguous blocks (owner[n] = n - n mod L, the paper's Eq. 18 layout) whose L*G query rows fit
+// two 128-row tiles; otherwise *done stays false.
+static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
+                            const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
+                            const mlkv::StageParams *stage)
+{
+    *done = false;
+    if (!c->step_fused || c->tile_tokens > 0 || c->l2_prefetch || c->m > mlkv::kFusedMaxBlocks ||
+        c->g > 255 || c->h > mlkv::kPrefillMaxHeads || (c->d != 64 && c->d != 128))
+        return MLKV_OK;
+    const int L = c->l / c->m;
+    const int L1 = 128 / c->G;
+    if (L * c->m != c->l || L1 < 1 || L > 2 * L1)
+        return MLKV_OK;
+    for (int n = 0; n < c->l; ++n)
+        if (c->owner[n] != n - n % L || c->slot[n] != n / L)
+            return MLKV_OK;
+    if (c->step_fused == 1) {
+        // Where the fused form pays, from measurements on GB300 against the decode kernel's
+        // launch.  A block of one layer shares nothing across layers (MHA, GQA-4, MQA at batch
+        // 256 and 1: 7-16% slower fused); blocks of two saved little or lost (batch 64 x 2000
+        // positions 49 vs 53 us, batch 256 x 8192 535 vs 548, batch 1 x 131072 66 vs 62, batch
+        // 1 x 128 11.6 vs 10.3).  For blocks of >= 3 layers the estimates in us per step, from the
+        // same measurements: the fused form ~1.1 per key tile its busiest SM takes plus ~6 fixed
+        // (+3 for the merge of a split); the decode kernel ~0.55 per (layer, sequence, KV head,
+        // 128 positions) item per SM plus ~3.  They pick the measured winner at batch 8, 64, 128
+        // and 256, batch 1 x 131072 and Llama-2-7B shapes.
+        if (L < 3)
+            return MLKV_OK;
+        long long units = 0;
+        const int kc = fused_plan(c, seq_lens, c->m, &units);
+        long long tiles = 0;
+        int n_kt_max = 0;
+        bool uniform = true;
+        for (int beta = 0; beta < c->b; ++beta) {
+            tiles += (seq_lens[beta] + 127) / 128;
+            n_kt_max = std::max(n_kt_max, (seq_lens[beta] + 127) / 128);
+            uniform = uniform && seq_lens[beta] == seq_lens[0];
+        }
+        // the busiest SM's key tiles: whole waves of equal units with one length; with varied
+        // lengths (units longest first) about the mean, and at least one unit
+        const long long busiest =
+            uniform ? (units + c->sm_count - 1) / c->sm_count * kc
+                    : std::max<long long>(kc, (tiles * c->m * c->g + c->sm_count - 1) /
+                                                  c->sm_count);
+        const double fused_us =
+            1.1 * static_cast<double>(busiest) + 6.0 + (kc < n_kt_max ? 3.0 : 0.0);
+        const double ml_us = 0.55 * static_cast<double>(tiles) * c->l * c->g / c->sm_count + 3.0;
+        if (fused_us >= ml_us)
+            return MLKV_OK;
+    }
+    bool has_map = false;   // the cache's tensor map of 128-position tiles
+    for (auto &v : c->variants)
+        has_map = has_map || v.v->tile_tokens == 128;
+    if (!has_map)
+        return MLKV_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    DeviceGuard guard(c->device);
+    if (in_ready != nullptr && (e = cudaStreamWaitEvent(s, in_ready, 0)) != cudaSuccess)
+        return fail_cuda(e, "step event");
+    int launches = 0;
+    if (stage != nullptr) {
+        if ((e = mlkv::launch_stage_copy(*stage, s)) != cudaSuccess)
+            return fail_cuda(e, "copy-in of the step's inputs");
+        ++launches;
+    }
+    // Every owner's new token at position L_beta - 1 of its slot, before any block reads it.
+    mlkv::AppendParams ap;
+    ap.K = reinterpret_cast<const __nv_bfloat16 *>(K);
+    ap.V = reinterpret_cast<const __nv_bfloat16 *>(V);
+    ap.cache = static_cast<__nv_bfloat16 *>(c->cache);
+    ap.b = c->b;
+    ap.g = c->g;
+    ap.d = c->d;
+    ap.max_seq = c->max_seq;
+    ap.slot = 0;
+    ap.n_slots = c->m;
+    std::memcpy(ap.seq_len, seq_lens, sizeof(int) * c->b);
+    if ((e = mlkv::launch_append_slots(ap, s)) != cudaSuccess)
+        return fail_cuda(e, "append launch (fused step)");
+    ++launches;
+    const int rc = fused_issue(c, Q, out, c->l, L, c->m, 0, seq_lens, s, &launches, true);
+    if (rc != MLKV_OK)
+        return rc;
+    c->last_cluster_k = 0;
+    c->last_tc = 0;
+    c->last_l2_prefetch = 0;
+    c->last_step_kernel = 1;
+    c->last_step_fused = 1;
+    c->last_seg_major = 0;
+    c->last_step_launches = launches - (stage != nullptr ? 1 : 0);
+    *done = true;
+    return MLKV_OK;
+}
+
 static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
                          const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
                          const mlkv::StageParams *stage = nullptr)
 {
     *done = false;
     c->last_step_kernel = 0;
+    c->last_step_fused = 0;
+    c->last_step_launches = 0;
     if (!c->step_kernel || c->tc || c->grid > 0 || c->l2_persist || c->l > mlkv::kMaxStepLayers)
         return MLKV_OK;
+    {
+        const int rc = issue_step_fused(c, Q, K, V, out, seq_lens, stream, in_ready, done, stage);
+        if (rc != MLKV_OK || *done)
+            return rc;
+    }
     bool uniform = true;
     long long len_sum = 0;
     for (int beta = 0; beta < c->b; ++beta) {
@@ -971,6 +1275,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     c->last_l2_prefetch = p.pf_own;
     c->last_step_kernel = 1;
     c->last_seg_major = seg_major;
+    c->last_step_launches = p.deferred_merge ? 2 : 1;
     *done = true;
     return MLKV_OK;
 }
@@ -983,6 +1288,9 @@ static int issue_step(mlkv_cache_t c, const char *Q, const char *K, const char *
                       const int *seq_lens, void *stream, cudaEvent_t in_ready = nullptr,
                       cudaEvent_t before_last = nullptr)
 {
+    c->last_step_kernel = 0;
+    c->last_step_fused = 0;
+    c->last_step_launches = 0;
     if (before_last == nullptr) {
         bool done = false;
         const int rc = issue_step_ml(c, Q, K, V, out, seq_lens, stream, in_ready, &done);
@@ -1051,6 +1359,7 @@ mlkv_cache::StepKey step_key_of(const mlkv_cache *c, const void *Q, const void *
     key.sk = c->step_kernel;
     key.sg = c->step_graph;
     key.ef = c->early_fetch;
+    key.sf = c->step_fused;
     return key;
 }
 
@@ -1125,6 +1434,8 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
         return fail(MLKV_ERR_INVALID_ARG, "null cache handle");
     if (Q == nullptr || K == nullptr || V == nullptr || out == nullptr)
         return fail(MLKV_ERR_INVALID_ARG, "Q, K, V and out must be non-NULL");
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out))
+        return fail(MLKV_ERR_INVALID_ARG, "Q, K, V and out must be 16-byte aligned");
     int rc = check_seq_lens(c, seq_lens);
     if (rc != MLKV_OK)
         return rc;
@@ -1496,117 +1807,9 @@ int mlkv_decode_block_fused(mlkv_cache_t c, int owner_layer, const void *Q, void
     if (os < qs + qbytes && qs < os + qbytes)
         return fail(MLKV_ERR_INVALID_ARG, "out overlaps Q");
     DeviceGuard guard(c->device);
-    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-    cudaError_t e;
-    if (!c->fused_ready) {
-        if ((e = mlkv::prepare_fused(c->d)) != cudaSuccess)
-            return fail_cuda(e, "cudaFuncSetAttribute(fused decode)");
-        c->fused_ready = 1;
-    }
-    static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
-    if (encode == nullptr)
-        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
-    // Q [L][b][h][d] as (channel, head in group, group, sequence, layer); a box of 64 channels x
-    // G heads x min(L1, L) layers is one tile's rows, layer-major.
-    CUtensorMap tmap_q;
-    const cuuint64_t dims[5] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->G),
-                                static_cast<cuuint64_t>(c->g), static_cast<cuuint64_t>(c->b),
-                                static_cast<cuuint64_t>(L)};
-    const cuuint64_t strides[4] = {static_cast<cuuint64_t>(c->d) * 2,
-                                   static_cast<cuuint64_t>(c->G) * c->d * 2,
-                                   static_cast<cuuint64_t>(c->h) * c->d * 2,
-                                   static_cast<cuuint64_t>(c->b) * c->h * c->d * 2};
-    const cuuint32_t box[5] = {64u, static_cast<cuuint32_t>(c->G), 1u, 1u,
-                               static_cast<cuuint32_t>(L < L1 ? L : L1)};
-    const cuuint32_t estr[5] = {1u, 1u, 1u, 1u, 1u};
-    CUresult r = encode(&tmap_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(Q), dims,
-                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS)
-        return fail(MLKV_ERR_CUDA, "cuTensorMapEncodeTiled(fused Q) failed (CUresult %d)",
-                    static_cast<int>(r));
-    const CUtensorMap *tmap_kv = nullptr;
-    for (auto &v : c->variants)
-        if (v.v->tile_tokens == 128)
-            tmap_kv = &v.tmap;
-    if (tmap_kv == nullptr)
-        return fail(MLKV_ERR_UNSUPPORTED, "no 128-position cache map for d=%d", c->d);
-
-    static thread_local mlkv::PrefillParams p;
-    p.out = static_cast<__nv_bfloat16 *>(out);
-    p.err = c->err;
-    p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->d)));
-    p.b = c->b;
-    p.h = c->h;
-    p.g = c->g;
-    p.G = c->G;
-    p.s_max = c->max_seq;
-    p.slot = c->slot[owner_layer];
-    p.head_pairs = 0;
-    p.fused_L = L;
-    p.fused_L1 = L1;
-    int max_len = 0;
-    for (int beta = 0; beta < c->b; ++beta) {
-        p.prompt_len[beta] = seq_lens[beta];
-        max_len = std::max(max_len, seq_lens[beta]);
-    }
-    // Units (sequence, KV head, chunk of the context): about one per SM when there are fewer
-    // (sequence, KV head) pairs than SMs, the chunks' partial results then merged.
-    const int n_kt_max = (max_len + 127) / 128;
-    const int want = std::max(1, 152 / (c->b * c->g));
-    int kc = (n_kt_max + want - 1) / want;
-    kc = std::max(kc, (n_kt_max + mlkv::kPrefillMaxBlocks - 1) / mlkv::kPrefillMaxBlocks);
-    const int cmax = (n_kt_max + kc - 1) / kc;
-    p.fused_kc = kc;
-    p.fused_cmax = cmax;
-    p.part = p.part_lse = nullptr;
-    if (cmax > 1) {
-        const size_t rows = static_cast<size_t>(c->b) * c->g * cmax * L * c->G;
-        const size_t floats = rows * (c->d + 1);
-        if (floats > c->fused_part_floats) {
-            if (c->fused_part)
-                cudaFree(c->fused_part);
-            c->fused_part = nullptr;
-            c->fused_part_floats = 0;
-            if ((e = cudaMalloc(&c->fused_part, floats * sizeof(float))) != cudaSuccess) {
-                c->fused_part = nullptr;
-                return fail(MLKV_ERR_OOM, "fused-decode partials (%zu bytes): %s",
-                            floats * sizeof(float), cudaGetErrorString(e));
-            }
-            c->fused_part_floats = floats;
-        }
-        p.part = c->fused_part;
-        p.part_lse = c->fused_part + rows * c->d;
-    }
-    // The longest sequences first.
-    std::vector<int> order(c->b);
-    for (int beta = 0; beta < c->b; ++beta)
-        order[beta] = beta;
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int x, int y) { return seq_lens[x] > seq_lens[y]; });
-    int n = 0;
-    for (int beta : order)
-        for (int j = 0; j < c->g; ++j)
-            for (int ch = 0; ch * kc < (seq_lens[beta] + 127) / 128; ++ch) {
-                p.units[n] = static_cast<uint32_t>(beta) | (static_cast<uint32_t>(ch) << 10) |
-                             (static_cast<uint32_t>(j) << 24);
-                if (++n == mlkv::kPrefillMaxUnits) {
-                    p.n_units = n;
-                    if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) !=
-                        cudaSuccess)
-                        return fail_cuda(e, "fused decode launch");
-                    n = 0;
-                }
-            }
-    if (n > 0) {
-        p.n_units = n;
-        if ((e = mlkv::launch_fused(c->d, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
-            return fail_cuda(e, "fused decode launch");
-    }
-    if (cmax > 1 && (e = mlkv::launch_fused_combine(c->d, p, stream)) != cudaSuccess)
-        return fail_cuda(e, "fused decode merge launch");
-    return MLKV_OK;
+    int launches = 0;
+    return fused_issue(c, Q, out, L, L, 1, c->slot[owner_layer], seq_lens,
+                       static_cast<cudaStream_t>(cuda_stream), &launches);
 }
 
 int mlkv_merge_kv_weights(const int *layer_owner, int n_layers, int n_q_heads, int n_kv_heads,
@@ -1776,6 +1979,18 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->step_kernel = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "step_fused") == 0) {
+        if (value < 0 || value > 2)
+            return fail(MLKV_ERR_INVALID_ARG, "step_fused must be 0, 1 or 2");
+        c->step_fused = static_cast<int>(value);
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "fused_kc") == 0) {
+        if (value < 0 || value > (1 << 20))
+            return fail(MLKV_ERR_INVALID_ARG, "fused_kc must be in [0, 2^20]");
+        c->fused_kc = static_cast<int>(value);
+        return MLKV_OK;
+    }
     if (std::strcmp(key, "cluster") == 0) {
         if (value != 0 && value != 1 && value != 2 && value != 4)
             return fail(MLKV_ERR_INVALID_ARG, "cluster must be 0, 1, 2 or 4");
@@ -1839,6 +2054,26 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "step_kernel") == 0) {
         *value = c->step_kernel;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "step_fused") == 0) {
+        *value = c->step_fused;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_step_fused") == 0) {
+        *value = c->last_step_fused;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_step_launches") == 0) {
+        *value = c->last_step_launches;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "last_fused_kc") == 0) {
+        *value = c->last_fused_kc;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "fused_kc") == 0) {
+        *value = c->fused_kc;
         return MLKV_OK;
     }
     if (std::strcmp(key, "last_step_kernel") == 0) {

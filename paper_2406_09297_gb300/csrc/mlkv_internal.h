@@ -93,6 +93,9 @@ struct DecodeParams {
 //   head_pairs = 1 (G even): tiles A and B are heads 2 sel and 2 sel + 1 at block qb_b.
 //   head_pairs = 0 (G odd):  both are head sel; A is block qb_b - 1 when qb_b is odd, else absent.
 constexpr int kPrefillMaxUnits = 6144;   // units per launch (more: several launches)
+// Unit word of the fused decode: sequence (10 bits), chunk (8), block (6), KV head (8).
+constexpr int kFusedMaxChunks = 256;
+constexpr int kFusedMaxBlocks = 64;
 constexpr int kPrefillMaxHeads = 256;    // sel has 8 bits
 constexpr int kPrefillMaxBlocks = 1 << 14;
 struct PrefillParams {
@@ -100,14 +103,21 @@ struct PrefillParams {
     int *err;                 // device error word
     float scale_log2;         // log2(e) / sqrt(D)
     int b, h, g, G, s_max, slot, n_units, head_pairs;
-    // Cross-layer fused decode (mlkv_decode_block_fused): the block's L layers, L1 of them in tile
-    // B (the rest in tile A); prompt_len holds the sequence lengths.  Both 0 for prefill.
-    int fused_L, fused_L1;
+    // Cross-layer fused decode (mlkv_decode_block_fused, and mlkv_decode_step's fused form): every
+    // block has L layers, L1 of them in tile B (the rest in tile A); prompt_len holds the sequence
+    // lengths.  Both 0 for prefill.  A unit's block blk (fused_nblk blocks in all) reads slot
+    // slot + blk and the layers blk*L .. blk*L + L - 1 of Q and out.
+    int fused_L, fused_L1, fused_nblk;
     // Split over the context: a unit holds key tiles [chunk*kc, chunk*kc + kc) of its sequence;
     // with more than one chunk (cmax > 1) it writes o = O/l (f32) and lse = m + log2(l) to part /
-    // part_lse [b][g][cmax][L*G rows] and combine_fused merges the chunks.
+    // part_lse [nblk][b][g][cmax][L*G rows] and combine_fused merges the chunks.
     int fused_kc, fused_cmax;
     float *part, *part_lse;
+    // 1: the previous kernel of the stream is this library's store of the new tokens, which
+    // triggers its dependents only after its own dependency wait; a unit without the sequence's
+    // last tile (the only one holding a new row) then skips the wait.
+    int fused_early;
+    int fused_combine_w;   // warps per output row of combine_fused (1, 2, 4 or 8)
     int prompt_len[MLKV_MAX_BATCH];
     uint32_t units[kPrefillMaxUnits];
 };
@@ -118,9 +128,10 @@ size_t prefill_smem_bytes(int head_dim);
 cudaError_t prepare_prefill(int head_dim);
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream);
-cudaError_t prepare_fused(int head_dim);
-cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
-                         const PrefillParams &p, cudaStream_t stream);
+// Fused decode: `one` = one query tile per CTA, two CTAs per SM (head_dim 64, L * G <= 128).
+cudaError_t prepare_fused(int head_dim, bool one);
+cudaError_t launch_fused(int head_dim, bool one, const CUtensorMap *tmap_q,
+                         const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream);
 cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream);
 
 // Copies through device-mapped page-locked host memory (mlkv_stage.cu): up to 4 segments, each a
@@ -146,10 +157,11 @@ struct MergeParams {
 cudaError_t launch_merge(const MergeParams &p, int n_slots, cudaStream_t stream);
 
 struct AppendParams {
-    const __nv_bfloat16 *K;   // [b][g][D]
+    const __nv_bfloat16 *K;   // [n_slots][b][g][D] (one slot for launch_append)
     const __nv_bfloat16 *V;
     __nv_bfloat16 *cache;     // [m][2][b][g][max_seq][D]
-    int b, g, d, max_seq, slot;
+    int b, g, d, max_seq, slot;   // K[s] and V[s] go to slot + s
+    int n_slots;
     int seq_len[MLKV_MAX_BATCH];
 };
 
@@ -227,6 +239,8 @@ constexpr int kCombineMaxPiecesHost = 1024;
 // How many k-CTA clusters of this variant can be resident at once.
 cudaError_t max_active_clusters(const DecodeVariant &v, int k, int *out);
 
+// Every owner slot's new token in one launch (mlkv_stage.cu), for the fused step.
+cudaError_t launch_append_slots(const AppendParams &p, cudaStream_t stream);
 cudaError_t launch_append(const AppendParams &p, cudaStream_t stream);
 
 }  // namespace mlkv

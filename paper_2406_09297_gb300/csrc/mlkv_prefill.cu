@@ -5,14 +5,20 @@
 // attention, Eqs. 2-3 with the MLKV maps of Eqs. 13-18).  Owner layers first store the prompt's
 // K/V in their slot (mlkv_host.cpp); every layer of the block then attends over it.
 //
-// Work unit (one CTA), head_dim 128 and the fused decode: two query tiles A and B of 128 prompt
-// positions that read the same KV head, so that every K/V tile is loaded once for both.  With an
-// even group size G they are two heads of one group at the same positions (identical causal
-// triangles); otherwise they are the blocks 2p and 2p+1 of one head (B sees one tile more; a last
-// block without a partner runs alone as B).  Prefill at head_dim 64: one query tile (as B) per CTA
-// and two CTAs per SM, each with half the tensor memory; the two CTAs' starts, first loads and
-// outputs overlap each other's key-tile loops (measured 8% faster than two tiles per CTA, although
-// every K/V tile is then fetched once per query tile).  Units that see the most keys run first.
+// Work unit (one CTA), head_dim 128: two query tiles A and B of 128 prompt positions that read the
+// same KV head, so that every K/V tile is loaded once for both.  With an even group size G they are
+// two heads of one group at the same positions (identical causal triangles); otherwise they are the
+// blocks 2p and 2p+1 of one head (B sees one tile more; a last block without a partner runs alone
+// as B).  Prefill at head_dim 64: one query tile (as B) per CTA and two CTAs per SM, each with half
+// the tensor memory; the two CTAs' starts, first loads and outputs overlap each other's key-tile
+// loops (measured 8% faster than two tiles per CTA, although every K/V tile is then fetched once
+// per query tile).  Units that see the most keys run first.
+//
+// Fused decode (one new token per sequence, every layer of an owner block at once, Sec. 3): the
+// query rows of a unit are the G heads of KV head j in each of the block's L layers, row = layer * G
+// + head, layers [0, L1) in tile B and [L1, L) in tile A (L1 = 128 / G); a unit takes one chunk of
+// the sequence's key tiles and reads each K/V tile once for all L * G rows.  At head_dim 64 with
+// L * G <= 128 the one-tile form (two CTAs per SM) runs it, otherwise the two-tile form.
 //
 // Per key tile t and query tile X (all MMAs tcgen05.mma kind::f16, bf16 in, fp32 accumulate):
 //   S_X = Q_X K_t^T  M = 128 queries (A = Q_X, K-major, 128-byte swizzle as TMA wrote it),
@@ -43,6 +49,8 @@
 // SM) and splits 56 / 200: 128 * 56 + 128 * 200 = 256 * 128.
 // Every wait is bounded; on expiry the kernel records an error bit, stops, lets its copies and MMAs
 // land and frees its TMEM.
+#include <type_traits>
+
 #include "mlkv_device.cuh"
 #include "mlkv_tcgen05.cuh"
 
@@ -109,17 +117,15 @@ __device__ __forceinline__ float max3f(float a, float b, float c)
     return d;
 }
 
-// The plan of a launch: one query tile per CTA for the head_dim 64 prefill.
-template <int D, bool kFused>
-using PlanOf = PrefillPlan<D, D == 64 && !kFused>;
-
-template <int D, bool kFused>
-__global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>::kMinBlocks)
+// kOne: one query tile per CTA (the head_dim 64 prefill; the fused decode of blocks whose rows fit
+// one tile at head_dim 64).
+template <int D, bool kFused, bool kOne>
+__global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D, kOne>::kMinBlocks)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_q,
                    const __grid_constant__ CUtensorMap tmap_kv,
                    const __grid_constant__ PrefillParams p)
 {
-    using PL = PlanOf<D, kFused>;
+    using PL = PrefillPlan<D, kOne>;
     // Query tile g's shared-memory slot and tensor-memory columns (the only tile of a one-tile CTA
     // is tile B, in slot 0).
     auto slot_of = [](int g) { return PL::kTiles == 1 ? 0 : g; };
@@ -141,14 +147,16 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     // The unit: sequence, last query block of B, head pair or head (see PrefillParams::units).
-    // Fused decode: sequence and KV head j; S is then the sequence length, every query row sees
-    // positions [0, S), and the tiles hold the block's layers [0, L1) (B) and [L1, L) (A).
+    // Fused decode: sequence, KV head j and owner block blk; S is then the sequence length, every
+    // query row sees positions [0, S), and the tiles hold the block's layers [0, L1) (B) and
+    // [L1, L) (A).
     const uint32_t u = p.units[blockIdx.x];
     const int beta = static_cast<int>(u & 0x3FFu);
     const int sel = static_cast<int>(u >> 24);
     const int S = p.prompt_len[beta];
     // Fused decode: key tiles [kt0, kt0 + n_b) of the sequence (a chunk of p.fused_kc tiles).
-    const int chunk = static_cast<int>((u >> 10) & 0x3FFFu);
+    const int chunk = static_cast<int>((u >> 10) & (kFused ? 0xFFu : 0x3FFFu));
+    const int blk = kFused ? static_cast<int>((u >> 18) & 0x3Fu) : 0;
     const int n_kt = (S + 127) / 128;
     const int kt0 = kFused ? chunk * p.fused_kc : 0;
     const int kt1 = kFused ? min(kt0 + p.fused_kc, n_kt) : 0;
@@ -161,7 +169,7 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                     : kFused ? (p.fused_L > p.fused_L1 ? n_b : 0)
                              : (p.head_pairs ? n_b : ((qb_b & 1) ? qb_b : 0));   // 0: no tile A
     const int j = kFused ? sel : head_b / p.G;                  // Eq. 15
-    const int zk = ((p.slot * 2 + 0) * p.b + beta) * p.g + j;
+    const int zk = (((p.slot + blk) * 2 + 0) * p.b + beta) * p.g + j;
     const int zv = zk + p.b * p.g;
 
     if (threadIdx.x == 0) {
@@ -210,25 +218,33 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
     __syncthreads();
     tmem_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem + PL::kFlags + 16);
-    // The owner's K/V may have just been stored by the previous kernel of the stream.
-    grid_dependency_wait();
+    // The owner's K/V may have just been stored by the previous kernel of the stream.  In the
+    // fused step that kernel stores only position L - 1 of each slot and was itself launched after
+    // every earlier kernel had finished (it triggers this launch only after its own dependency
+    // wait): the queries and every tile but the one holding position L - 1 are loaded at once, the
+    // producer waits before that tile, and the output waits before its stores.
+    const bool early = kFused && p.fused_early;
+    if (!early)
+        grid_dependency_wait();
     grid_dependents_launch();
     if (warp == PL::kProducer) {
         // ------------------------------------ producer ------------------------------------------
         setmaxnreg_dec<PL::kRegsLow>();
         if (lane == 0) {
             if (kFused) {
-                // Q [L][b][h][D] as (channel, head in group, group, sequence, layer): a box of
-                // min(L1, L) layers x G heads = the tile's rows, layer-major (row = layer*G + i).
+                // Q [layers][b][h][D] as (channel, head in group, group, sequence, layer): a box
+                // of min(L1, L) layers x G heads = the tile's rows, layer-major (row = layer*G + i),
+                // from the block's first layer (tile B) and its layer L1 (tile A).
                 const int box_rows = (p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1) * p.G;
+                const int lay0 = blk * p.fused_L;
                 mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kSub * box_rows * 128);
 #pragma unroll
                 for (int sub = 0; sub < PL::kSub; ++sub) {
                     if (n_a > 0)
                         tma_load_5d(sbase + PL::kQ + sub * 16384, &tmap_q, bar_q, sub * 64, 0, j,
-                                    beta, p.fused_L1);
-                    tma_load_5d(sbase + PL::kQ + PL::kTileBytes + sub * 16384, &tmap_q, bar_q,
-                                sub * 64, 0, j, beta, 0);
+                                    beta, lay0 + p.fused_L1);
+                    tma_load_5d(sbase + PL::kQ + slot_of(1) * PL::kTileBytes + sub * 16384,
+                                &tmap_q, bar_q, sub * 64, 0, j, beta, lay0);
                 }
             } else {
                 mbar_arrive_expect_tx(bar_q, (n_a > 0 ? 2 : 1) * PL::kTileBytes);
@@ -243,6 +259,7 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
             }
             const int n_idx = 2 * n_b;   // K_0, V_0, K_1, V_1, ...
             int idx = 0;
+            bool waited = !early;
             for (; idx < n_idx; ++idx) {
                 const int s = idx % R;
                 if (idx >= R && !flags[0] &&
@@ -252,6 +269,10 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                 }
                 if (flags[0])
                     break;
+                if (!waited && has_end && (idx >> 1) + kt0 == n_kt - 1) {
+                    grid_dependency_wait();   // the tile that holds the new row
+                    waited = true;
+                }
                 const uint32_t fb = bar_full + 8 * s;
                 mbar_arrive_expect_tx(fb, PL::kTileBytes);
                 const uint32_t dst = sbase + PL::kRing + s * PL::kTileBytes;
@@ -443,12 +464,14 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                     tmem_ld32_nowait(col_s + c * 32, sv[c]);
                 tmem_wait_ld();
                 if (diag) {
+                    // Keys [0, lim) of the tile are visible: up to the sequence's end (fused
+                    // decode) or to the query's own position (causal mask).
+                    const int lim = kFused ? S - q0 : r + 1;
 #pragma unroll
                     for (int c = 0; c < 4; ++c)
 #pragma unroll
                         for (int k = 0; k < 32; ++k)
-                            if (kFused ? q0 + c * 32 + k >= S   // past the sequence
-                                       : c * 32 + k > r)        // a later position: causal mask
+                            if (c * 32 + k >= lim)
                                 sv[c][k] = NEG_INF;
                 }
             };
@@ -573,6 +596,8 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                 mbar_arrive(p_ready);
         }
         // ---------------- the tile's output: o = O / l ----------------
+        if (early)
+            grid_dependency_wait();   // earlier kernels of the stream have finished with out
         if (n_g > 0) {
             wait(pv_done, PL::kPSep ? n_g - 1 : 0);   // with P over S only the last P V commits
             tmem_fence_after();
@@ -580,16 +605,17 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
             bool valid;
             __nv_bfloat16 *orow;
             if (kFused) {
-                // Row r: layer (grp ? 0 : L1) + r / G of the block, head j*G + r % G; out [L][b][h][D].
+                // Row r: layer (grp ? 0 : L1) + r / G of the block, head j*G + r % G; out
+                // [layers][b][h][D], the block's first layer blk * L.
                 const int L1 = p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1;
                 valid = r < (grp ? L1 : p.fused_L - p.fused_L1) * p.G;
                 const int layer = (grp ? 0 : p.fused_L1) + r / p.G;
-                orow = p.out + ((static_cast<size_t>(layer) * p.b + beta) * p.h + j * p.G +
-                                r % p.G) * D;
+                orow = p.out + ((static_cast<size_t>(blk * p.fused_L + layer) * p.b + beta) * p.h +
+                                j * p.G + r % p.G) * D;
                 if (p.fused_cmax > 1) {
                     // One chunk of the context: o = O / l and lse = m + log2(l) for the merge.
-                    const size_t row = ((static_cast<size_t>(beta) * p.g + j) * p.fused_cmax +
-                                        chunk) * (p.fused_L * p.G) +
+                    const size_t row = (((static_cast<size_t>(blk) * p.b + beta) * p.g + j) *
+                                            p.fused_cmax + chunk) * (p.fused_L * p.G) +
                                        layer * p.G + r % p.G;
                     float *prow = p.part + row * D;
                     if (valid && !flags[0])
@@ -608,6 +634,44 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
                         }
                     }
                     valid = false;   // nothing more to store for this row
+                } else {
+                    // The warp's 32 rows go through this tile's query slot (its last S has
+                    // completed), 16-byte chunks swizzled by row, and out 16 bytes a lane: the G
+                    // heads of a layer are contiguous rows of out, so the stores coalesce, which
+                    // matters most when out is page-locked host memory.
+                    uint8_t *stage = smem + PL::kQ + sg * PL::kTileBytes;
+                    constexpr int kChunks = D * 2 / 16;   // 16-byte chunks of a row
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        float ov[32];
+                        tmem_ld32_nowait(col_o + c * 32, ov);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int k = 0; k < 32; k += 8)
+                            *reinterpret_cast<uint4 *>(stage + r * (D * 2) +
+                                                       ((((c * 32 + k) >> 3) ^ (r & 7)) << 4)) =
+                                make_uint4(pack_bf16x2(ov[k] * inv, ov[k + 1] * inv),
+                                           pack_bf16x2(ov[k + 2] * inv, ov[k + 3] * inv),
+                                           pack_bf16x2(ov[k + 4] * inv, ov[k + 5] * inv),
+                                           pack_bf16x2(ov[k + 6] * inv, ov[k + 7] * inv));
+                    }
+                    __syncwarp();
+                    const int rw0 = (warp & 3) * 32;
+                    const int n_rows = (grp ? L1 : p.fused_L - p.fused_L1) * p.G;
+#pragma unroll
+                    for (int it = 0; it < kChunks; ++it) {
+                        const int cidx = it * 32 + lane;
+                        const int rr = rw0 + cidx / kChunks, ch = cidx % kChunks;
+                        if (rr < n_rows && !flags[0]) {
+                            const int lay = (grp ? 0 : p.fused_L1) + rr / p.G;
+                            __nv_bfloat16 *o =
+                                p.out + ((static_cast<size_t>(blk * p.fused_L + lay) * p.b + beta) *
+                                             p.h + j * p.G + rr % p.G) * D;
+                            *reinterpret_cast<uint4 *>(o + ch * 8) = *reinterpret_cast<const uint4 *>(
+                                stage + rr * (D * 2) + ((ch ^ (rr & 7)) << 4));
+                        }
+                    }
+                    valid = false;
                 }
             } else {
                 valid = q0 + r < S;
@@ -643,86 +707,166 @@ __global__ void __launch_bounds__(PlanOf<D, kFused>::kThreads, PlanOf<D, kFused>
     }
 }
 
-// Merges the context chunks of the fused decode: per output row (sequence, KV head, block layer,
-// group head), weights 2^(lse_c - max) over the sequence's chunks.  One warp per row.
+// Merges the context chunks of the fused decode: per output row (block, sequence, KV head, block
+// layer, group head) o = sum_c 2^(lse_c - M) o_c / sum_c 2^(lse_c - M), M = max_c lse_c.  W warps
+// per row (fused_combine_w: 1, 2, 4 or 8, more for more chunks): warp w takes chunks w, w + W, ...,
+// 4 of them in flight, and each lane keeps a running maximum, sum of weights and weighted sum for
+// its D / 32 columns; the W warps' states are then merged through shared memory.
 template <int D>
-__global__ void __launch_bounds__(256) combine_fused_kernel(const __grid_constant__ PrefillParams p)
+__global__ void __launch_bounds__(256, D == 64 ? 6 : 4) combine_fused_kernel(const __grid_constant__ PrefillParams p)
 {
-    const int rows_per_head = p.fused_L * p.G;
-    const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (row >= static_cast<long long>(p.b) * p.g * rows_per_head)
-        return;
-    const int rr = static_cast<int>(row % rows_per_head);
-    const int bj = static_cast<int>(row / rows_per_head);
-    const int beta = bj / p.g, j = bj - beta * p.g;
-    const int n_kt = (p.prompt_len[beta] + 127) / 128;
-    const int chunks = (n_kt + p.fused_kc - 1) / p.fused_kc;
-    const size_t base = static_cast<size_t>(bj) * p.fused_cmax * rows_per_head + rr;
-    float mx = -__int_as_float(0x7f800000);
-    for (int c = 0; c < chunks; ++c)
-        mx = fmaxf(mx, p.part_lse[base + static_cast<size_t>(c) * rows_per_head]);
+    // Launched while the decode grid still runs: the partials are read after it has finished.
+    grid_dependency_wait();
+    grid_dependents_launch();
     constexpr int E = D / 32;   // columns per lane
+    using Vec = typename std::conditional<E == 2, float2, float4>::type;
+    __shared__ float s_m[8], s_l[8];
+    __shared__ Vec s_acc[8][32];
+    const int W = p.fused_combine_w;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int w = warp % W;
+    const int rows_per_head = p.fused_L * p.G;
+    const long long row = static_cast<long long>(blockIdx.x) * (8 / W) + warp / W;
+    const bool live = row < static_cast<long long>(p.fused_nblk) * p.b * p.g * rows_per_head;
+    const float NEG_INF = -__int_as_float(0x7f800000);
+    int rr = 0, j = 0, beta = 0, blk = 0, chunks = 0;
+    size_t base = 0;
+    if (live) {
+        rr = static_cast<int>(row % rows_per_head);
+        const long long bj = row / rows_per_head;   // (block, sequence, KV head)
+        j = static_cast<int>(bj % p.g);
+        const long long bb = bj / p.g;
+        beta = static_cast<int>(bb % p.b);
+        blk = static_cast<int>(bb / p.b);
+        const int n_kt = (p.prompt_len[beta] + 127) / 128;
+        chunks = (n_kt + p.fused_kc - 1) / p.fused_kc;
+        base = static_cast<size_t>(bj) * p.fused_cmax * rows_per_head + rr;
+    }
+    float m = NEG_INF, l = 0.f;
     float acc[E] = {};
-    float wsum = 0.f;
-    for (int c = 0; c < chunks; ++c) {
-        const size_t r = base + static_cast<size_t>(c) * rows_per_head;
-        const float w = exp2f(p.part_lse[r] - mx);
-        wsum += w;
+    for (int c0 = w; c0 < chunks; c0 += 4 * W) {
+        float lse[4];
+        Vec v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int c = c0 + u * W;
+            const size_t r = base + static_cast<size_t>(c) * rows_per_head;
+            if (c < chunks) {
+                lse[u] = p.part_lse[r];
+                v[u] = *reinterpret_cast<const Vec *>(p.part + r * D + lane * E);
+            } else {
+                lse[u] = NEG_INF;
+                v[u] = Vec{};
+            }
+        }
+        const float mx = fmaxf(fmaxf(m, fmaxf(lse[0], lse[1])), fmaxf(lse[2], lse[3]));
+        const float scale = m == NEG_INF ? 0.f : exp2f(m - mx);
+        l *= scale;
 #pragma unroll
         for (int e = 0; e < E; ++e)
-            acc[e] += w * p.part[r * D + lane * E + e];
+            acc[e] *= scale;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const float wt = lse[u] == NEG_INF ? 0.f : exp2f(lse[u] - mx);
+            l += wt;
+            const float *x = reinterpret_cast<const float *>(&v[u]);
+#pragma unroll
+            for (int e = 0; e < E; ++e)
+                acc[e] += wt * x[e];
+        }
+        m = mx;
     }
-    const float inv = 1.f / wsum;
+    if (W > 1) {
+        if (lane == 0) {
+            s_m[warp] = m;
+            s_l[warp] = l;
+        }
+        Vec a;
+        float *ap = reinterpret_cast<float *>(&a);
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            ap[e] = acc[e];
+        s_acc[warp][lane] = a;
+        __syncthreads();
+        if (w != 0 || !live)
+            return;
+        // warp 0 of the row: every warp of the row against the largest maximum (warp 0 holds
+        // chunk 0, so M is finite)
+        float M = NEG_INF;
+        for (int k = 0; k < W; ++k)
+            M = fmaxf(M, s_m[warp + k]);
+        l = 0.f;
+#pragma unroll
+        for (int e = 0; e < E; ++e)
+            acc[e] = 0.f;
+        for (int k = 0; k < W; ++k) {
+            const float wt = s_m[warp + k] == NEG_INF ? 0.f : exp2f(s_m[warp + k] - M);
+            l += wt * s_l[warp + k];
+            const Vec b = s_acc[warp + k][lane];
+            const float *x = reinterpret_cast<const float *>(&b);
+#pragma unroll
+            for (int e = 0; e < E; ++e)
+                acc[e] += wt * x[e];
+        }
+    } else if (!live) {
+        return;
+    }
+    const float inv = 1.f / l;
     const int layer = rr / p.G, i = rr - layer * p.G;
-    __nv_bfloat16 *orow = p.out + ((static_cast<size_t>(layer) * p.b + beta) * p.h + j * p.G + i) * D;
+    __nv_bfloat16 *orow =
+        p.out + ((static_cast<size_t>(blk * p.fused_L + layer) * p.b + beta) * p.h + j * p.G + i) * D;
 #pragma unroll
     for (int e = 0; e < E; e += 2)
         *reinterpret_cast<uint32_t *>(orow + lane * E + e) =
             pack_bf16x2(acc[e] * inv, acc[e + 1] * inv);
 }
 
-template <int D, bool kFused = false>
+template <int D, bool kFused, bool kOne>
 const void *prefill_fn()
 {
-    return reinterpret_cast<const void *>(&prefill_kernel<D, kFused>);
+    return reinterpret_cast<const void *>(&prefill_kernel<D, kFused, kOne>);
 }
 
+// The forms built: prefill at head_dim 64 with one query tile per CTA, at 128 with two; the fused
+// decode with two tiles (either head_dim) or, at head_dim 64, one.
 template <typename F>
-auto plan_value(int head_dim, bool fused, F f)
+auto plan_value(int head_dim, bool one, F f)
 {
-    if (fused)
-        return head_dim == 64 ? f(PlanOf<64, true>{}) : f(PlanOf<128, true>{});
-    return head_dim == 64 ? f(PlanOf<64, false>{}) : f(PlanOf<128, false>{});
+    if (head_dim == 64)
+        return one ? f(PrefillPlan<64, true>{}) : f(PrefillPlan<64, false>{});
+    return f(PrefillPlan<128, false>{});
 }
-int threads_of(int head_dim, bool fused)
+int threads_of(int head_dim, bool one)
 {
-    return plan_value(head_dim, fused, [](auto pl) { return decltype(pl)::kThreads; });
+    return plan_value(head_dim, one, [](auto pl) { return decltype(pl)::kThreads; });
 }
-int regs_of(int head_dim, bool fused)
+int regs_of(int head_dim, bool one)
 {
-    return plan_value(head_dim, fused, [](auto pl) { return decltype(pl)::kRegsLaunch; });
+    return plan_value(head_dim, one, [](auto pl) { return decltype(pl)::kRegsLaunch; });
 }
-size_t smem_of(int head_dim, bool fused)
+size_t smem_of(int head_dim, bool one)
 {
-    return plan_value(head_dim, fused,
+    return plan_value(head_dim, one,
                       [](auto pl) { return static_cast<size_t>(decltype(pl)::kAlloc); });
 }
 
-const void *kernel_fn(int head_dim, bool fused)
+const void *kernel_fn(int head_dim, bool fused, bool one)
 {
-    if (fused)
-        return head_dim == 64 ? prefill_fn<64, true>() : prefill_fn<128, true>();
-    return head_dim == 64 ? prefill_fn<64>() : prefill_fn<128>();
+    if (fused) {
+        if (head_dim == 64)
+            return one ? prefill_fn<64, true, true>() : prefill_fn<64, true, false>();
+        return prefill_fn<128, true, false>();
+    }
+    return head_dim == 64 ? prefill_fn<64, false, true>() : prefill_fn<128, false, false>();
 }
 
-cudaError_t launch(int head_dim, bool fused, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
-                   const PrefillParams &p, cudaStream_t stream)
+cudaError_t launch(int head_dim, bool fused, bool one, const CUtensorMap *tmap_q,
+                   const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
-    cfg.blockDim = dim3(static_cast<unsigned>(threads_of(head_dim, fused)));
-    cfg.dynamicSmemBytes = smem_of(head_dim, fused);
+    cfg.blockDim = dim3(static_cast<unsigned>(threads_of(head_dim, one)));
+    cfg.dynamicSmemBytes = smem_of(head_dim, one);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -731,54 +875,65 @@ cudaError_t launch(int head_dim, bool fused, const CUtensorMap *tmap_q, const CU
     cfg.numAttrs = 1;
     void *args[] = {const_cast<CUtensorMap *>(tmap_q), const_cast<CUtensorMap *>(tmap_kv),
                     const_cast<PrefillParams *>(&p)};
-    return cudaLaunchKernelExC(&cfg, kernel_fn(head_dim, fused), args);
+    return cudaLaunchKernelExC(&cfg, kernel_fn(head_dim, fused, one), args);
 }
+
+// The prefill form of a head_dim.
+bool prefill_one(int head_dim) { return head_dim == 64; }
 
 }  // namespace
 
-size_t prefill_smem_bytes(int head_dim) { return smem_of(head_dim, false); }
+size_t prefill_smem_bytes(int head_dim) { return smem_of(head_dim, prefill_one(head_dim)); }
 
 // The warpgroups' register split (setmaxnreg) adds up to the registers the block is launched with;
 // a kernel built with another per-thread count would wait forever in setmaxnreg.inc, so it is
 // refused here instead of launched.
-cudaError_t prepare(int head_dim, bool fused)
+cudaError_t prepare(int head_dim, bool fused, bool one)
 {
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, kernel_fn(head_dim, fused));
+    const void *fn = kernel_fn(head_dim, fused, one);
+    cudaError_t e = cudaFuncGetAttributes(&fa, fn);
     if (e != cudaSuccess)
         return e;
-    if (fa.numRegs != regs_of(head_dim, fused))
+    if (fa.numRegs != regs_of(head_dim, one))
         return cudaErrorInvalidKernelImage;
-    return cudaFuncSetAttribute(kernel_fn(head_dim, fused),
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(smem_of(head_dim, fused)));
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(smem_of(head_dim, one)));
 }
 
-cudaError_t prepare_prefill(int head_dim) { return prepare(head_dim, false); }
+cudaError_t prepare_prefill(int head_dim) { return prepare(head_dim, false, prefill_one(head_dim)); }
 
-cudaError_t prepare_fused(int head_dim) { return prepare(head_dim, true); }
+cudaError_t prepare_fused(int head_dim, bool one) { return prepare(head_dim, true, one); }
 
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream)
 {
-    return launch(head_dim, false, tmap_q, tmap_kv, p, stream);
+    return launch(head_dim, false, prefill_one(head_dim), tmap_q, tmap_kv, p, stream);
 }
 
-cudaError_t launch_fused(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
-                         const PrefillParams &p, cudaStream_t stream)
+cudaError_t launch_fused(int head_dim, bool one, const CUtensorMap *tmap_q,
+                         const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream)
 {
-    return launch(head_dim, true, tmap_q, tmap_kv, p, stream);
+    return launch(head_dim, true, one && head_dim == 64, tmap_q, tmap_kv, p, stream);
 }
 
 cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream)
 {
-    const long long rows = static_cast<long long>(p.b) * p.g * p.fused_L * p.G;
-    const unsigned blocks = static_cast<unsigned>((rows + 7) / 8);
-    if (head_dim == 64)
-        combine_fused_kernel<64><<<blocks, 256, 0, stream>>>(p);
-    else
-        combine_fused_kernel<128><<<blocks, 256, 0, stream>>>(p);
-    return cudaGetLastError();
+    const long long rows = static_cast<long long>(p.fused_nblk) * p.b * p.g * p.fused_L * p.G;
+    const int per_cta = 8 / p.fused_combine_w;   // rows of a CTA
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>((rows + per_cta - 1) / per_cta));
+    cfg.blockDim = dim3(256);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void *args[] = {const_cast<PrefillParams *>(&p)};
+    const void *fn = head_dim == 64 ? reinterpret_cast<const void *>(&combine_fused_kernel<64>)
+                                    : reinterpret_cast<const void *>(&combine_fused_kernel<128>);
+    return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
 }  // namespace mlkv

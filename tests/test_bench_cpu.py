@@ -57,13 +57,17 @@ def test_recorded_traffic_needs_current_kernel_and_launch_kind():
     from mlkv_synth import workloads
     with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
         rec = json.load(f)
-    for name, entry in rec.items():
-        assert entry["launch"] in ("multi-layer", "per-layer")
+    forms = ("multi-layer", "fused", "per-layer")
+    for entry in rec["entries"]:
+        assert entry["launch"] in forms
         assert entry["dram_bytes_per_launch"] > 0
-        w = workloads.by_name(name)
-        current = entry["kernel_source_sha256_16"] == bench._kernel_source_hash()
+        w = workloads.by_name(entry["workload"])
+        current = entry["kernel_source_sha256_16"] == bench._kernel_source_hash(entry["kernel"])
         got = bench._recorded_traffic(w, entry["kernel"], entry["launch"])
         assert got == (entry["dram_bytes_per_launch"] if current else None)
-        other = "per-layer" if entry["launch"] == "multi-layer" else "multi-layer"
-        assert bench._recorded_traffic(w, entry["kernel"], other) is None
+        for other in forms:
+            if other != entry["launch"] and not any(
+                    e["workload"] == entry["workload"] and e["launch"] == other
+                    for e in rec["entries"]):
+                assert bench._recorded_traffic(w, entry["kernel"], other) is None
         assert bench._recorded_traffic(w, "no_such_kernel", entry["launch"]) is None

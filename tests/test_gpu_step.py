@@ -27,6 +27,16 @@ def _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref):
     return qb, kn, vn
 
 
+def _fused_applies(owner, h, g):
+    """Maps the step can run in the cross-layer fused form (option step_fused 2 forces it there):
+    equal contiguous owner blocks whose L * G query rows fit two tiles of 128."""
+    l, m = len(owner), len(set(owner))
+    L, G = l // m, h // g
+    return (L * m == l and all(owner[n] == n - n % L for n in range(l)) and
+            128 // G >= 1 and L <= 2 * (128 // G))
+
+
+@pytest.mark.parametrize("fused", [2, 0])
 @pytest.mark.parametrize("owner,h,g,d,b,lens,max_seq", [
     ([0, 0, 2, 2, 2, 5], 12, 2, 64, 5, [1, 300, 1000, 77, 640], 1024),
     ([0, 0, 0, 0], 12, 1, 64, 64, [2048] * 64, 2048),            # whole segments per CTA
@@ -35,7 +45,7 @@ def _inputs(owner, h, g, d, b, lens, max_seq, seed, cache, ref):
     ([0] * 6 + [6] * 6, 12, 1, 64, 64, [1024] * 64, 1024),
     ([0, 0, 2], 16, 4, 128, 3, [5000, 20, 4096], 5000),
 ])
-def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
+def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq, fused):
     import torch
 
     import paper_2406_09297_gb300 as mlkv
@@ -50,11 +60,13 @@ def test_step_matches_oracle_and_layer_calls(owner, h, g, d, b, lens, max_seq):
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.full((l, b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
         cache.set_option("step_graph", 1)   # always through the recorded graph
+        cache.set_option("step_fused", fused)
         for rep in range(4):   # direct, record, then replay twice
             out.fill_(float("nan"))
             cache.decode_step(Q, K, V, out, lens)
         torch.cuda.synchronize()
         assert cache.get_option("step_graph_replays") == 3
+        assert cache.get_option("last_step_fused") == int(fused > 0 and _fused_applies(owner, h, g))
         # the same layer calls one by one on a second cache
         owners = sorted(set(owner))
         out2 = torch.full_like(out, float("nan"))
@@ -232,6 +244,7 @@ def test_step_single_long_segment(step_kernel):
     lens = np.full(b, L, dtype=np.int32)
     with mlkv.MLKVCache(len(owner), h, d, owner, g, b, L) as cache:
         cache.set_option("step_kernel", step_kernel)
+        cache.set_option("step_fused", 0)   # the decode kernel's launch shapes
         ref = oracle.OracleCache(owner, h, g, d, b, L)
         qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 61, cache, ref)
         out = torch.full((len(owner), b, h, d), float("nan"), dtype=torch.bfloat16, device="cuda")
@@ -309,6 +322,7 @@ def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
         cache.set_option("step_graph", 1)   # always through the recorded graph
+        cache.set_option("step_fused", 0)   # the decode kernel's multi-layer launch
         results = []
         for rep in range(3):   # direct, record, replay
             out.fill_(float("nan"))
@@ -316,6 +330,7 @@ def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
             torch.cuda.synchronize()
             results.append(out.clone())
             assert cache.get_option("last_step_kernel") == 1
+            assert cache.get_option("last_step_fused") == 0
             assert cache.get_option("last_grid") == grid
         assert cache.get_option("step_graph_replays") == 2
         for r in results[1:]:
@@ -337,13 +352,14 @@ def test_multi_layer_step_kernel(owner, h, g, d, b, L, grid):
 
 
 
+@pytest.mark.parametrize("fused", [2, 0])
 @pytest.mark.parametrize("owner,h,g,d,lens", [
     # varied lengths: segments sorted longest first and dealt in a snake round-robin
     ([0, 0, 0, 3, 3, 3], 12, 4, 64, [1, 127, 128, 129, 3000, 64, 700, 2048, 5, 1999] * 4),
     ([0, 0, 2, 2], 32, 8, 128, [300, 1, 1500, 900, 64, 65, 1024, 777]),
     ([0, 1, 1, 3], 12, 1, 64, [int(x) for x in np.random.default_rng(7).integers(1, 4097, 96)]),
 ])
-def test_multi_layer_step_varied_lengths(owner, h, g, d, lens):
+def test_multi_layer_step_varied_lengths(owner, h, g, d, lens, fused):
     import torch
 
     import paper_2406_09297_gb300 as mlkv
@@ -355,6 +371,7 @@ def test_multi_layer_step_varied_lengths(owner, h, g, d, lens):
         qb, kn, vn = _inputs(owner, h, g, d, b, lens, max_seq, 91, cache, ref)
         Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
         out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        cache.set_option("step_fused", fused)
         results = []
         for rep in range(3):   # direct, record, replay
             out.fill_(float("nan"))
@@ -362,6 +379,8 @@ def test_multi_layer_step_varied_lengths(owner, h, g, d, lens):
             torch.cuda.synchronize()
             results.append(out.clone())
             assert cache.get_option("last_step_kernel") == 1
+            assert cache.get_option("last_step_fused") == int(fused > 0 and
+                                                               _fused_applies(owner, h, g))
         for r in results[1:]:
             assert torch.equal(r.view(torch.int16), results[0].view(torch.int16))
         for n in range(l):
@@ -371,4 +390,69 @@ def test_multi_layer_step_varied_lengths(owner, h, g, d, lens):
             expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
             mx, mean = errors(from_dev(results[0][n]), expect)
             assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
+
+
+@pytest.mark.parametrize("owner,h,g,d,b,L,kc,units", [
+    ([0] * 6 + [6] * 6, 12, 1, 64, 64, 2048, 16, 128),  # the benchmark's shape: 72 rows a unit
+    ([0, 0, 2, 2, 4, 4, 6, 6, 8, 8, 10, 10], 12, 1, 64, 1, 128, 1, 6),   # one tile per block
+    ([0] * 12, 12, 1, 64, 4, 3000, 1, 96),              # 144 rows: query tiles A and B
+    ([0, 0, 2, 2], 12, 1, 64, 40, 700, 6, 80),           # ragged last tile
+    ([0, 0, 2, 2], 4, 4, 64, 8, 333, 2, 128),            # one head per KV head: two rows a unit
+    ([0, 0, 0, 3, 3, 3], 12, 4, 64, 16, 1000, 8, 128),   # GQA groups of 3 under MLKV: 9 rows
+    ([0, 0, 2, 2], 32, 8, 128, 8, 1500, 12, 128),        # head_dim 128, groups of 4: 8 rows
+    ([0] * 20, 16, 2, 128, 2, 600, 1, 20),               # head_dim 128, 160 rows in two tiles
+    ([0, 0, 0], 16, 2, 64, 3, 1, 1, 6),                  # a single position
+    # few long segments: every segment in chunks, partial records, one merge launch
+    ([0] * 6 + [6] * 6, 12, 1, 64, 1, 131072, 14, 148),  # 74 chunks of 14 tiles a segment
+    ([0, 0, 2, 2], 12, 4, 64, 2, 9000, 8, 144),          # ragged last tile in the last chunk
+    ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 27, 144),       # head_dim 128
+    ([0, 1, 2, 3], 12, 1, 64, 3, 5000, 4, 120),          # blocks of one layer (forced)
+])
+def test_fused_step(owner, h, g, d, b, L, kc, units):
+    # The step in the cross-layer fused form (forced: option step_fused 2): one launch storing
+    # every owner's new token, then units of (sequence, KV head, owner block, chunk of the
+    # context), each loading every K/V tile of its chunk once for the L * G query rows of its
+    # block's layers, the context split only as far as the units fit one per SM (152), and a
+    # merge launch when a segment has several chunks.  Every output of every layer against the
+    # oracle; the new tokens in the cache; the recorded graph's replay bit for bit.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    lens = np.full(b, L, dtype=np.int32)
+    l = len(owner)
+    owners = sorted(set(owner))
+    with mlkv.MLKVCache(l, h, d, owner, g, b, L) as cache:
+        ref = oracle.OracleCache(owner, h, g, d, b, L)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 83, cache, ref)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        cache.set_option("step_graph", 1)   # direct, record, replay
+        cache.set_option("step_fused", 2)   # wherever the map allows it
+        results = []
+        for rep in range(3):
+            out.fill_(float("nan"))
+            cache.decode_step(Q, K, V, out, lens)
+            torch.cuda.synchronize()
+            results.append(out.clone())
+            assert cache.get_option("last_step_fused") == 1
+            assert cache.get_option("last_fused_kc") == kc
+            assert cache.get_option("last_grid") == units
+            assert cache.get_option("last_deferred_merge") == int(kc < (L + 127) // 128)
+            assert cache.get_option("last_step_launches") == 2 + int(kc < (L + 127) // 128)
+        assert cache.get_option("step_graph_replays") == 2
+        for r in results[1:]:
+            assert torch.equal(r.view(torch.int16), results[0].view(torch.int16))
+        for n in range(l):
+            if owner[n] == n:
+                k = owners.index(n)
+                ref.append(n, gen.bf16_bits_to_f64(kn[k]), gen.bf16_bits_to_f64(vn[k]), lens)
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
+            mx, mean = errors(from_dev(results[0][n]), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        from tests.test_gpu_cache import _read_cache
+        whole = _read_cache(cache, b, g, L, d)          # int16 [m][2][b][g][L][d]
+        for k, n in enumerate(owners):
+            assert (whole[cache.owner_slot(n)[1], 0, :, :, L - 1] == kn[k].view(np.int16)).all()
+            assert (whole[cache.owner_slot(n)[1], 1, :, :, L - 1] == vn[k].view(np.int16)).all()
         cache.sync_status()

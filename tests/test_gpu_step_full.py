@@ -110,6 +110,8 @@ def check_step_full_size(w, n_betas=4, seed=0, options=None, host_buffers=False)
             direct = (cache.get_option("step_graph") == 2 and
                       cache.get_option("last_step_kernel") == 1)
             assert cache.get_option("step_graph_replays") == (0 if direct else 2)
+        fused = cache.get_option("last_step_fused")
+        sm_count = cache.get_option("sm_count")
         cache.sync_status()
         worst = 0.0
         for own in w.owners():
@@ -127,12 +129,20 @@ def check_step_full_size(w, n_betas=4, seed=0, options=None, host_buffers=False)
                         mx, mean = errors(got, expect)
                         assert mx <= MAX_ABS and mean <= MEAN_ABS, (w.name, n, beta, j, mx, mean)
                         worst = max(worst, mx)
-        return worst
+        return worst, fused, sm_count
+
+
+# Which benchmark configurations run the step in the cross-layer fused form by default (blocks of
+# >= 3 layers where its cost estimate beats the decode kernel's): MLKV-2 b64, GQA-4 + MLKV-4 b128
+# and the Llama-2-7B shapes do; the batch-1 MLKV-6 map of pairs does not.
+FUSED_BY_DEFAULT = {1: 0, 2: 1, 3: 1, 4: 1}
 
 
 @pytest.mark.parametrize("index", [1, 2, 3, 4])
 def test_step_config_full_size(index):
-    check_step_full_size(workloads.config(index), seed=index)
+    w = workloads.config(index)
+    _, fused, _ = check_step_full_size(w, seed=index)
+    assert fused == FUSED_BY_DEFAULT[index]
 
 
 @pytest.mark.parametrize("name", [w.name for w in workloads.sweep(False)])
@@ -154,13 +164,15 @@ def test_step_host_buffers_config2_full_size():
 @pytest.mark.parametrize("options", [{"l2_prefetch": 0}, {"l2_persist": 1}, {"step_kernel": 0},
                                      {"step_graph": 1}, {"step_kernel": 0, "early_fetch": 0},
                                      {"step_kernel": 0, "early_fetch": 2},
-                                     {"step_kernel": 0, "pdl": 0}])
+                                     {"step_kernel": 0, "pdl": 0}, {"step_fused": 0},
+                                     {"step_fused": 0, "step_graph": 1}])
 def test_step_options_full_size(options):
     """Options that change where bytes come from or how the step is launched, never the result:
     the default workload and the varied-length GQA workload (slots larger than L2) with the L2
-    prefetch off, with L2 persistence on, with per-layer launches instead of one multi-layer
-    launch (overlapping; with no read, or only the first cache tile, before the previous layer's
-    end; in plain stream order), and with the multi-layer launch replayed from a recorded graph."""
+    prefetch off, with L2 persistence on, with per-layer launches instead of one multi-layer launch (overlapping; with
+    no read, or only the first cache tile, before the previous layer's end; in plain stream
+    order), with the multi-layer decode launch instead of the fused form, and with the step
+    replayed from a recorded graph."""
     import paper_2406_09297_gb300 as mlkv
     for index in (2, 3):
         try:
