@@ -261,6 +261,10 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *   "fused_kc"     > 0 = key tiles of 128 positions per unit of the fused form (clamped to what
  *                  the unit word holds); 0 (default) = planned: a sequence is split only as far
  *                  as the units still number at most the SMs.
+ *   "fused_deep"   1 (default) = a fused launch at head_dim 64 whose blocks' rows fit one 128-row
+ *                  tile and whose units number at most the SMs runs one CTA per SM with a
+ *                  12-tile K/V ring and two S buffers in tensor memory; 0 = two CTAs per SM with a
+ *                  5-tile ring.  Same results.
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through

@@ -125,7 +125,8 @@ struct mlkv_cache {
     int early_fetch = 1;        // per-layer step: later layers read Q and tiles before the wait
     int tc = 0;                 // 1: the tcgen05 kernel where a variant exists (slower here)
     int prefill_ready = 0;      // the prefill kernel's shared-memory limit is set
-    int fused_ready = 0;        // the same for the fused-decode forms (bit 1: two tiles, 2: one)
+    int fused_ready = 0;        // the same for the fused-decode forms (bit 1 << form)
+    int fused_deep = 1;         // fused decode: the deep one-tile form where one unit per SM
     float *fused_part = nullptr;   // context-chunk partials of the fused decode
     size_t fused_part_floats = 0;
     int step_fused = 1;         // mlkv_decode_step: the cross-layer fused form where it pays (1),
@@ -801,13 +802,20 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
                        bool after_store = false)
 {
     const int L1 = 128 / c->G;
-    const bool one = c->d == 64 && L <= L1;   // one query tile per CTA, two CTAs per SM
-    const int form = one ? 2 : 1;
+    // The CTA form: one query tile when the block's rows fit one (head_dim 64); then with at most
+    // one unit per SM one CTA per SM with a deep ring and two S buffers (its tiles come from HBM
+    // one after another), else two CTAs per SM.  Rows past one tile: two query tiles.
+    long long n_units = 0;
+    const int kc = fused_plan(c, seq_lens, nblk, &n_units);
+    const bool one = c->d == 64 && L <= L1;
+    const int form = !one ? mlkv::kFusedTwoTiles
+                          : (n_units <= c->sm_count && c->fused_deep ? mlkv::kFusedOneDeep
+                                                                     : mlkv::kFusedOneTile);
     cudaError_t e;
-    if (!(c->fused_ready & form)) {
-        if ((e = mlkv::prepare_fused(c->d, one)) != cudaSuccess)
+    if (!(c->fused_ready & (1 << form))) {
+        if ((e = mlkv::prepare_fused(c->d, form)) != cudaSuccess)
             return fail_cuda(e, "cudaFuncSetAttribute(fused decode)");
-        c->fused_ready |= form;
+        c->fused_ready |= 1 << form;
     }
     static EncodeTiledFn encode = driver_entry<EncodeTiledFn>("cuTensorMapEncodeTiled");
     if (encode == nullptr)
@@ -864,7 +872,6 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
         kt_sum += nkt;
         uniform = uniform && seq_lens[beta] == seq_lens[0];
     }
-    const int kc = fused_plan(c, seq_lens, nblk, nullptr);
     (void)kt_sum;
     const int cmax = (n_kt_max + kc - 1) / kc;
     p.fused_kc = kc;
@@ -910,7 +917,7 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
                     ++total_units;
                     if (++n == mlkv::kPrefillMaxUnits) {
                         p.n_units = n;
-                        if ((e = mlkv::launch_fused(c->d, one, &tmap_q, tmap_kv, p, stream)) !=
+                        if ((e = mlkv::launch_fused(c->d, form, &tmap_q, tmap_kv, p, stream)) !=
                             cudaSuccess)
                             return fail_cuda(e, "fused decode launch");
                         ++*launches;
@@ -919,7 +926,7 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
                 }
     if (n > 0) {
         p.n_units = n;
-        if ((e = mlkv::launch_fused(c->d, one, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
+        if ((e = mlkv::launch_fused(c->d, form, &tmap_q, tmap_kv, p, stream)) != cudaSuccess)
             return fail_cuda(e, "fused decode launch");
         ++*launches;
     }
@@ -1985,6 +1992,12 @@ int mlkv_set_option(mlkv_cache_t c, const char *key, int64_t value)
         c->step_fused = static_cast<int>(value);
         return MLKV_OK;
     }
+    if (std::strcmp(key, "fused_deep") == 0) {
+        if (value != 0 && value != 1)
+            return fail(MLKV_ERR_INVALID_ARG, "fused_deep must be 0 or 1");
+        c->fused_deep = static_cast<int>(value);
+        return MLKV_OK;
+    }
     if (std::strcmp(key, "fused_kc") == 0) {
         if (value < 0 || value > (1 << 20))
             return fail(MLKV_ERR_INVALID_ARG, "fused_kc must be in [0, 2^20]");
@@ -2074,6 +2087,10 @@ int mlkv_get_option(mlkv_cache_t c, const char *key, int64_t *value)
     }
     if (std::strcmp(key, "fused_kc") == 0) {
         *value = c->fused_kc;
+        return MLKV_OK;
+    }
+    if (std::strcmp(key, "fused_deep") == 0) {
+        *value = c->fused_deep;
         return MLKV_OK;
     }
     if (std::strcmp(key, "last_step_kernel") == 0) {

@@ -128,9 +128,12 @@ size_t prefill_smem_bytes(int head_dim);
 cudaError_t prepare_prefill(int head_dim);
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream);
-// Fused decode: `one` = one query tile per CTA, two CTAs per SM (head_dim 64, L * G <= 128).
-cudaError_t prepare_fused(int head_dim, bool one);
-cudaError_t launch_fused(int head_dim, bool one, const CUtensorMap *tmap_q,
+// Fused decode forms (head_dim 64 with L * G <= 128 may take either one-tile form; otherwise the
+// two-tile form is used whatever is asked): 0 two query tiles per CTA; 1 one tile, two CTAs per
+// SM; 2 one tile, one CTA per SM with a 12-tile ring and two S buffers.
+constexpr int kFusedTwoTiles = 0, kFusedOneTile = 1, kFusedOneDeep = 2;
+cudaError_t prepare_fused(int head_dim, int form);
+cudaError_t launch_fused(int head_dim, int form, const CUtensorMap *tmap_q,
                          const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream);
 cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream);
 

@@ -57,45 +57,64 @@
 namespace mlkv {
 namespace {
 
-// kOne: one query tile per CTA and two CTAs per SM (prefill at head_dim 64): each CTA holds half
-// the tensor memory and a third of the registers of the two-tile form, and two independent CTAs
-// hide each other's start, first loads and output; the key tiles are fetched once per query tile.
-// Otherwise two query tiles per CTA share every K/V tile, one CTA per SM.
-template <int D, bool kOne>
+// Forms of the CTA (kForm):
+//   kTwoTiles  two query tiles share every K/V tile, one CTA per SM (head_dim 128; the fused
+//              decode of blocks whose rows exceed one tile);
+//   kOneTile   one query tile per CTA and two CTAs per SM (prefill at head_dim 64; the fused
+//              decode with more units than SMs): each CTA holds half the tensor memory and a third
+//              of the registers of the two-tile form, and two independent CTAs hide each other's
+//              start, first loads and output;
+//   kOneDeep   one query tile, one CTA per SM (the fused decode with at most one unit per SM, its
+//              K/V tiles streamed from HBM): a ring of 12 tiles keeps ~6 K/V pairs in flight, and
+//              the key tiles alternate between two softmax warpgroups on the same 128 query rows,
+//              each with its own S, P and O columns and its own running maximum and sum, merged
+//              per row at the end -- two key tiles' softmax chains run at once, and S of the next
+//              tile is computed while this one's softmax runs.
+constexpr int kTwoTiles = 0, kOneTile = 1, kOneDeep = 2;
+
+template <int D, int kForm>
 struct PrefillPlan {
+    static constexpr bool kOne = kForm != kTwoTiles;
     static constexpr int kTiles = kOne ? 1 : 2;              // query tiles per CTA
-    static constexpr int kSoftWarps = 4 * kTiles;
+    static constexpr int kSBuf = kForm == kOneDeep ? 2 : 1;  // S, P and O buffers per query tile
+    static constexpr int kSoftWarps = 4 * kTiles * kSBuf;    // a warpgroup per tile or buffer
     static constexpr int kThreads = (kSoftWarps + 4) * 32;
-    static constexpr int kMinBlocks = kOne ? 2 : 1;
-    static constexpr int kRegsLaunch = kOne ? 128 : 168;
-    static constexpr int kRegsLow = kOne ? 56 : (D == 64 ? 72 : 88);
-    static constexpr int kRegsHigh = kOne ? 200 : (D == 64 ? 216 : 208);
+    static constexpr int kMinBlocks = kForm == kOneTile ? 2 : 1;
+    // registers at launch, then the other warps' share and the softmax warps' (setmaxnreg)
+    static constexpr int kRegsLaunch = kForm == kOneTile ? 128 : 168;
+    static constexpr int kRegsLow = kForm == kOneTile ? 56 : (D == 64 ? 72 : 88);
+    static constexpr int kRegsHigh = kForm == kOneTile ? 200 : (D == 64 ? 216 : 208);
     static constexpr int kProducer = kSoftWarps, kMma = kSoftWarps + 1;
     static constexpr int kSub = D / 64;                      // 64-channel blocks of a row
     static constexpr int kTileBytes = 128 * D * 2;           // 128 rows of Q, K or V
-    static constexpr int kRingTiles = kOne ? 5 : (D == 64 ? 8 : 4);   // K_t and V_t alternate
+    // K_t and V_t alternate in the ring
+    static constexpr int kRingTiles = kForm == kOneDeep ? 12 : kOne ? 5 : (D == 64 ? 8 : 4);
     static constexpr int kQ = 0;                             // [kTiles] query tiles
     static constexpr int kRing = kQ + kTiles * kTileBytes;
     static constexpr int kFlags = kRing + kRingTiles * kTileBytes;   // int [4], TMEM base at +16
     // u64 barriers: q, full[R], empty[R], s_ready[2], s_free[2], p_ready[2], pv_done[2], fin[2]
+    // (s_ready and s_free per query tile, or per S buffer in the deep form)
     static constexpr int kBars = kFlags + 32;
     static constexpr int kNumBars = 1 + 2 * kRingTiles + 8 + 2;
-    static constexpr int kBytes = kBars + kNumBars * 8;
+    // the second warpgroup's running maximum and sum per row, for the merge (two buffers)
+    static constexpr int kML = kBars + kNumBars * 8;
+    static constexpr int kBytes = kML + (kSBuf == 2 ? 128 * 8 : 0);
     static constexpr int kAlloc = kBytes + 1024;             // base aligned up to 1024
     static_assert(kMinBlocks * (kAlloc + 1024) <= 228 * 1024, "shared memory of the resident CTAs");
-    static constexpr int kTmemCols = kOne ? 256 : 512;
+    static constexpr int kTmemCols = kForm == kOneTile ? 256 : 512;
     static constexpr bool kPSep = D == 64;                   // P in columns of its own
-    static constexpr int kColS = 0;                          // + 128 per query tile
-    static constexpr int kColO = 128 * kTiles;               // + D per query tile
-    static constexpr int kColP = kColO + D * kTiles;         // + 64 per query tile (kPSep)
+    static constexpr int kColS = 0;                          // + 128 per query tile or buffer
+    static constexpr int kColO = 128 * kTiles * kSBuf;       // + D per query tile or buffer
+    static constexpr int kColP = kColO + D * kTiles * kSBuf; // + 64 per tile or buffer (kPSep)
     static_assert(D == 64 || D == 128, "head_dim 64 or 128");
     static_assert(!kOne || D == 64, "one query tile per CTA only at head_dim 64");
     static_assert(kRing % 1024 == 0 && kTileBytes % 1024 == 0, "swizzled tiles 1024-aligned");
-    static_assert((kPSep ? kColP + 64 * kTiles : kColO + D * kTiles) <= kTmemCols,
+    static_assert((kPSep ? kColP + 64 * kTiles * kSBuf : kColO + D * kTiles) <= kTmemCols,
                   "TMEM columns overlap");
     static_assert(128 * kRegsLow + 32 * kSoftWarps * kRegsHigh <= kThreads * kRegsLaunch,
                   "register split");
     static_assert(kMinBlocks * kThreads * kRegsLaunch <= 65536, "registers of the resident CTAs");
+    static_assert(kSBuf == 1 || (kTiles == 1 && kPSep), "two buffers: one tile, P apart");
 };
 
 template <int N>
@@ -117,15 +136,15 @@ __device__ __forceinline__ float max3f(float a, float b, float c)
     return d;
 }
 
-// kOne: one query tile per CTA (the head_dim 64 prefill; the fused decode of blocks whose rows fit
-// one tile at head_dim 64).
-template <int D, bool kFused, bool kOne>
-__global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D, kOne>::kMinBlocks)
+template <int D, bool kFused, int kForm>
+__global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
+                                  PrefillPlan<D, kForm>::kMinBlocks)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_q,
                    const __grid_constant__ CUtensorMap tmap_kv,
                    const __grid_constant__ PrefillParams p)
 {
-    using PL = PrefillPlan<D, kOne>;
+    using PL = PrefillPlan<D, kForm>;
+    constexpr bool kSplit = PL::kSBuf == 2;   // key tiles alternate between two warpgroups
     // Query tile g's shared-memory slot and tensor-memory columns (the only tile of a one-tile CTA
     // is tile B, in slot 0).
     auto slot_of = [](int g) { return PL::kTiles == 1 ? 0 : g; };
@@ -203,10 +222,10 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
     if (kFused && warp < PL::kSoftWarps) {
         // The tiles' rows past the TMA box (box_rows = G x min(L1, L)) are never loaded; zero them
         // so that their (discarded) scores stay finite.  TMA writes only rows below box_rows.
-        const int grp = warp >> 2, r = threadIdx.x & 127;
+        const int grp = PL::kTiles == 1 ? 1 : warp >> 2, r = threadIdx.x & 127;
         const int box_rows = (p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1) * p.G;
-        if (r >= box_rows) {
-            uint8_t *qrow = smem + PL::kQ + grp * PL::kTileBytes;
+        if (r >= box_rows && warp < 4 * PL::kTiles) {   // one warpgroup per query tile
+            uint8_t *qrow = smem + PL::kQ + slot_of(grp) * PL::kTileBytes;
 #pragma unroll
             for (int c = 0; c < 8 * PL::kSub; ++c)
                 *reinterpret_cast<uint4 *>(qrow + (c >> 3) * 16384 + r * 128 +
@@ -333,26 +352,29 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
             auto issue_s = [&](int g, int t) {
                 const uint64_t qa = dq + slot_of(g) * kSlot;
                 const uint64_t kb = dk + ((2 * t) % R) * kSlot;
+                const int sb = kSplit ? (t & 1) : g;   // S buffer and its barrier
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
                     const uint32_t off = (k >> 2) * 1024 + (k & 3) * 2;   // 16384 B, 32 B
-                    umma_f16(tmem + PL::kColS + 128 * slot_of(g), qa + off, kb + off, kIdS,
-                             k > 0 ? 1 : 0);
+                    umma_f16(tmem + PL::kColS + 128 * (kSplit ? sb : slot_of(g)), qa + off,
+                             kb + off, kIdS, k > 0 ? 1 : 0);
                 }
-                umma_commit(bar_s_ready + 8 * g);
+                umma_commit(bar_s_ready + 8 * sb);
             };
             auto issue_pv = [&](int g, int t, bool last) {
                 const uint64_t vb = dv + ((2 * t + 1) % R) * kSlot;
                 const int sg = slot_of(g);
+                const int ob = kSplit ? (t & 1) : sg;   // P and O buffer (warpgroup t mod 2)
                 const uint32_t pc =
-                    tmem + (PL::kPSep ? PL::kColP + 64 * sg : PL::kColS + 128 * sg);
+                    tmem + (PL::kPSep ? PL::kColP + 64 * ob : PL::kColS + 128 * sg);
+                const bool first = kSplit ? t < 2 : t == 0;   // the buffer's first product
 #pragma unroll
                 for (int k = 0; k < 8; ++k)   // 16 keys = 2048 B of V, 8 TMEM columns of P
-                    umma_f16_ts(tmem + PL::kColO + D * sg, pc + 8 * k, vb + k * 128, kIdPV,
-                                (t > 0 || k > 0) ? 1 : 0);
+                    umma_f16_ts(tmem + PL::kColO + D * ob, pc + 8 * k, vb + k * 128, kIdPV,
+                                (!first || k > 0) ? 1 : 0);
                 // With P over S, the next S's completion already implies this product's.
                 if (PL::kPSep || last)
-                    umma_commit(bar_pv_done + 8 * g);
+                    umma_commit(bar_pv_done + 8 * (kSplit ? (t & 1) : g));
             };
             if (do_s && wait(bar_q, 0) && tile_full(0)) {
                 tmem_fence_after();
@@ -371,7 +393,12 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
                         const int ng = g ? n_b : n_a;
                         if (!do_s || !ok || t + 1 >= ng)
                             continue;
-                        if (!wait(bar_s_free + 8 * g, t) || !tile_full(2 * t + 2))
+                        // S(t + 1) once its columns are free: tile t's S read (one buffer), or
+                        // tile t - 1's (two buffers: S(t + 1) then runs during tile t's softmax)
+                        if (kSplit ? (t >= 1 && !wait(bar_s_free + 8 * ((t + 1) & 1), (t - 1) >> 1))
+                                   : !wait(bar_s_free + 8 * g, t))
+                            break;
+                        if (!tile_full(2 * t + 2))
                             break;
                         tmem_fence_after();
                         issue_s(g, t + 1);
@@ -381,7 +408,8 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
                         const int ng = g ? n_b : n_a;
                         if (!do_pv || !ok || t >= ng)
                             continue;
-                        if (!tile_full(2 * t + 1) || !wait(bar_p_ready + 8 * g, t))
+                        if (!tile_full(2 * t + 1) ||
+                            !wait(bar_p_ready + 8 * (kSplit ? (t & 1) : g), kSplit ? (t >> 1) : t))
                             break;
                         tmem_fence_after();
                         issue_pv(g, t, t + 1 >= ng);
@@ -425,12 +453,18 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
         const int head = grp ? head_b : head_a;
         const int q0 = (kt0 + n_g - 1) * 128;       // first position of the unit's last tile
         const int sg = slot_of(grp);
-        const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * sg;
-        const uint32_t col_o = tmem + lane_off + PL::kColO + D * sg;
+        // the warpgroup's buffer: the tile's own, or (split keys) this warpgroup's tiles t = wg,
+        // wg + 2, ... with S, P and O buffer wg
+        const int wg = kSplit ? warp >> 2 : 0;
+        const int bsel = kSplit ? wg : grp;
+        const uint32_t col_s = tmem + lane_off + PL::kColS + 128 * (kSplit ? wg : sg);
+        const uint32_t col_o = tmem + lane_off + PL::kColO + D * (kSplit ? wg : sg);
         const uint32_t col_p =
-            tmem + lane_off + (PL::kPSep ? PL::kColP + 64 * sg : PL::kColS + 128 * sg);
-        const uint32_t s_ready = bar_s_ready + 8 * grp, s_free = bar_s_free + 8 * grp;
-        const uint32_t p_ready = bar_p_ready + 8 * grp, pv_done = bar_pv_done + 8 * grp;
+            tmem + lane_off +
+            (PL::kPSep ? PL::kColP + 64 * (kSplit ? wg : sg) : PL::kColS + 128 * sg);
+        const uint32_t s_ready = bar_s_ready + 8 * bsel, s_free = bar_s_free + 8 * bsel;
+        const uint32_t p_ready = bar_p_ready + 8 * bsel, pv_done = bar_pv_done + 8 * bsel;
+        constexpr int kStep = kSplit ? 2 : 1;   // tiles between this warpgroup's
         // The prompt's last block holds keys past its end; the first tile to reach it zeroes them.
         const bool zero_v = n_g > 0 && (kFused ? has_end : n_g == (S + 127) / 128) &&
                             (grp == 0 || n_a != n_b);
@@ -443,13 +477,15 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
             }
         };
         float m_run = NEG_INF, l_run = 0.f;
-        for (int t = 0; t < n_g; ++t) {
-            wait(s_ready, t);
-            // Tile B's first warp frees ring slots whose readers have all completed: K_0 once S_B(0)
-            // is done; V_{t-1} and K_t once S_B(t) (P over S) or P_B V_{t-1} (own P) is done.
+        for (int t = wg; t < n_g; t += kStep) {
+            const int u = kSplit ? t >> 1 : t;   // this warpgroup's use of its buffers
+            wait(s_ready, u);
+            // Tile B's first warp frees ring slots whose readers have all completed: K_t once S_B(t)
+            // is done (S_A(t) was issued before it by the same thread); V_{t-1} once S_B(t) (P over
+            // S: issued after P V_{t-1}) or P_B V_{t-1} (own P) is done.
             const bool releaser = grp == 1 && (warp & 3) == 0 && lane == 0;
-            if (releaser && t == 0)
-                mbar_arrive(bar_empty);
+            if (releaser && (t == 0 || PL::kPSep))   // K_t
+                mbar_arrive(bar_empty + 8 * ((2 * t) % R));
             if (releaser && t > 0 && !PL::kPSep) {
                 mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
                 mbar_arrive(bar_empty + 8 * ((2 * t) % R));
@@ -495,10 +531,10 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
                 if (__any_sync(0xffffffffu, raise)) {
                     const float m_new = raise ? fmaxf(m_run, m_tile) : m_run;
                     const float alpha = fast_exp2(m_run - m_new);   // 0 while nothing is summed
-                    if (t > 0) {
+                    if (u > 0) {
                         // Rescale this row of O once the previous tile's product has landed.
                         if (PL::kPSep)
-                            wait(pv_done, t - 1);
+                            wait(pv_done, u - 1);
                         tmem_fence_after();
 #pragma unroll
                         for (int c = 0; c < D / 32; ++c) {
@@ -565,12 +601,10 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
             }
             // The P buffer of the previous tile must have been read by its P V; the weights above
             // were computed while that product ran.
-            if (PL::kPSep && t > 0) {
-                wait(pv_done, t - 1);
-                if (releaser) {
-                    mbar_arrive(bar_empty + 8 * ((2 * t - 1) % R));
-                    mbar_arrive(bar_empty + 8 * ((2 * t) % R));
-                }
+            if (PL::kPSep && u > 0) {
+                wait(pv_done, u - 1);
+                if (releaser)   // V of this warpgroup's previous tile
+                    mbar_arrive(bar_empty + 8 * ((2 * (t - kStep) + 1) % R));
             }
             tmem_fence_after();
             tmem_st32_nowait(col_p, w[0]);
@@ -598,8 +632,47 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
         // ---------------- the tile's output: o = O / l ----------------
         if (early)
             grid_dependency_wait();   // earlier kernels of the stream have finished with out
-        if (n_g > 0) {
-            wait(pv_done, PL::kPSep ? n_g - 1 : 0);   // with P over S only the last P V commits
+        // Split keys: the second warpgroup hands its running maximum and sum to the first, which
+        // merges the two O buffers row by row (O = O_0 2^(m_0 - M) + O_1 2^(m_1 - M), likewise l).
+        const int n_mine = kSplit ? (n_g - wg + 1) / 2 : n_g;   // this warpgroup's tiles
+        float a0 = 1.f, a1 = 0.f;
+        if (kSplit) {
+            if (n_mine > 0)
+                wait(pv_done, n_mine - 1);
+            float2 *ml = reinterpret_cast<float2 *>(smem + PL::kML);
+            if (wg == 1)
+                ml[r] = make_float2(m_run, l_run);
+            asm volatile("bar.sync 1, %0;" ::"n"(8 * 32) : "memory");
+            if (wg == 1)
+                m_run = NEG_INF;   // done: nothing to store
+            else {
+                const float2 o1 = ml[r];
+                if (o1.y > 0.f) {
+                    const float mx = fmaxf(m_run, o1.x);
+                    a0 = fast_exp2(m_run - mx);
+                    a1 = fast_exp2(o1.x - mx);
+                    l_run = l_run * a0 + o1.y * a1;
+                    m_run = mx;
+                }
+            }
+        }
+        // O of this row, 32 columns at c: this warpgroup's buffer, merged with the second's
+        auto load_o = [&](int c, float (&ov)[32]) {
+            tmem_ld32_nowait(col_o + c * 32, ov);
+            if (kSplit && a1 > 0.f) {
+                float o1[32];
+                tmem_ld32_nowait(col_o + D + c * 32, o1);
+                tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 32; ++k)
+                    ov[k] = ov[k] * a0 + o1[k] * a1;
+            } else {
+                tmem_wait_ld();
+            }
+        };
+        if (n_g > 0 && wg == 0) {
+            if (!kSplit)
+                wait(pv_done, PL::kPSep ? n_g - 1 : 0);   // with P over S only the last P V commits
             tmem_fence_after();
             const float inv = fast_rcp(l_run);
             bool valid;
@@ -623,8 +696,7 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         float ov[32];
-                        tmem_ld32_nowait(col_o + c * 32, ov);
-                        tmem_wait_ld();
+                        load_o(c, ov);
                         if (valid && !flags[0]) {
 #pragma unroll
                             for (int k = 0; k < 32; k += 4)
@@ -644,8 +716,7 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         float ov[32];
-                        tmem_ld32_nowait(col_o + c * 32, ov);
-                        tmem_wait_ld();
+                        load_o(c, ov);
 #pragma unroll
                         for (int k = 0; k < 32; k += 8)
                             *reinterpret_cast<uint4 *>(stage + r * (D * 2) +
@@ -678,7 +749,7 @@ __global__ void __launch_bounds__(PrefillPlan<D, kOne>::kThreads, PrefillPlan<D,
                 orow = p.out + ((static_cast<size_t>(beta) * p.s_max + (q0 + r)) * p.h + head) * D;
             }
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
+            for (int c = 0; c < (kFused ? 0 : D / 32); ++c) {   // the prefill's rows
                 float ov[32];
                 tmem_ld32_nowait(col_o + c * 32, ov);
                 tmem_wait_ld();
@@ -821,52 +892,57 @@ __global__ void __launch_bounds__(256, D == 64 ? 6 : 4) combine_fused_kernel(con
             pack_bf16x2(acc[e] * inv, acc[e + 1] * inv);
 }
 
-template <int D, bool kFused, bool kOne>
+template <int D, bool kFused, int kForm>
 const void *prefill_fn()
 {
-    return reinterpret_cast<const void *>(&prefill_kernel<D, kFused, kOne>);
+    return reinterpret_cast<const void *>(&prefill_kernel<D, kFused, kForm>);
 }
 
 // The forms built: prefill at head_dim 64 with one query tile per CTA, at 128 with two; the fused
-// decode with two tiles (either head_dim) or, at head_dim 64, one.
+// decode in the two-tile form (either head_dim) or, at head_dim 64, either one-tile form.
 template <typename F>
-auto plan_value(int head_dim, bool one, F f)
+auto plan_value(int head_dim, int form, F f)
 {
-    if (head_dim == 64)
-        return one ? f(PrefillPlan<64, true>{}) : f(PrefillPlan<64, false>{});
-    return f(PrefillPlan<128, false>{});
+    if (head_dim == 64) {
+        if (form == kOneDeep)
+            return f(PrefillPlan<64, kOneDeep>{});
+        return form == kOneTile ? f(PrefillPlan<64, kOneTile>{}) : f(PrefillPlan<64, kTwoTiles>{});
+    }
+    return f(PrefillPlan<128, kTwoTiles>{});
 }
-int threads_of(int head_dim, bool one)
+int threads_of(int head_dim, int form)
 {
-    return plan_value(head_dim, one, [](auto pl) { return decltype(pl)::kThreads; });
+    return plan_value(head_dim, form, [](auto pl) { return decltype(pl)::kThreads; });
 }
-int regs_of(int head_dim, bool one)
+int regs_of(int head_dim, int form)
 {
-    return plan_value(head_dim, one, [](auto pl) { return decltype(pl)::kRegsLaunch; });
+    return plan_value(head_dim, form, [](auto pl) { return decltype(pl)::kRegsLaunch; });
 }
-size_t smem_of(int head_dim, bool one)
+size_t smem_of(int head_dim, int form)
 {
-    return plan_value(head_dim, one,
+    return plan_value(head_dim, form,
                       [](auto pl) { return static_cast<size_t>(decltype(pl)::kAlloc); });
 }
 
-const void *kernel_fn(int head_dim, bool fused, bool one)
+const void *kernel_fn(int head_dim, bool fused, int form)
 {
     if (fused) {
         if (head_dim == 64)
-            return one ? prefill_fn<64, true, true>() : prefill_fn<64, true, false>();
-        return prefill_fn<128, true, false>();
+            return form == kOneDeep   ? prefill_fn<64, true, kOneDeep>()
+                   : form == kOneTile ? prefill_fn<64, true, kOneTile>()
+                                      : prefill_fn<64, true, kTwoTiles>();
+        return prefill_fn<128, true, kTwoTiles>();
     }
-    return head_dim == 64 ? prefill_fn<64, false, true>() : prefill_fn<128, false, false>();
+    return head_dim == 64 ? prefill_fn<64, false, kOneTile>() : prefill_fn<128, false, kTwoTiles>();
 }
 
-cudaError_t launch(int head_dim, bool fused, bool one, const CUtensorMap *tmap_q,
+cudaError_t launch(int head_dim, bool fused, int form, const CUtensorMap *tmap_q,
                    const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_units));
-    cfg.blockDim = dim3(static_cast<unsigned>(threads_of(head_dim, one)));
-    cfg.dynamicSmemBytes = smem_of(head_dim, one);
+    cfg.blockDim = dim3(static_cast<unsigned>(threads_of(head_dim, form)));
+    cfg.dynamicSmemBytes = smem_of(head_dim, form);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -875,46 +951,53 @@ cudaError_t launch(int head_dim, bool fused, bool one, const CUtensorMap *tmap_q
     cfg.numAttrs = 1;
     void *args[] = {const_cast<CUtensorMap *>(tmap_q), const_cast<CUtensorMap *>(tmap_kv),
                     const_cast<PrefillParams *>(&p)};
-    return cudaLaunchKernelExC(&cfg, kernel_fn(head_dim, fused, one), args);
+    return cudaLaunchKernelExC(&cfg, kernel_fn(head_dim, fused, form), args);
 }
 
-// The prefill form of a head_dim.
-bool prefill_one(int head_dim) { return head_dim == 64; }
+// The prefill form of a head_dim; a fused-decode form valid for the head_dim.
+int prefill_form(int head_dim) { return head_dim == 64 ? kOneTile : kTwoTiles; }
+int fused_form(int head_dim, int form) { return head_dim == 64 ? form : kTwoTiles; }
 
 }  // namespace
 
-size_t prefill_smem_bytes(int head_dim) { return smem_of(head_dim, prefill_one(head_dim)); }
+size_t prefill_smem_bytes(int head_dim) { return smem_of(head_dim, prefill_form(head_dim)); }
 
 // The warpgroups' register split (setmaxnreg) adds up to the registers the block is launched with;
 // a kernel built with another per-thread count would wait forever in setmaxnreg.inc, so it is
 // refused here instead of launched.
-cudaError_t prepare(int head_dim, bool fused, bool one)
+cudaError_t prepare(int head_dim, bool fused, int form)
 {
     cudaFuncAttributes fa;
-    const void *fn = kernel_fn(head_dim, fused, one);
+    const void *fn = kernel_fn(head_dim, fused, form);
     cudaError_t e = cudaFuncGetAttributes(&fa, fn);
     if (e != cudaSuccess)
         return e;
-    if (fa.numRegs != regs_of(head_dim, one))
+    if (fa.numRegs != regs_of(head_dim, form))
         return cudaErrorInvalidKernelImage;
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(smem_of(head_dim, one)));
+                                static_cast<int>(smem_of(head_dim, form)));
 }
 
-cudaError_t prepare_prefill(int head_dim) { return prepare(head_dim, false, prefill_one(head_dim)); }
+cudaError_t prepare_prefill(int head_dim)
+{
+    return prepare(head_dim, false, prefill_form(head_dim));
+}
 
-cudaError_t prepare_fused(int head_dim, bool one) { return prepare(head_dim, true, one); }
+cudaError_t prepare_fused(int head_dim, int form)
+{
+    return prepare(head_dim, true, fused_form(head_dim, form));
+}
 
 cudaError_t launch_prefill(int head_dim, const CUtensorMap *tmap_q, const CUtensorMap *tmap_kv,
                            const PrefillParams &p, cudaStream_t stream)
 {
-    return launch(head_dim, false, prefill_one(head_dim), tmap_q, tmap_kv, p, stream);
+    return launch(head_dim, false, prefill_form(head_dim), tmap_q, tmap_kv, p, stream);
 }
 
-cudaError_t launch_fused(int head_dim, bool one, const CUtensorMap *tmap_q,
+cudaError_t launch_fused(int head_dim, int form, const CUtensorMap *tmap_q,
                          const CUtensorMap *tmap_kv, const PrefillParams &p, cudaStream_t stream)
 {
-    return launch(head_dim, true, one && head_dim == 64, tmap_q, tmap_kv, p, stream);
+    return launch(head_dim, true, fused_form(head_dim, form), tmap_q, tmap_kv, p, stream);
 }
 
 cudaError_t launch_fused_combine(int head_dim, const PrefillParams &p, cudaStream_t stream)

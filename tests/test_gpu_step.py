@@ -409,7 +409,8 @@ def test_multi_layer_step_varied_lengths(owner, h, g, d, lens, fused):
     ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 27, 144),       # head_dim 128
     ([0, 1, 2, 3], 12, 1, 64, 3, 5000, 4, 120),          # blocks of one layer (forced)
 ])
-def test_fused_step(owner, h, g, d, b, L, kc, units):
+@pytest.mark.parametrize("deep", [1, 0])
+def test_fused_step(owner, h, g, d, b, L, kc, units, deep):
     # The step in the cross-layer fused form (forced: option step_fused 2): one launch storing
     # every owner's new token, then units of (sequence, KV head, owner block, chunk of the
     # context), each loading every K/V tile of its chunk once for the L * G query rows of its
@@ -429,6 +430,9 @@ def test_fused_step(owner, h, g, d, b, L, kc, units):
         out = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
         cache.set_option("step_graph", 1)   # direct, record, replay
         cache.set_option("step_fused", 2)   # wherever the map allows it
+        # head_dim 64 with the block's rows in one tile: one CTA per SM with a 12-tile ring and two
+        # S buffers when the units fit one per SM (deep), else two CTAs per SM
+        cache.set_option("fused_deep", deep)
         results = []
         for rep in range(3):
             out.fill_(float("nan"))
