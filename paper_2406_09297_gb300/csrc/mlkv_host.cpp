@@ -471,6 +471,7 @@ int mlkv_append(mlkv_cache_t c, int layer, const void *K, const void *V, const i
     p.max_seq = c->max_seq;
     p.slot = c->slot[layer];
     p.n_slots = 1;
+    p.trigger_first = 0;
     std::memcpy(p.seq_len, seq_lens, sizeof(int) * c->b);
     DeviceGuard guard(c->device);
     cudaError_t e = mlkv::launch_append(p, static_cast<cudaStream_t>(cuda_stream));
@@ -799,7 +800,7 @@ static int fused_plan(const mlkv_cache *c, const int *seq_lens, int nblk, long l
 // added to *launches.
 static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers, int L, int nblk,
                        int slot0, const int *seq_lens, cudaStream_t stream, int *launches,
-                       bool after_store = false)
+                       int after_store = 0)
 {
     const int L1 = 128 / c->G;
     // The CTA form: one query tile when the block's rows fit one (head_dim 64); then with at most
@@ -861,7 +862,7 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
     p.fused_L = L;
     p.fused_L1 = L1;
     p.fused_nblk = nblk;
-    p.fused_early = after_store ? 1 : 0;
+    p.fused_early = after_store;
     int n_kt_max = 0;
     long long kt_sum = 0;
     bool uniform = true;
@@ -1022,11 +1023,16 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
     ap.max_seq = c->max_seq;
     ap.slot = 0;
     ap.n_slots = c->m;
+    // After this library's input copy (host buffers) the fused launch goes at once and fetches
+    // cache tiles while the copy runs; otherwise it follows the store's dependency wait and also
+    // fetches the queries at once.
+    ap.trigger_first = stage != nullptr ? 1 : 0;
     std::memcpy(ap.seq_len, seq_lens, sizeof(int) * c->b);
     if ((e = mlkv::launch_append_slots(ap, s)) != cudaSuccess)
         return fail_cuda(e, "append launch (fused step)");
     ++launches;
-    const int rc = fused_issue(c, Q, out, c->l, L, c->m, 0, seq_lens, s, &launches, true);
+    const int rc = fused_issue(c, Q, out, c->l, L, c->m, 0, seq_lens, s, &launches,
+                               stage != nullptr ? 2 : 1);
     if (rc != MLKV_OK)
         return rc;
     c->last_cluster_k = 0;

@@ -113,9 +113,11 @@ struct PrefillParams {
     // part_lse [nblk][b][g][cmax][L*G rows] and combine_fused merges the chunks.
     int fused_kc, fused_cmax;
     float *part, *part_lse;
-    // 1: the previous kernel of the stream is this library's store of the new tokens, which
-    // triggers its dependents only after its own dependency wait; a unit without the sequence's
-    // last tile (the only one holding a new row) then skips the wait.
+    // What the fused launch may read before its dependency wait (the previous kernel of the
+    // stream is this library's store of the new tokens): 1 -- the store triggered this launch
+    // after its own wait, so everything but the tile holding the new row (the queries too);
+    // 2 -- the store triggered it at once (the step's inputs still being copied in), so only
+    // cache tiles that hold no new row; 0 -- nothing.
     int fused_early;
     int fused_combine_w;   // warps per output row of combine_fused (1, 2, 4 or 8)
     int prompt_len[MLKV_MAX_BATCH];
@@ -165,6 +167,7 @@ struct AppendParams {
     __nv_bfloat16 *cache;     // [m][2][b][g][max_seq][D]
     int b, g, d, max_seq, slot;   // K[s] and V[s] go to slot + s
     int n_slots;
+    int trigger_first;            // append_slots: trigger the dependent launch before the wait
     int seq_len[MLKV_MAX_BATCH];
 };
 

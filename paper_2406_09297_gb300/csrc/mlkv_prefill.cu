@@ -243,6 +243,7 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
     // wait): the queries and every tile but the one holding position L - 1 are loaded at once, the
     // producer waits before that tile, and the output waits before its stores.
     const bool early = kFused && p.fused_early;
+    const bool q_early = kFused && p.fused_early == 1;   // the queries before the wait too
     if (!early)
         grid_dependency_wait();
     grid_dependents_launch();
@@ -250,6 +251,26 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
         // ------------------------------------ producer ------------------------------------------
         setmaxnreg_dec<PL::kRegsLow>();
         if (lane == 0) {
+            bool waited = !early;
+            // mode 2: the cache tiles that hold no new row first, as far as the ring goes
+            int idx_pre = 0;
+            if (early && !q_early) {
+                const int n_pre = 2 * n_b < R ? 2 * n_b : R;
+                for (; idx_pre < n_pre; ++idx_pre) {
+                    if (has_end && (idx_pre >> 1) + kt0 == n_kt - 1)
+                        break;
+                    const uint32_t fb = bar_full + 8 * idx_pre;
+                    mbar_arrive_expect_tx(fb, PL::kTileBytes);
+                    const uint32_t dst = sbase + PL::kRing + idx_pre * PL::kTileBytes;
+                    const int z = (idx_pre & 1) ? zv : zk;
+#pragma unroll
+                    for (int sub = 0; sub < PL::kSub; ++sub)
+                        tma_load_3d(dst + sub * 16384, &tmap_kv, fb, sub * 64,
+                                    ((idx_pre >> 1) + kt0) * 128, z);
+                }
+                grid_dependency_wait();   // the step's inputs are in place
+                waited = true;
+            }
             if (kFused) {
                 // Q [layers][b][h][D] as (channel, head in group, group, sequence, layer): a box
                 // of min(L1, L) layers x G heads = the tile's rows, layer-major (row = layer*G + i),
@@ -277,8 +298,7 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
                 }
             }
             const int n_idx = 2 * n_b;   // K_0, V_0, K_1, V_1, ...
-            int idx = 0;
-            bool waited = !early;
+            int idx = idx_pre;
             for (; idx < n_idx; ++idx) {
                 const int s = idx % R;
                 if (idx >= R && !flags[0] &&

@@ -35,8 +35,13 @@ __global__ void __launch_bounds__(256) stage_copy_kernel(const __grid_constant__
 __global__ void __launch_bounds__(256) append_slots_kernel(const __grid_constant__ AppendParams p)
 {
     // Earlier kernels of the stream may still read the cache: nothing is stored before they end.
+    // The dependent (the fused decode) is let go after that wait, or at once when it is told to
+    // read only what no kernel in flight writes (trigger_first).
+    if (p.trigger_first)
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (!p.trigger_first)
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int vecs = p.d / 8;
     const long long total = 2LL * p.n_slots * p.b * p.g * vecs;
     const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;

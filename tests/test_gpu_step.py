@@ -460,3 +460,46 @@ def test_fused_step(owner, h, g, d, b, L, kc, units, deep):
             assert (whole[cache.owner_slot(n)[1], 0, :, :, L - 1] == kn[k].view(np.int16)).all()
             assert (whole[cache.owner_slot(n)[1], 1, :, :, L - 1] == vn[k].view(np.int16)).all()
         cache.sync_status()
+
+
+@pytest.mark.parametrize("chunked", [False, True])
+def test_fused_step_host_buffers(chunked):
+    # mlkv_decode_step_host in the fused form: the store launch lets the fused launch go at once,
+    # which fetches cache tiles while the step's inputs are still being copied in and waits before
+    # the queries and the newest tile; its results equal the device-buffer step's bit for bit.
+    import torch
+
+    import paper_2406_09297_gb300 as mlkv
+    owner, h, g, d = [0] * 6 + [6] * 6, 12, 1, 64
+    b, L = (1, 20000) if chunked else (16, 1000)
+    lens = np.full(b, L, dtype=np.int32)
+    l = len(owner)
+    with mlkv.MLKVCache(l, h, d, owner, g, b, L) as cache, \
+            mlkv.MLKVCache(l, h, d, owner, g, b, L) as cache2:
+        ref = oracle.OracleCache(owner, h, g, d, b, L)
+        qb, kn, vn = _inputs(owner, h, g, d, b, lens, L, 89, cache, ref)
+        _inputs(owner, h, g, d, b, lens, L, 89, cache2, None)
+        for c in (cache, cache2):
+            c.set_option("step_fused", 2)
+        Q, K, V = to_dev(qb), to_dev(kn), to_dev(vn)
+        want = torch.empty((l, b, h, d), dtype=torch.bfloat16, device="cuda")
+        cache2.decode_step(Q, K, V, want, lens)
+        torch.cuda.synchronize()
+        hq, hk, hv = Q.cpu().pin_memory(), K.cpu().pin_memory(), V.cpu().pin_memory()
+        out = torch.full((l, b, h, d), float("nan"), dtype=torch.bfloat16).pin_memory()
+        for _ in range(3):
+            out.fill_(float("nan"))
+            cache.decode_step_host(hq, hk, hv, out, lens)
+            torch.cuda.synchronize()
+            assert cache.get_option("last_step_fused") == 1
+            assert torch.equal(out.view(torch.int16), want.cpu().view(torch.int16))
+        owners = sorted(set(owner))
+        for n in range(l):
+            if owner[n] == n:
+                k = owners.index(n)
+                ref.append(n, gen.bf16_bits_to_f64(kn[k]), gen.bf16_bits_to_f64(vn[k]), lens)
+            expect = ref.decode(n, gen.bf16_bits_to_f64(qb[n]), lens, nthreads=8)
+            mx, mean = errors(out[n].float().numpy().astype(np.float64), expect)
+            assert mx <= MAX_ABS and mean <= MEAN_ABS, (n, mx, mean)
+        cache.sync_status()
+        cache2.sync_status()
