@@ -494,6 +494,11 @@ def run(args, w):
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind,
                          "frac_vs_8tbs": achieved / 8000.0,
+                         # achieved counts every layer's K/V (the per-layer reads the paper's
+                         # implementation makes): "effective" once layers share a slot, since the
+                         # step moves each owner slot from DRAM once (dram_frac_step; traffic)
+                         "achieved_bytes": "logical K/V + Q + out of every layer (effective "
+                                           "where layers share a slot)",
                          "kernel": kernel_name, "step_form": form,
                          "alg_bytes_per_launch": launch_bytes,
                          "mean_launch_ms": launch_ms, "launches_per_step": launches_per_step,
