@@ -237,12 +237,18 @@ KERNEL_SOURCES = {
 
 
 def _kernel_source_hash(kernel="decode_kernel"):
-    """sha256[:16] over a kernel's sources, in KERNEL_SOURCES order."""
+    """sha256[:16] over a kernel's sources, in KERNEL_SOURCES order, with comments, trailing
+    blanks and empty lines removed (so that a capture stays valid while only comments change)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for name in KERNEL_SOURCES[kernel]:
-        with open(os.path.join(ROOT, "paper_2406_09297_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2406_09297_gb300", "csrc", name)) as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        lines = [ln.rstrip() for ln in text.splitlines()]
+        h.update("\n".join(ln for ln in lines if ln).encode())
     return h.hexdigest()[:16]
 
 

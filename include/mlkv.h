@@ -263,8 +263,9 @@ int mlkv_kv_ptr(mlkv_cache_t c, int slot, void **k_base, void **v_base, int64_t 
  *                  as the units still number at most the SMs.
  *   "fused_deep"   1 (default) = a fused launch at head_dim 64 whose blocks' rows fit one 128-row
  *                  tile and whose units number at most the SMs runs one CTA per SM with a
- *                  12-tile K/V ring and two S buffers in tensor memory; 0 = two CTAs per SM with a
- *                  5-tile ring.  Same results.
+ *                  12-tile K/V ring, its key tiles alternating between two softmax warpgroups
+ *                  (S, P and O in two buffers of tensor memory, merged per row at the end); 0 =
+ *                  two CTAs per SM with a 5-tile ring.  Same results within the tolerance.
  *   "cluster"      1 (default) = when every sequence has one length and each (sequence, KV head)
  *                  splits into 2 or 4 equal pieces without lengthening the one-wave makespan,
  *                  run the pieces of a segment as one thread-block cluster and merge them through

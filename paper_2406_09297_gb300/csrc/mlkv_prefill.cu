@@ -18,7 +18,9 @@
 // query rows of a unit are the G heads of KV head j in each of the block's L layers, row = layer * G
 // + head, layers [0, L1) in tile B and [L1, L) in tile A (L1 = 128 / G); a unit takes one chunk of
 // the sequence's key tiles and reads each K/V tile once for all L * G rows.  At head_dim 64 with
-// L * G <= 128 the one-tile form (two CTAs per SM) runs it, otherwise the two-tile form.
+// L * G <= 128 a one-tile form runs it: with at most one unit per SM the deep form (one CTA per SM,
+// a 12-tile ring, key tiles alternating between two softmax warpgroups), else two CTAs per SM;
+// otherwise the two-tile form.
 //
 // Per key tile t and query tile X (all MMAs tcgen05.mma kind::f16, bf16 in, fp32 accumulate):
 //   S_X = Q_X K_t^T  M = 128 queries (A = Q_X, K-major, 128-byte swizzle as TMA wrote it),
