@@ -161,16 +161,19 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
 
 /*
  * mlkv_decode_step_host - mlkv_decode_step with the step's tensors in host memory (the user's end
- * of a step): Q, K and V are copied to device staging buffers held by the cache, the step runs on
- * them and every layer's output is copied back to out, all queued on cuda_stream with one
- * cudaMemcpyAsync per tensor.  Layouts as for mlkv_decode_step, in host memory.
- * With page-locked buffers (cudaHostAlloc, cudaHostRegister) and option "step_graph" = 1 the copies
- * and the launches of a step are recorded into one CUDA graph the second time the same arguments
- * come and replayed after (as for mlkv_decode_step; with 2, the default, a one-launch step and
- * its input copy are issued directly); pageable buffers run directly, and their
- * copies synchronise with the host as CUDA's pageable copies do.  out holds the step's outputs
- * once the stream has reached the end of the call's work.  The staging buffers, 2 * (l*b*h*d +
- * m*b*g*d) bf16, are allocated on the first call and kept until mlkv_cache_destroy.
+ * of a step).  Layouts as for mlkv_decode_step, in host memory; everything is queued on
+ * cuda_stream, and out holds the step's outputs once the stream has reached the end of the call's
+ * work.
+ * Page-locked, 16-byte-aligned buffers (cudaHostAlloc, cudaHostRegister) are used through their
+ * device-mapped addresses: in the cross-layer fused form the kernels read the queries and the new
+ * tokens and write the outputs there directly (no copy); otherwise one copy kernel brings Q, K and
+ * V into device staging buffers right before the launch and the kernels write the outputs in
+ * place.  With option "step_graph" = 1 the launches of a step are recorded into one CUDA graph the
+ * second time the same arguments come and replayed after (as for mlkv_decode_step; with 2, the
+ * default, a one-launch or fused step is issued directly).  Other buffers take one
+ * cudaMemcpyAsync per tensor, in and out, and synchronise with the host as CUDA's pageable copies
+ * do.  The staging buffers, 2 * (l*b*h*d + m*b*g*d) bf16, are allocated on the first call and
+ * kept until mlkv_cache_destroy.
  * Errors: as mlkv_decode_step, and MLKV_ERR_OOM for the staging buffers.
  */
 int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,

@@ -800,7 +800,7 @@ static int fused_plan(const mlkv_cache *c, const int *seq_lens, int nblk, long l
 // added to *launches.
 static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers, int L, int nblk,
                        int slot0, const int *seq_lens, cudaStream_t stream, int *launches,
-                       int after_store = 0)
+                       int after_store = 0, bool q_in_host = false)
 {
     const int L1 = 128 / c->G;
     // The CTA form: one query tile when the block's rows fit one (head_dim 64); then with at most
@@ -863,6 +863,8 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
     p.fused_L1 = L1;
     p.fused_nblk = nblk;
     p.fused_early = after_store;
+    // queries in page-locked host memory (Q is its device-mapped address): read row by row
+    p.q_host = q_in_host ? static_cast<const __nv_bfloat16 *>(Q) : nullptr;
     int n_kt_max = 0;
     long long kt_sum = 0;
     bool uniform = true;
@@ -949,7 +951,7 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
 // two 128-row tiles; otherwise *done stays false.
 static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
                             const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
-                            const mlkv::StageParams *stage)
+                            const mlkv::StageParams *stage, bool host_inputs = false)
 {
     *done = false;
     if (!c->step_fused || c->tile_tokens > 0 || c->l2_prefetch || c->m > mlkv::kFusedMaxBlocks ||
@@ -1031,8 +1033,10 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
     if ((e = mlkv::launch_append_slots(ap, s)) != cudaSuccess)
         return fail_cuda(e, "append launch (fused step)");
     ++launches;
+    // With the inputs in page-locked host memory (host_inputs: Q, K, V and out are device-mapped
+    // addresses) the store reads the new tokens and the fused units their query rows from there.
     const int rc = fused_issue(c, Q, out, c->l, L, c->m, 0, seq_lens, s, &launches,
-                               stage != nullptr ? 2 : 1);
+                               stage != nullptr ? 2 : 1, host_inputs);
     if (rc != MLKV_OK)
         return rc;
     c->last_cluster_k = 0;
@@ -1048,7 +1052,7 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
 
 static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
                          const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
-                         const mlkv::StageParams *stage = nullptr)
+                         const mlkv::StageParams *stage = nullptr, bool host_inputs = false)
 {
     *done = false;
     c->last_step_kernel = 0;
@@ -1057,9 +1061,10 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     if (!c->step_kernel || c->tc || c->grid > 0 || c->l2_persist || c->l > mlkv::kMaxStepLayers)
         return MLKV_OK;
     {
-        const int rc = issue_step_fused(c, Q, K, V, out, seq_lens, stream, in_ready, done, stage);
-        if (rc != MLKV_OK || *done)
-            return rc;
+        const int rc =
+            issue_step_fused(c, Q, K, V, out, seq_lens, stream, in_ready, done, stage, host_inputs);
+        if (rc != MLKV_OK || *done || host_inputs)
+            return rc;   // host inputs: only the fused form reads them where they are
     }
     bool uniform = true;
     long long len_sum = 0;
@@ -1543,6 +1548,15 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
     }
     auto issue = [&](cudaStream_t s) {
         if (mapped) {
+            // The fused form reads the inputs where they are: no copy.
+            bool direct = false;
+            int r0 = issue_step_ml(c, static_cast<const char *>(dev[0]),
+                                   static_cast<const char *>(dev[1]),
+                                   static_cast<const char *>(dev[2]),
+                                   static_cast<char *>(const_cast<void *>(dev[3])), seq_lens, s,
+                                   nullptr, &direct, nullptr, true);
+            if (r0 != MLKV_OK || direct)
+                return r0;
             // One multi-layer launch: a single copy of every input right before it.
             mlkv::StageParams all{};
             all.n = 3;
@@ -1608,6 +1622,15 @@ int mlkv_decode_step_host(mlkv_cache_t c, const void *Q, const void *K, const vo
         if ((e = cudaStreamIsCapturing(stream, &cap0)) != cudaSuccess)
             return fail_cuda(e, "cudaStreamIsCapturing");
         if (cap0 == cudaStreamCaptureStatusNone) {
+            // The fused form, reading the inputs where they are, issued directly.
+            bool direct = false;
+            rc = issue_step_ml(c, static_cast<const char *>(dev[0]),
+                               static_cast<const char *>(dev[1]),
+                               static_cast<const char *>(dev[2]),
+                               static_cast<char *>(const_cast<void *>(dev[3])), seq_lens, stream,
+                               nullptr, &direct, nullptr, true);
+            if (rc != MLKV_OK || direct)
+                return rc;
             // One multi-layer launch: its input copy and the launch, issued directly.
             mlkv::StageParams all{};
             all.n = 3;

@@ -120,6 +120,9 @@ struct PrefillParams {
     // cache tiles that hold no new row; 0 -- nothing.
     int fused_early;
     int fused_combine_w;   // warps per output row of combine_fused (1, 2, 4 or 8)
+    // Fused decode: non-null -- the queries [layers][b][h][D] are page-locked host memory (this is
+    // its device-mapped address): each unit loads its rows with plain loads, not the tensor map.
+    const __nv_bfloat16 *q_host;
     int prompt_len[MLKV_MAX_BATCH];
     uint32_t units[kPrefillMaxUnits];
 };

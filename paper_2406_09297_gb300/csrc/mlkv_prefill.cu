@@ -194,7 +194,9 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
     const int zv = zk + p.b * p.g;
 
     if (threadIdx.x == 0) {
-        mbar_init(bar_q, 1);
+        // the query tiles' barrier: the producer's tensor-map copy, or every softmax warp's share
+        // of the rows read from host memory
+        mbar_init(bar_q, (kFused && p.q_host != nullptr) ? PL::kSoftWarps : 1);
         for (int s = 0; s < R; ++s) {
             mbar_init(bar_full + 8 * s, 1);
             mbar_init(bar_empty + 8 * s, 1);
@@ -222,11 +224,14 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     if (kFused && warp < PL::kSoftWarps) {
-        // The tiles' rows past the TMA box (box_rows = G x min(L1, L)) are never loaded; zero them
-        // so that their (discarded) scores stay finite.  TMA writes only rows below box_rows.
+        // The tiles' rows past the loaded ones (the TMA box, G x min(L1, L) rows) are never
+        // written; zero them so that their (discarded) scores stay finite.
         const int grp = PL::kTiles == 1 ? 1 : warp >> 2, r = threadIdx.x & 127;
         const int box_rows = (p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1) * p.G;
-        if (r >= box_rows && warp < 4 * PL::kTiles) {   // one warpgroup per query tile
+        // rows the load writes: the box (tensor map), or tile A's own rows (read from host)
+        const int keep = (p.q_host != nullptr && grp == 0) ? (p.fused_L - p.fused_L1) * p.G
+                                                           : box_rows;
+        if (r >= keep && warp < 4 * PL::kTiles) {   // one warpgroup per query tile
             uint8_t *qrow = smem + PL::kQ + slot_of(grp) * PL::kTileBytes;
 #pragma unroll
             for (int c = 0; c < 8 * PL::kSub; ++c)
@@ -273,7 +278,9 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
                 grid_dependency_wait();   // the step's inputs are in place
                 waited = true;
             }
-            if (kFused) {
+            if (kFused && p.q_host != nullptr) {
+                // the softmax warps read the queries from host memory
+            } else if (kFused) {
                 // Q [layers][b][h][D] as (channel, head in group, group, sequence, layer): a box
                 // of min(L1, L) layers x G heads = the tile's rows, layer-major (row = layer*G + i),
                 // from the block's first layer (tile B) and its layer L1 (tile A).
@@ -498,6 +505,50 @@ __global__ void __launch_bounds__(PrefillPlan<D, kForm>::kThreads,
                 atomicOr(p.err, kErrWaitFull);
             }
         };
+        if (kFused && p.q_host != nullptr) {
+            // The unit's query rows from page-locked host memory through its device-mapped
+            // address (16 bytes a load, four in flight per thread), written into the query tiles
+            // the way the tensor map would have (128-byte swizzle); rows past them stay zero.
+            const int nth = 32 * PL::kSoftWarps;
+            const int L1r = p.fused_L < p.fused_L1 ? p.fused_L : p.fused_L1;
+            const int rows_b = L1r * p.G;
+            const int rows_a = n_a > 0 ? (p.fused_L - p.fused_L1) * p.G : 0;
+            constexpr int kC = D / 8;   // 16-byte chunks of a row
+            const int total = (rows_b + rows_a) * kC;
+            for (int k0 = threadIdx.x; k0 < total; k0 += 4 * nth) {
+                uint4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int k = k0 + u * nth;
+                    if (k < total) {
+                        const int rr = k / kC, c = k - rr * kC;
+                        const bool in_b = rr < rows_b;
+                        const int rw = in_b ? rr : rr - rows_b;
+                        const int lay = blk * p.fused_L + (in_b ? 0 : p.fused_L1) + rw / p.G;
+                        v[u] = *reinterpret_cast<const uint4 *>(
+                            p.q_host + ((static_cast<size_t>(lay) * p.b + beta) * p.h + j * p.G +
+                                        rw % p.G) * D + c * 8);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int k = k0 + u * nth;
+                    if (k < total) {
+                        const int rr = k / kC, c = k - rr * kC;
+                        const bool in_b = rr < rows_b;
+                        const int rw = in_b ? rr : rr - rows_b;
+                        *reinterpret_cast<uint4 *>(smem + PL::kQ +
+                                                   slot_of(in_b ? 1 : 0) * PL::kTileBytes +
+                                                   (c >> 3) * 16384 + rw * 128 +
+                                                   (((c & 7) ^ (rw & 7)) << 4)) = v[u];
+                    }
+                }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(bar_q);
+        }
         float m_run = NEG_INF, l_run = 0.f;
         for (int t = wg; t < n_g; t += kStep) {
             const int u = kSplit ? t >> 1 : t;   // this warpgroup's use of its buffers
