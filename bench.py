@@ -362,6 +362,7 @@ def run(args, w):
     step_ms = [a.elapsed_time(b) for a, b in ev]
     ms = max_over_ranks(sum(step_ms) / len(step_ms), dist, "cuda")
     value = job_value(w.b, world, ms)
+    spread = sorted(step_ms)   # the per-step times behind the mean, for the record
 
     # ---- the same step as a model runs it: one layer after another -----------------------------
     # A model computes layer n's queries from layer n-1's output, so its attention for layer n
@@ -481,7 +482,9 @@ def run(args, w):
     if rank == 0:
         result = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": ms,
+            "step_ms": {"min": spread[0], "median": spread[len(spread) // 2], "max": spread[-1]},
+            "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": _config_dict(w),
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms},
@@ -847,8 +850,8 @@ def run_fused(args, w):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--config", default=DEFAULT_WORKLOAD)
     ap.add_argument("--tile", type=int, default=0)

@@ -1003,6 +1003,17 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
         has_map = has_map || v.v->tile_tokens == 128;
     if (!has_map)
         return MLKV_OK;
+    if (host_inputs) {
+        // Inputs read in place only when no sequence is split: every chunk of a split sequence
+        // would read its query rows over the CPU-GPU link again (measured at batch 1 x 131072
+        // positions, MLKV-1: 47.7 us end to end against 36.9 on the device); the caller copies
+        // them in instead.
+        int n_kt_max = 0;
+        for (int beta = 0; beta < c->b; ++beta)
+            n_kt_max = std::max(n_kt_max, (seq_lens[beta] + 127) / 128);
+        if (fused_plan(c, seq_lens, c->m, nullptr) < n_kt_max)
+            return MLKV_OK;
+    }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaSuccess;
     DeviceGuard guard(c->device);
