@@ -61,6 +61,11 @@ def test_recorded_traffic_needs_current_kernel_and_launch_kind():
     for entry in rec["entries"]:
         assert entry["launch"] in forms
         assert entry["dram_bytes_per_launch"] > 0
+        # the summary the figure comes from states it and the sources it was taken on
+        with open(os.path.join(ROOT, entry["source"])) as f:
+            summary = f.read()
+        assert f"{entry['dram_bytes_per_launch']:,}" in summary, entry["source"]
+        assert entry["kernel_source_sha256_16"] in summary, entry["source"]
         w = workloads.by_name(entry["workload"])
         current = entry["kernel_source_sha256_16"] == bench._kernel_source_hash(entry["kernel"])
         got = bench._recorded_traffic(w, entry["kernel"], entry["launch"])
