@@ -969,7 +969,8 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
         // launch.  A block of one layer shares nothing across layers (MHA, GQA-4, MQA at batch
         // 256 and 1: 7-16% slower fused); blocks of two saved little or lost (batch 64 x 2000
         // positions 49 vs 53 us, batch 256 x 8192 535 vs 548, batch 1 x 131072 66 vs 62, batch
-        // 1 x 128 11.6 vs 10.3).  For blocks of >= 3 layers the estimates in us per step, from the
+        // 1 x 128 11.6 vs 10.3; with the split-key CTA form 53.2 vs 52.6, 548.9 vs 548.0, 60.3
+        // vs 59.3, 12.5 vs 10.7).  For blocks of >= 3 layers the estimates in us per step, from the
         // same measurements: the fused form ~1.1 per key tile its busiest SM takes plus ~6 fixed
         // (+3 for the merge of a split); the decode kernel ~0.55 per (layer, sequence, KV head,
         // 128 positions) item per SM plus ~3.  They pick the measured winner at batch 8, 64, 128
