@@ -160,6 +160,31 @@ int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V
                      const int *seq_lens, void *cuda_stream);
 
 /*
+ * mlkv_plan_step - the form mlkv_decode_step takes for a map and a step's lengths, decided on the
+ * host with no GPU and no cache: the same decision a cache of this map makes on a device with
+ * sm_count SMs (152 on GB300), with its options "step_fused", "fused_kc" and "fused_deep" at the
+ * given values (-1: the default) and every other option at its default, for device buffers.
+ *
+ * Paper: Sec. 3, Eq. 18 (the equal contiguous owner blocks the fused form requires).
+ *
+ *   layer_owner .. max_seq  as for mlkv_cache_create (same validation and error codes)
+ *   seq_lens    host int32[batch], as for mlkv_decode_step (each in [1, max_seq])
+ *   plan        host int64[4], written on success:
+ *               [0] 1 if the step runs in the cross-layer fused form, else 0 (the decode kernel);
+ *               [1] the fused launch's CTA form: 0 two 128-row query tiles per CTA, 1 one tile at
+ *                   two CTAs per SM, 2 one tile at one CTA per SM with the key tiles alternating
+ *                   between two softmax warpgroups; -1 when not fused;
+ *               [2] key tiles of 128 positions per unit (the context split; 0 when not fused);
+ *               [3] units of the fused launch (sequence, KV head, owner block, chunk), 0 when not
+ *                   fused.
+ * Errors: MLKV_ERR_INVALID_ARG (NULL plan, sm_count < 1, an option out of range), and those of
+ * mlkv_cache_create and of the lengths' check.
+ */
+int mlkv_plan_step(int n_layers, int n_q_heads, int head_dim, const int *layer_owner,
+                   int kv_heads_per_owner, int batch, int max_seq, const int *seq_lens,
+                   int sm_count, int step_fused, int fused_kc, int fused_deep, int64_t plan[4]);
+
+/*
  * mlkv_decode_step_host - mlkv_decode_step with the step's tensors in host memory (the user's end
  * of a step).  Layouts as for mlkv_decode_step, in host memory; everything is queued on
  * cuda_stream, and out holds the step's outputs once the stream has reached the end of the call's

@@ -242,6 +242,30 @@ void free_all(mlkv_cache *c)
     c->err = nullptr;
 }
 
+// The owner map's shape in c: sizes, owners, and each layer's slot (the rank of its owner among
+// the distinct owners, Eq. 18's k); c->m the number of slots.
+void assign_map(mlkv_cache *c, int l, int h, int d, const int *owner, int g, int b, int max_seq)
+{
+    c->l = l;
+    c->h = h;
+    c->d = d;
+    c->g = g;
+    c->G = h / g;
+    c->b = b;
+    c->max_seq = max_seq;
+    c->owner.assign(owner, owner + l);
+    c->slot.assign(l, -1);
+    c->m = 0;
+    for (int n = 0; n < l; ++n) {
+        if (c->owner[n] == n) {
+            for (int q = 0; q < l; ++q)
+                if (c->owner[q] == n)
+                    c->slot[q] = c->m;
+            ++c->m;
+        }
+    }
+}
+
 int validate_map(int l, int h, int d, const int *owner, int g, int b, int max_seq)
 {
     if (l < 1 || h < 1 || g < 1 || b < 1 || max_seq < 1 || d < 1)
@@ -304,23 +328,7 @@ int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_d
         return rc;
 
     mlkv_cache *c = new mlkv_cache();
-    c->l = n_layers;
-    c->h = n_q_heads;
-    c->d = head_dim;
-    c->g = kv_heads_per_owner;
-    c->G = n_q_heads / kv_heads_per_owner;
-    c->b = batch;
-    c->max_seq = max_seq;
-    c->owner.assign(layer_owner, layer_owner + n_layers);
-    c->slot.assign(n_layers, -1);
-    for (int n = 0; n < n_layers; ++n) {
-        if (c->owner[n] == n) {
-            for (int q = 0; q < n_layers; ++q)
-                if (c->owner[q] == n)
-                    c->slot[q] = c->m;
-            ++c->m;
-        }
-    }
+    assign_map(c, n_layers, n_q_heads, head_dim, layer_owner, kv_heads_per_owner, batch, max_seq);
     const long long rows = static_cast<long long>(c->m) * 2 * c->b * c->g;
     if (rows > 0x7fffffffLL) {
         delete c;
@@ -735,16 +743,6 @@ int mlkv_append_decode_attention(mlkv_cache_t c, int layer, const void *K, const
     return decode_impl(c, layer, nullptr, nullptr, Q, out, seq_lens, cuda_stream);
 }
 
-// The whole decode step as one launch of the decode kernel over every (layer, segment) item
-// (DecodeParams::ml_layers), where that applies: every sequence has one length, the mma.sync
-// kernel, default grid, no L2-persistence windows (they are per layer), at most kMaxStepLayers
-// layers, and a makespan no longer than the
-// per-layer launches' (below).  Items are whole segments, so nothing is merged and no
-// scratch is shared; every layer takes its segments' newest rows from the step's new tokens,
-// and owner layers store them.  *done tells whether it was issued.  With in_ready, the launch
-// waits for it (queries still arriving).
-// With `stage`, the copy of the step's inputs it describes is launched right before the step's
-// kernel, which may then start (and fetch its first cache tiles) while the copy runs.
 // The fused decode's context split for nblk blocks: kc key tiles of 128 positions a unit; *units
 // (if given) the units it makes.  Measured on GB300 (batch 64 x 2048 positions, 72 rows a unit):
 // one CTA keeps an SM's softmax and tensor core about as busy as two do, while every unit costs
@@ -792,6 +790,18 @@ static int fused_plan(const mlkv_cache *c, const int *seq_lens, int nblk, long l
     return kc;
 }
 
+// The fused decode's CTA form for blocks of L layers and n_units units: one query tile when the
+// block's rows fit one (head_dim 64); then with at most one unit per SM one CTA per SM with a deep
+// ring and two S buffers (its tiles come from HBM one after another), else two CTAs per SM.  Rows
+// past one tile: two query tiles.
+static int fused_cta_form(const mlkv_cache *c, int L, long long n_units)
+{
+    const bool one = c->d == 64 && L <= 128 / c->G;
+    if (!one)
+        return mlkv::kFusedTwoTiles;
+    return n_units <= c->sm_count && c->fused_deep ? mlkv::kFusedOneDeep : mlkv::kFusedOneTile;
+}
+
 // The cross-layer fused decode (the fused form of prefill_kernel) over nblk owner blocks of L
 // layers each: block k reads slot slot0 + k and attends for the layers k*L .. k*L + L - 1 of Q and
 // out ([n_q_layers][b][h][d]).  A unit (sequence, KV head, block, chunk of the context) loads each
@@ -803,15 +813,9 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
                        int after_store = 0, bool q_in_host = false)
 {
     const int L1 = 128 / c->G;
-    // The CTA form: one query tile when the block's rows fit one (head_dim 64); then with at most
-    // one unit per SM one CTA per SM with a deep ring and two S buffers (its tiles come from HBM
-    // one after another), else two CTAs per SM.  Rows past one tile: two query tiles.
     long long n_units = 0;
     const int kc = fused_plan(c, seq_lens, nblk, &n_units);
-    const bool one = c->d == 64 && L <= L1;
-    const int form = !one ? mlkv::kFusedTwoTiles
-                          : (n_units <= c->sm_count && c->fused_deep ? mlkv::kFusedOneDeep
-                                                                     : mlkv::kFusedOneTile);
+    const int form = fused_cta_form(c, L, n_units);
     cudaError_t e;
     if (!(c->fused_ready & (1 << form))) {
         if ((e = mlkv::prepare_fused(c->d, form)) != cudaSuccess)
@@ -945,25 +949,23 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
     return MLKV_OK;
 }
 
-// mlkv_decode_step in the cross-layer fused form: one append launch for every owner's new token,
-// then the fused decode of every block in one launch (and one merge).  Applies to maps of equal
+// Whether mlkv_decode_step takes the cross-layer fused form for these lengths: maps of equal
 // contiguous blocks (owner[n] = n - n mod L, the paper's Eq. 18 layout) whose L*G query rows fit
-// two 128-row tiles; otherwise *done stays false.
-static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
-                            const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
-                            const mlkv::StageParams *stage, bool host_inputs = false)
+// two 128-row tiles, under the options (step_fused; no tile length or L2 prefetch forced), and
+// with step_fused = 1 where the estimates below favour it.  host_inputs: the step's buffers are
+// page-locked host memory read in place.
+static bool fused_step_applies(const mlkv_cache *c, const int *seq_lens, bool host_inputs)
 {
-    *done = false;
     if (!c->step_fused || c->tile_tokens > 0 || c->l2_prefetch || c->m > mlkv::kFusedMaxBlocks ||
         c->g > 255 || c->h > mlkv::kPrefillMaxHeads || (c->d != 64 && c->d != 128))
-        return MLKV_OK;
+        return false;
     const int L = c->l / c->m;
     const int L1 = 128 / c->G;
     if (L * c->m != c->l || L1 < 1 || L > 2 * L1)
-        return MLKV_OK;
+        return false;
     for (int n = 0; n < c->l; ++n)
         if (c->owner[n] != n - n % L || c->slot[n] != n / L)
-            return MLKV_OK;
+            return false;
     if (c->step_fused == 1) {
         // Where the fused form pays, from measurements on GB300 against the decode kernel's
         // launch.  A block of one layer shares nothing across layers (MHA, GQA-4, MQA at batch
@@ -976,7 +978,7 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
         // 128 positions) item per SM plus ~3.  They pick the measured winner at batch 8, 64, 128
         // and 256, batch 1 x 131072 and Llama-2-7B shapes.
         if (L < 3)
-            return MLKV_OK;
+            return false;
         long long units = 0;
         const int kc = fused_plan(c, seq_lens, c->m, &units);
         long long tiles = 0;
@@ -997,13 +999,8 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
             1.1 * static_cast<double>(busiest) + 6.0 + (kc < n_kt_max ? 3.0 : 0.0);
         const double ml_us = 0.55 * static_cast<double>(tiles) * c->l * c->g / c->sm_count + 3.0;
         if (fused_us >= ml_us)
-            return MLKV_OK;
+            return false;
     }
-    bool has_map = false;   // the cache's tensor map of 128-position tiles
-    for (auto &v : c->variants)
-        has_map = has_map || v.v->tile_tokens == 128;
-    if (!has_map)
-        return MLKV_OK;
     if (host_inputs) {
         // Inputs read in place only when no sequence is split: every chunk of a split sequence
         // would read its query rows over the CPU-GPU link again (measured at batch 1 x 131072
@@ -1013,8 +1010,27 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
         for (int beta = 0; beta < c->b; ++beta)
             n_kt_max = std::max(n_kt_max, (seq_lens[beta] + 127) / 128);
         if (fused_plan(c, seq_lens, c->m, nullptr) < n_kt_max)
-            return MLKV_OK;
+            return false;
     }
+    return true;
+}
+
+// mlkv_decode_step in the cross-layer fused form, where fused_step_applies: one append launch for
+// every owner's new token, then the fused decode of every block in one launch (and one merge);
+// otherwise *done stays false.
+static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
+                            const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
+                            const mlkv::StageParams *stage, bool host_inputs = false)
+{
+    *done = false;
+    if (!fused_step_applies(c, seq_lens, host_inputs))
+        return MLKV_OK;
+    bool has_map = false;   // the cache's tensor map of 128-position tiles
+    for (auto &v : c->variants)
+        has_map = has_map || v.v->tile_tokens == 128;
+    if (!has_map)
+        return MLKV_OK;
+    const int L = c->l / c->m;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaSuccess;
     DeviceGuard guard(c->device);
@@ -1062,6 +1078,24 @@ static int issue_step_fused(mlkv_cache_t c, const char *Q, const char *K, const 
     return MLKV_OK;
 }
 
+// The options under which mlkv_decode_step may issue a step as one launch (the decode kernel's
+// multi-layer launch or the fused form): the mma.sync kernel, default grid, no L2-persistence
+// windows (they are per layer), at most kMaxStepLayers layers.
+static bool step_launch_allowed(const mlkv_cache *c)
+{
+    return c->step_kernel && !c->tc && c->grid <= 0 && !c->l2_persist &&
+           c->l <= mlkv::kMaxStepLayers;
+}
+
+// The whole decode step in one launch: the cross-layer fused form where it applies
+// (issue_step_fused), else one launch of the decode kernel over every (layer, segment) item
+// (DecodeParams::ml_layers) where that applies: every sequence has one length and the makespan is
+// no longer than the per-layer launches' (below).  Items are whole segments, so nothing is merged
+// and no scratch is shared; every layer takes its segments' newest rows from the step's new
+// tokens, and owner layers store them.  *done tells whether it was issued.  With in_ready, the
+// launch waits for it (queries still arriving).  With `stage`, the copy of the step's inputs it
+// describes is launched right before the step's kernel, which may then start (and fetch its first
+// cache tiles) while the copy runs.
 static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const char *V, char *out,
                          const int *seq_lens, void *stream, cudaEvent_t in_ready, bool *done,
                          const mlkv::StageParams *stage = nullptr, bool host_inputs = false)
@@ -1070,7 +1104,7 @@ static int issue_step_ml(mlkv_cache_t c, const char *Q, const char *K, const cha
     c->last_step_kernel = 0;
     c->last_step_fused = 0;
     c->last_step_launches = 0;
-    if (!c->step_kernel || c->tc || c->grid > 0 || c->l2_persist || c->l > mlkv::kMaxStepLayers)
+    if (!step_launch_allowed(c))
         return MLKV_OK;
     {
         const int rc =
@@ -1456,6 +1490,48 @@ int record_or_replay(mlkv_cache *c, const mlkv_cache::StepKey &key, mlkv_cache::
 }  // namespace
 
 extern "C" {
+
+int mlkv_plan_step(int n_layers, int n_q_heads, int head_dim, const int *layer_owner,
+                   int kv_heads_per_owner, int batch, int max_seq, const int *seq_lens,
+                   int sm_count, int step_fused, int fused_kc, int fused_deep, int64_t plan[4])
+{
+    if (plan == nullptr)
+        return fail(MLKV_ERR_INVALID_ARG, "plan is NULL");
+    int rc = validate_map(n_layers, n_q_heads, head_dim, layer_owner, kv_heads_per_owner, batch,
+                          max_seq);
+    if (rc != MLKV_OK)
+        return rc;
+    if (sm_count < 1)
+        return fail(MLKV_ERR_INVALID_ARG, "sm_count %d must be positive", sm_count);
+    if (step_fused > 2 || fused_deep > 1 || fused_kc > (1 << 20))
+        return fail(MLKV_ERR_INVALID_ARG, "step_fused %d, fused_kc %d or fused_deep %d out of range",
+                    step_fused, fused_kc, fused_deep);
+    // The decision of mlkv_decode_step, on a cache description that holds nothing on a device.
+    mlkv_cache c;
+    assign_map(&c, n_layers, n_q_heads, head_dim, layer_owner, kv_heads_per_owner, batch, max_seq);
+    c.sm_count = sm_count;
+    if (step_fused >= 0)
+        c.step_fused = step_fused;
+    if (fused_kc >= 0)
+        c.fused_kc = fused_kc;
+    if (fused_deep >= 0)
+        c.fused_deep = fused_deep;
+    if ((rc = check_seq_lens(&c, seq_lens)) != MLKV_OK)
+        return rc;
+    plan[0] = 0;
+    plan[1] = -1;
+    plan[2] = 0;
+    plan[3] = 0;
+    if (step_launch_allowed(&c) && fused_step_applies(&c, seq_lens, false)) {
+        long long units = 0;
+        const int kc = fused_plan(&c, seq_lens, c.m, &units);
+        plan[0] = 1;
+        plan[1] = fused_cta_form(&c, c.l / c.m, units);
+        plan[2] = kc;
+        plan[3] = units;
+    }
+    return MLKV_OK;
+}
 
 int mlkv_decode_step(mlkv_cache_t c, const void *Q, const void *K, const void *V, void *out,
                      const int *seq_lens, void *cuda_stream)

@@ -31,7 +31,7 @@ EXPORTED = [
     "mlkv_set_option", "mlkv_get_option", "mlkv_sync_status", "mlkv_last_error",
     "mlkv_block_owner_map", "mlkv_version", "mlkv_decode_attention_static", "mlkv_prefill",
     "mlkv_merge_kv_weights", "mlkv_decode_block_fused", "mlkv_decode_step_host",
-    "mlkv_static_status", "mlkv_read_bandwidth_probe",
+    "mlkv_static_status", "mlkv_read_bandwidth_probe", "mlkv_plan_step",
 ]
 
 
@@ -75,6 +75,8 @@ def _load():
     L.mlkv_prefill.argtypes = [vp, ci, vp, vp, vp, vp, ip, ci, vp]
     L.mlkv_merge_kv_weights.argtypes = [ip, ci, ci, ci, i64, vp, vp, vp]
     L.mlkv_decode_block_fused.argtypes = [vp, ci, vp, vp, ip, vp]
+    L.mlkv_plan_step.argtypes = [ci, ci, ci, ip, ci, ci, ci, ip, ci, ci, ci, ci,
+                                 ctypes.POINTER(i64)]
     return L
 
 
@@ -216,6 +218,21 @@ def mlkv_block_owner_map(n_layers, n_owners):
 
 def mlkv_version():
     return lib.mlkv_version()
+
+
+def mlkv_plan_step(layer_owner, n_q_heads, head_dim, kv_heads_per_owner, seq_lens, max_seq,
+                   sm_count, step_fused=-1, fused_kc=-1, fused_deep=-1):
+    """The form mlkv_decode_step takes (no GPU needed): dict of fused (0/1), form (-1, 0, 1, 2),
+    kc (key tiles of 128 positions per unit) and units of the fused launch."""
+    owner = np.ascontiguousarray(np.asarray(layer_owner, dtype=np.int32))
+    a, p = _lens_ptr(seq_lens)
+    plan = (ctypes.c_int64 * 4)()
+    _check(lib.mlkv_plan_step(len(owner), n_q_heads, head_dim,
+                              owner.ctypes.data_as(ctypes.POINTER(ctypes.c_int)),
+                              kv_heads_per_owner, len(a), max_seq, p, sm_count, step_fused,
+                              fused_kc, fused_deep, plan))
+    return {"fused": int(plan[0]), "form": int(plan[1]), "kc": int(plan[2]),
+            "units": int(plan[3])}
 
 
 def mlkv_decode_attention_static(kv_slot, batch, n_q_heads, kv_heads, head_dim, max_seq, Q, out,

@@ -12,6 +12,28 @@ from mlkv_synth import gen
 MAX_ABS = 2e-2
 MEAN_ABS = 2e-3
 
+# The decode step in the cross-layer fused form (option step_fused 2) on a device of 152 SMs:
+# layout, the plan's key tiles of 128 positions per unit (kc) and units, and the query tiles of a
+# unit (1: the block's L x G rows fit one tile at head_dim 64; 2: two tiles).
+FUSED_STEP_SMS = 152
+FUSED_STEP_CASES = [
+    # owner, h, g, d, b, L, kc, units, tiles
+    ([0] * 6 + [6] * 6, 12, 1, 64, 64, 2048, 16, 128, 1),  # the benchmark's shape: 72 rows a unit
+    ([0, 0, 2, 2, 4, 4, 6, 6, 8, 8, 10, 10], 12, 1, 64, 1, 128, 1, 6, 1),   # one tile per block
+    ([0] * 12, 12, 1, 64, 4, 3000, 1, 96, 2),              # 144 rows: query tiles A and B
+    ([0, 0, 2, 2], 12, 1, 64, 40, 700, 6, 80, 1),           # ragged last tile
+    ([0, 0, 2, 2], 4, 4, 64, 8, 333, 2, 128, 1),            # one head per KV head: two rows a unit
+    ([0, 0, 0, 3, 3, 3], 12, 4, 64, 16, 1000, 8, 128, 1),   # GQA groups of 3 under MLKV: 9 rows
+    ([0, 0, 2, 2], 32, 8, 128, 8, 1500, 12, 128, 2),        # head_dim 128, groups of 4: 8 rows
+    ([0] * 20, 16, 2, 128, 2, 600, 1, 20, 2),               # head_dim 128, 160 rows in two tiles
+    ([0, 0, 0], 16, 2, 64, 3, 1, 1, 6, 1),                  # a single position
+    # few long segments: every segment in chunks, partial records, one merge launch
+    ([0] * 6 + [6] * 6, 12, 1, 64, 1, 131072, 14, 148, 1),  # 74 chunks of 14 tiles a segment
+    ([0, 0, 2, 2], 12, 4, 64, 2, 9000, 8, 144, 1),          # ragged last tile in the last chunk
+    ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 27, 144, 2),       # head_dim 128
+    ([0, 1, 2, 3], 12, 1, 64, 3, 5000, 4, 120, 1),          # blocks of one layer (forced)
+]
+
 
 def to_dev(bits):
     import torch

@@ -5,7 +5,8 @@ import pytest
 
 import oracle
 from mlkv_synth import gen
-from tests.mlkv_cases import MAX_ABS, MEAN_ABS, errors, from_dev, to_dev
+from tests.mlkv_cases import (FUSED_STEP_CASES, FUSED_STEP_SMS, MAX_ABS, MEAN_ABS, errors,
+                              from_dev, to_dev)
 
 pytestmark = pytest.mark.gpu
 
@@ -393,24 +394,9 @@ def test_multi_layer_step_varied_lengths(owner, h, g, d, lens, fused):
         cache.sync_status()
 
 
-@pytest.mark.parametrize("owner,h,g,d,b,L,kc,units", [
-    ([0] * 6 + [6] * 6, 12, 1, 64, 64, 2048, 16, 128),  # the benchmark's shape: 72 rows a unit
-    ([0, 0, 2, 2, 4, 4, 6, 6, 8, 8, 10, 10], 12, 1, 64, 1, 128, 1, 6),   # one tile per block
-    ([0] * 12, 12, 1, 64, 4, 3000, 1, 96),              # 144 rows: query tiles A and B
-    ([0, 0, 2, 2], 12, 1, 64, 40, 700, 6, 80),           # ragged last tile
-    ([0, 0, 2, 2], 4, 4, 64, 8, 333, 2, 128),            # one head per KV head: two rows a unit
-    ([0, 0, 0, 3, 3, 3], 12, 4, 64, 16, 1000, 8, 128),   # GQA groups of 3 under MLKV: 9 rows
-    ([0, 0, 2, 2], 32, 8, 128, 8, 1500, 12, 128),        # head_dim 128, groups of 4: 8 rows
-    ([0] * 20, 16, 2, 128, 2, 600, 1, 20),               # head_dim 128, 160 rows in two tiles
-    ([0, 0, 0], 16, 2, 64, 3, 1, 1, 6),                  # a single position
-    # few long segments: every segment in chunks, partial records, one merge launch
-    ([0] * 6 + [6] * 6, 12, 1, 64, 1, 131072, 14, 148),  # 74 chunks of 14 tiles a segment
-    ([0, 0, 2, 2], 12, 4, 64, 2, 9000, 8, 144),          # ragged last tile in the last chunk
-    ([0, 0, 2, 2], 32, 8, 128, 1, 30000, 27, 144),       # head_dim 128
-    ([0, 1, 2, 3], 12, 1, 64, 3, 5000, 4, 120),          # blocks of one layer (forced)
-])
+@pytest.mark.parametrize("owner,h,g,d,b,L,kc,units,tiles", FUSED_STEP_CASES)
 @pytest.mark.parametrize("deep", [1, 0])
-def test_fused_step(owner, h, g, d, b, L, kc, units, deep):
+def test_fused_step(owner, h, g, d, b, L, kc, units, tiles, deep):
     # The step in the cross-layer fused form (forced: option step_fused 2): one launch storing
     # every owner's new token, then units of (sequence, KV head, owner block, chunk of the
     # context), each loading every K/V tile of its chunk once for the L * G query rows of its
@@ -433,6 +419,14 @@ def test_fused_step(owner, h, g, d, b, L, kc, units, deep):
         # head_dim 64 with the block's rows in one tile: one CTA per SM with a 12-tile ring and two
         # S buffers when the units fit one per SM (deep), else two CTAs per SM
         cache.set_option("fused_deep", deep)
+        # the host planner's decision for this device (the table holds the one for 152 SMs)
+        sms = cache.get_option("sm_count")
+        plan = mlkv.mlkv_plan_step(owner, h, d, g, lens, L, sms, step_fused=2, fused_deep=deep)
+        if sms == FUSED_STEP_SMS:
+            assert (plan["kc"], plan["units"]) == (kc, units)
+        kc, units = plan["kc"], plan["units"]
+        assert plan["fused"] == 1 and plan["form"] == (0 if tiles == 2 else 2 if deep and
+                                                       units <= sms else 1)
         results = []
         for rep in range(3):
             out.fill_(float("nan"))
