@@ -870,16 +870,12 @@ static int fused_issue(mlkv_cache_t c, const void *Q, void *out, int n_q_layers,
     // queries in page-locked host memory (Q is its device-mapped address): read row by row
     p.q_host = q_in_host ? static_cast<const __nv_bfloat16 *>(Q) : nullptr;
     int n_kt_max = 0;
-    long long kt_sum = 0;
     bool uniform = true;
     for (int beta = 0; beta < c->b; ++beta) {
         p.prompt_len[beta] = seq_lens[beta];
-        const int nkt = (seq_lens[beta] + 127) / 128;
-        n_kt_max = std::max(n_kt_max, nkt);
-        kt_sum += nkt;
+        n_kt_max = std::max(n_kt_max, (seq_lens[beta] + 127) / 128);
         uniform = uniform && seq_lens[beta] == seq_lens[0];
     }
-    (void)kt_sum;
     const int cmax = (n_kt_max + kc - 1) / kc;
     p.fused_kc = kc;
     p.fused_cmax = cmax;
