@@ -365,7 +365,7 @@ int mlkv_cache_create(mlkv_cache_t *out, int n_layers, int n_q_heads, int head_d
                                                           v->smem_bytes);
         if (e != cudaSuccess || var.ctas_per_sm < 1) {
             delete c;
-            return fail(MLKV_ERR_CUDA, "decode variant d=%d T=%d cannot be resident", c->d, T);
+            return fail(MLKV_ERR_CUDA, "decode variant d=%d T=%d cannot be resident", head_dim, T);
         }
         c->max_ctas = std::max(c->max_ctas, var.ctas_per_sm * c->sm_count);
         for (int k : {2, 4}) {
