@@ -1499,7 +1499,8 @@ int mlkv_plan_step(int n_layers, int n_q_heads, int head_dim, const int *layer_o
         return rc;
     if (sm_count < 1)
         return fail(MLKV_ERR_INVALID_ARG, "sm_count %d must be positive", sm_count);
-    if (step_fused > 2 || fused_deep > 1 || fused_kc > (1 << 20))
+    if (step_fused < -1 || step_fused > 2 || fused_deep < -1 || fused_deep > 1 || fused_kc < -1 ||
+        fused_kc > (1 << 20))
         return fail(MLKV_ERR_INVALID_ARG, "step_fused %d, fused_kc %d or fused_deep %d out of range",
                     step_fused, fused_kc, fused_deep);
     // The decision of mlkv_decode_step, on a cache description that holds nothing on a device.

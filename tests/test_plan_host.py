@@ -140,6 +140,8 @@ def test_planner_rejects_bad_arguments():
                       (dict(seq_lens=[0, 5]), mlkv.MLKV_ERR_RANGE),
                       (dict(sm_count=0), mlkv.MLKV_ERR_INVALID_ARG),
                       (dict(step_fused=3), mlkv.MLKV_ERR_INVALID_ARG),
+                      (dict(step_fused=-2), mlkv.MLKV_ERR_INVALID_ARG),
+                      (dict(fused_kc=-2), mlkv.MLKV_ERR_INVALID_ARG),
                       (dict(fused_deep=2), mlkv.MLKV_ERR_INVALID_ARG)]:
         with pytest.raises(mlkv.MLKVError) as e:
             mlkv.mlkv_plan_step(**{**ok, **bad})
